@@ -1,0 +1,184 @@
+/*
+ * cofie_ngff.h -- C ABI of libcofie_ngff.so, a GB300 (sm_103a) implementation
+ * of Novelty-Guided Frame Filtering (NGFF), the coarse, pre-encoder stage of
+ * CoFiE (Sec. 3.2, Eqs. 2-5; hyperparameters from App. A and App. B.2).
+ *
+ * What the library computes for every frame I_t of a stream, in order:
+ *   1. grayscale Y of every pixel: ITU-R BT.601 luma with integer weights,
+ *      Y = floor((wR R + wG G + wB B + floor(den/2)) / den), default
+ *      (299, 587, 114) / 1000 (the paper names no conversion; Sec. 3.2);
+ *   2. the B-bin histogram h_t over the intensity range, bin = floor(Y B / 256),
+ *      kept as integer counts c_t (h_t = c_t / N, N = W H; Sec. 3.2, App. A);
+ *   3. the total-variation distances (Eq. 2) to the previous frame, s_adj,
+ *      and to the most recent retained frame r(t), s_ref (Eq. 3), and the
+ *      novelty score s = max(s_adj, s_ref) (Eq. 4), each distance evaluated
+ *      in fp32 as sum_b |c_i[b] - c_j[b]| / (2N) (one IEEE division);
+ *   4. the retention decision (Eq. 5 and the first-frame safeguard): the
+ *      stream's first frame is kept; frame t > 0 is kept when s >= tau_h or
+ *      t - r(t) >= L_max.
+ * Decisions are causal and final when a push completes; the closing
+ * safeguards of Sec. 3.2 that need the end of the prefix (the last frame, the
+ * M_min uniform fill) are applied by cofie_ngff_candidates.
+ *
+ * Conventions for every entry point:
+ *   - All calls are asynchronous on `cuda_stream` (a cudaStream_t passed as
+ *     void*; NULL means the legacy default stream) unless stated otherwise.
+ *     Buffers passed in must stay valid until that stream has passed the call.
+ *   - Frame data is uint8 RGB, height x width x 3 (HWC), frames back to back
+ *     (3 W H bytes per frame), in device memory or in host memory (pinned
+ *     host memory is copied asynchronously; pageable host memory works but
+ *     the copy is synchronous with the host).
+ *   - Output buffers may be device or host memory; the library detects which.
+ *   - A nonzero return is an error code below; on error nothing was enqueued
+ *     and no stream state changed, and cofie_ngff_last_error() describes it.
+ *   - A handle is not thread-safe: calls on one handle must be serialised.
+ *   - Nothing aborts, traps or prints. Device-side waits are bounded; a wait
+ *     that runs out sets an error word that cofie_ngff_status() reports.
+ */
+#ifndef COFIE_NGFF_H
+#define COFIE_NGFF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define COFIE_NGFF_ABI_VERSION 1
+
+/* Return codes. */
+#define COFIE_OK 0
+#define COFIE_EINVAL 1   /* bad argument: null pointer, size, stream index, parameter */
+#define COFIE_ENOMEM 2   /* a device or pinned-host allocation failed */
+#define COFIE_ECUDA 3    /* a CUDA runtime call failed */
+#define COFIE_ETIMEOUT 4 /* a device-side bounded wait ran out (cofie_ngff_status) */
+
+/* Keep codes written to keep_out. Nonzero means retained (a candidate). */
+#define COFIE_KEEP_DROP 0
+#define COFIE_KEEP_NOVELTY 1 /* s >= tau_h (Eq. 5, first term) */
+#define COFIE_KEEP_GAP 2     /* t - r(t) >= L_max and not novelty (Eq. 5, second term) */
+#define COFIE_KEEP_FIRST 3   /* the stream's first frame (Sec. 3.2 safeguard) */
+
+/* Limits. */
+#define COFIE_NGFF_MAX_BINS 256
+#define COFIE_NGFF_MAX_LMAX 256
+#define COFIE_NGFF_MAX_BATCH 64 /* descriptors per cofie_ngff_push_batch call */
+
+typedef struct cofie_ngff cofie_ngff_t;
+
+/*
+ * Parameters of a handle. Fill with cofie_ngff_default_params() and override.
+ *   width, height     frame size in pixels, >= 1 each.
+ *   bins              B, 1..256; default 32 (App. A).
+ *   l_max             L_max in sampled-frame indices, 1..256; default 30 (App. B.2).
+ *   m_min             M_min, used by cofie_ngff_candidates only; default 4 (App. B.2).
+ *   tau               tau_h, any non-NaN float; default 0.30f (App. B.2).
+ *   luma_w, luma_den  grayscale weights (wR, wG, wB) / den; each weight <= 65535,
+ *                     wR + wG + wB == den; default (299, 587, 114) / 1000.
+ *   max_streams       number of independent streams the handle holds, >= 1.
+ *   max_frames_per_push
+ *                     sizes the device scratch; larger pushes are processed in
+ *                     pieces of this many frames (results are identical).
+ *   device            CUDA device ordinal, or -1 for the calling thread's current device.
+ *   host_stage_bytes  size of each of the two device staging buffers used when
+ *                     frames come from host memory; 0 picks 256 MiB (at least one frame).
+ */
+typedef struct {
+  uint32_t width, height;
+  uint32_t bins;
+  uint32_t l_max;
+  uint32_t m_min;
+  float tau;
+  uint32_t luma_w[3];
+  uint32_t luma_den;
+  uint32_t max_streams;
+  uint32_t max_frames_per_push;
+  int32_t device;
+  uint64_t host_stage_bytes;
+} cofie_ngff_params;
+
+/* One stream's frames in a batched push (see cofie_ngff_push_batch). */
+typedef struct {
+  uint32_t stream;        /* stream index, < max_streams; distinct within one batch */
+  uint32_t n;             /* number of frames, may be 0 */
+  const uint8_t* frames;  /* n frames, device memory, 16-byte aligned */
+  float* scores_out;      /* n floats, device memory, or NULL */
+  uint8_t* keep_out;      /* n keep codes, device memory, or NULL */
+} cofie_ngff_push_desc;
+
+/* Fills *p with the paper's defaults for a width x height stream. */
+void cofie_ngff_default_params(cofie_ngff_params* p, uint32_t width, uint32_t height);
+
+/*
+ * Creates a handle: validates *p and allocates the device state of
+ * max_streams streams (a ring of the last L_max histograms each) and the
+ * scratch for max_frames_per_push frames. Synchronous. On success *out owns
+ * the allocations until cofie_ngff_destroy. Errors: COFIE_EINVAL (bad
+ * parameter; *out untouched), COFIE_ENOMEM, COFIE_ECUDA.
+ */
+int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out);
+
+/* Frees everything the handle owns (after synchronising its device). NULL is a no-op. */
+void cofie_ngff_destroy(cofie_ngff_t* h);
+
+/*
+ * Pushes n new frames of stream `stream` (Sec. 3.2: the next frames of the
+ * sampled prefix V_{1:T}) and decides each one.
+ *   frames      n frames (3 W H bytes each), device or host memory.
+ *   scores_out  n floats or NULL: s = max(s_adj, s_ref) per frame (Eq. 4);
+ *               0 for the stream's first frame.
+ *   keep_out    n bytes or NULL: keep code per frame (COFIE_KEEP_*).
+ * n == 0 is a no-op. Splitting a stream into pushes of any sizes gives the
+ * same results as one push. Errors: COFIE_EINVAL (null handle or frames with
+ * n > 0, stream out of range), COFIE_ECUDA.
+ */
+int cofie_ngff_push(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n,
+                    float* scores_out, uint8_t* keep_out, void* cuda_stream);
+
+/*
+ * cofie_ngff_push, and also writes the integer histograms c_t of the n frames
+ * to hist_out (n * bins uint32, row-major, device or host memory; NULL skips).
+ * sum_b c_t[b] = W H for every frame.
+ */
+int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n,
+                       float* scores_out, uint8_t* keep_out, uint32_t* hist_out, void* cuda_stream);
+
+/*
+ * Pushes frames of several streams in one set of launches (serving many
+ * concurrent streams). desc[i] is as in cofie_ngff_push for stream
+ * desc[i].stream; device memory only; streams distinct within the call;
+ * nd <= COFIE_NGFF_MAX_BATCH and the total frame count <= max_frames_per_push.
+ * Equivalent to one cofie_ngff_push per descriptor. Errors: COFIE_EINVAL,
+ * COFIE_ECUDA.
+ */
+int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream);
+
+/* Restarts stream `stream` at t = 0 (its next frame is a first frame). */
+int cofie_ngff_reset(cofie_ngff_t* h, uint32_t stream, void* cuda_stream);
+
+/*
+ * Synchronises cuda_stream and reports device-side failures of earlier
+ * calls on the handle: COFIE_ETIMEOUT if a bounded wait inside a kernel ran
+ * out (the affected results are invalid), COFIE_ECUDA on a CUDA error,
+ * COFIE_OK otherwise. Clears the device error word.
+ */
+int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream);
+
+/*
+ * Number of frames stream `stream` has been pushed since creation or its
+ * last reset, as enqueued (host-side count, no synchronisation).
+ */
+int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_out);
+
+/* Text of the last error on this handle (empty string if none). Never NULL. */
+const char* cofie_ngff_last_error(const cofie_ngff_t* h);
+
+/* Text of the last error from a call that had no valid handle (create). Never NULL. */
+const char* cofie_ngff_global_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* COFIE_NGFF_H */
