@@ -1,0 +1,331 @@
+"""NGFF throughput on GB300: frames/s and pixel GB/s of the whole filtering
+path (histogram kernel + windowed-distance kernel + scan kernel) over the
+1080p stream (3600 uint8 RGB frames of 1920x1080, one whole-stream push).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+One step = reset the stream, then push all 3600 frames through the library
+and decide every frame. Inputs (22.4 GB per step) are larger than L2, so no
+flush is needed between steps. Prints one JSON line (rank 0).
+
+Under torchrun each rank filters its own independently seeded 1080p stream
+(weak scaling, no collective on the data path); timing is the max over
+ranks. ``--impl reference`` times the single-threaded C oracle on the host
+cores on a bounded sample of the same stream (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+REPO = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, REPO)
+
+METRIC = "NGFF frames/s and pixel GB/s (fraction of HBM peak) at 1 GB300 vs CPU oracle"
+UNIT = "frames/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+K1_SOURCE = os.path.join(REPO, "paper_2609_03675_gb300", "csrc", "ngff_hist.cu")
+K1_TRAFFIC = os.path.join(REPO, "profiles", "k1_hist_1080p_traffic.json")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=600)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def peaks():
+    try:
+        with open(os.path.join(REPO, "MEASURED_PEAKS.json")) as fh:
+            d = json.load(fh)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:  # noqa: BLE001 -- file absent: the recipe's fallback
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def k1_traffic_per_launch():
+    """DRAM bytes per histogram launch from the committed ncu summary, or None
+    when the kernel source changed since the counters were taken."""
+    try:
+        with open(K1_TRAFFIC) as fh:
+            d = json.load(fh)
+        src = hashlib.sha256(open(K1_SOURCE, "rb").read()).hexdigest()
+        if d.get("source_sha256") != src:
+            return None
+        return float(d["dram_bytes_per_launch_full"])
+    except Exception:  # noqa: BLE001
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.proc = None
+        self.gpu_id = gpu_id
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.file, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        self.file.flush()
+        self.file.seek(0)
+        rows = [ln.strip().split(", ") for ln in self.file.read().splitlines() if ln.strip()]
+        os.unlink(self.file.name)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[0]))
+                mx = float(r[1])
+                for name, v in zip(names, r[4:8]):
+                    if v.strip().lower() == "active":
+                        reasons.add(name)
+            except (ValueError, IndexError):
+                continue
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def oracle_sample(frames_u8_ptr, spec, target_s: float):
+    """The oracle as it stands (single-threaded C) on the first k frames of the
+    stream; k sized to about target_s seconds of CPU work."""
+    import ctypes
+
+    import numpy as np
+
+    import oracle as O
+    o = O.load()
+    p = O.Params(spec.width, spec.height)
+    fb = spec.frame_bytes
+
+    def run(k):
+        arr = np.ctypeslib.as_array((ctypes.c_uint8 * (k * fb)).from_address(frames_u8_ptr))
+        t = time.perf_counter()
+        o.run(arr.reshape(k, spec.height, spec.width, 3), p)
+        return time.perf_counter() - t
+
+    t2 = run(2)
+    k = int(max(2, min(spec.frames, target_s / max(t2 / 2, 1e-6))))
+    dt = run(k)
+    return k, dt
+
+
+def bench_gb300(args):
+    import numpy as np  # noqa: F401
+    import torch
+    import torch.distributed as dist
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    spec = synth.hd1080(seed=synth.SEED_BASE + 3 + rank)
+    T = spec.frames
+    # inputs: generated on the host (pinned, kept for the end-to-end leg), resident in HBM for the timed region
+    host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.to("cuda", non_blocking=True)
+    scores = torch.empty(T, dtype=torch.float32, device="cuda")
+    keep = torch.empty(T, dtype=torch.uint8, device="cuda")
+    f = NGFF(spec.width, spec.height, max_frames_per_push=T)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        f.reset()
+        f.push(dev, scores=scores, keep=keep)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    f.status()
+
+    props = torch.cuda.get_device_properties(local)
+    gpu_id = "GPU-" + str(props.uuid) if getattr(props, "uuid", None) else str(local)
+    f.profile_reset(time_kernels=True)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(gpu_id) as clk:
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        start.record(stream)
+        for _ in range(args.steps):
+            step()
+        end.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+    f.status()
+    prof = f.profile_read()
+    ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    clocks = clk.summary()
+    kept = int((keep != 0).sum().item())
+
+    frames_total = args.steps * T * world
+    value = frames_total / (ms / 1e3)
+    pixel_gbs = frames_total * spec.frame_bytes / (ms / 1e3) / 1e9
+
+    # roofline of the dominant kernel (histogram): algorithmic bytes per launch / mean event-timed duration
+    peak, peak_kind = peaks()
+    k1_ms = prof["hist_ms"] / max(prof["hist_timed"], 1)
+    k1_bytes = prof["hist_bytes"] / max(prof["hist_launches"], 1)
+    achieved = k1_bytes / (k1_ms / 1e3) / 1e9
+    traffic = k1_traffic_per_launch()
+
+    # end to end through the same C entry point with host buffers: H2D of the
+    # step's frames and D2H of its scores and keep codes inside the timed region
+    e2e = None
+    if not args.no_e2e:
+        hs = torch.empty(T, dtype=torch.float32, pin_memory=True)
+        hk = torch.empty(T, dtype=torch.uint8, pin_memory=True)
+        fe = NGFF(spec.width, spec.height, max_frames_per_push=T)
+
+        def estep():
+            fe.reset()
+            fe.push(host, scores=hs, keep=hk)
+
+        estep()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            estep()
+        torch.cuda.synchronize()
+        el = time.perf_counter() - t0
+        if world > 1:
+            tt = torch.tensor([el], device="cuda")
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            el = float(tt.item())
+        fe.status()
+        assert torch.equal(hk.to("cuda"), keep), "end-to-end keep codes differ from the device-resident run"
+        e2e = {"value": args.e2e_steps * T * world / el, "unit": UNIT,
+               "h2d_bytes_per_step": T * spec.frame_bytes, "d2h_bytes_per_step": T * (4 + 1),
+               "ms_per_step": el / args.e2e_steps * 1e3}
+        fe.close()
+
+    cpu = None
+    if rank == 0 and world == 1:
+        k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds)
+        cpu = {"value": k / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"first {k} frames of the 1080p stream, single-threaded C oracle (histograms + selection)"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u8", "data": "synthetic",
+            "config": {"workload": "1080p stream: 3600 uint8 RGB frames of 1920x1080 (HWC), one whole-stream push "
+                                   "per step, B=32, L_max=30, tau_h=0.30",
+                       "frames_per_step": T, "width": spec.width, "height": spec.height, "bins": 32, "l_max": 30,
+                       "tau": 0.30, "l2": "inputs larger than L2 (22.4 GB per step), no flush",
+                       "parallelism": f"{world} independent stream(s), one per GPU"},
+            "pixel_gbs": pixel_gbs,
+            "frac_of_nominal_8tbs": pixel_gbs / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                         "peak_kind": f"{peak_kind} copy bandwidth", "traffic": traffic,
+                         "kernel": "ngff histogram (K1)", "launch_ms": k1_ms, "bytes_per_launch": k1_bytes},
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+            "gpu_launches": int(prof["hist_launches"] + prof["select_launches"]),
+            "clocks": clocks,
+            "kept_frames_last_step": kept,
+        }
+        print(json.dumps(line), flush=True)
+    f.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def bench_reference(args):
+    """The oracle (single-threaded C, host cores) on the same workload and metric."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import numpy as np
+
+    import oracle as O
+    import synth
+    spec = synth.hd1080()
+    o = O.load()
+    p = O.Params(spec.width, spec.height)
+    # each step: a bounded sample of frames so that the whole run stays within about two minutes
+    t_frame = 0.012
+    per_step = int(max(2, min(64, 120.0 / max(args.steps + args.warmup, 1) / t_frame)))
+    frames = synth.generate(spec, 0, per_step)
+    for _ in range(args.warmup):
+        o.run(frames, p)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        o.run(frames, p)
+    el = time.perf_counter() - t0
+    value = args.steps * per_step / el
+    sample = f"first {per_step} frames of the 1080p stream per step, single-threaded C oracle"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u8", "data": "synthetic",
+        "config": {"workload": "1080p stream: 3600 uint8 RGB frames of 1920x1080 (HWC), B=32, L_max=30, tau_h=0.30",
+                   "frames_per_step": per_step, "width": spec.width, "height": spec.height},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    del np
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        bench_reference(args)
+    else:
+        bench_gb300(args)
+
+
+if __name__ == "__main__":
+    main()

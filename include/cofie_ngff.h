@@ -29,8 +29,10 @@
  *     host memory is copied asynchronously; pageable host memory works but
  *     the copy is synchronous with the host).
  *   - Output buffers may be device or host memory; the library detects which.
- *   - A nonzero return is an error code below; on error nothing was enqueued
- *     and no stream state changed, and cofie_ngff_last_error() describes it.
+ *   - A nonzero return is an error code below and cofie_ngff_last_error()
+ *     describes it. Argument errors (COFIE_EINVAL) are found before anything
+ *     is enqueued, so they leave the stream state unchanged; a COFIE_ECUDA
+ *     from a failed launch may leave earlier pieces of the call enqueued.
  *   - A handle is not thread-safe: calls on one handle must be serialised.
  *   - Nothing aborts, traps or prints. Device-side waits are bounded; a wait
  *     that runs out sets an error word that cofie_ngff_status() reports.
@@ -170,6 +172,36 @@ int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream);
  * last reset, as enqueued (host-side count, no synchronisation).
  */
 int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_out);
+
+/*
+ * Diagnostic: applies the fast histogram kernel's own per-pixel grayscale and
+ * bin functions to n_pixels RGB triples (device memory, 3 * n_pixels bytes,
+ * n_pixels a multiple of 4) and writes one bin index per pixel to bins_out
+ * (device memory, n_pixels bytes). Lets tests check the device binning of
+ * every RGB triple. COFIE_EINVAL if the handle's parameters only run the
+ * generic kernel.
+ */
+int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pixels, uint8_t* bins_out,
+                          void* cuda_stream);
+
+/*
+ * Launch counters and kernel timing (a tracing aid). Counters run always;
+ * with timing on, every launch of the histogram kernel is bracketed by two
+ * CUDA events recorded on the stream it is launched on.
+ */
+typedef struct {
+  uint64_t hist_launches;   /* histogram-kernel launches since the last reset */
+  uint64_t select_launches; /* distance + scan kernel launches since the last reset */
+  uint64_t hist_bytes;      /* algorithmic bytes of those histogram launches: frame bytes read + counts written */
+  uint64_t hist_timed;      /* histogram launches that were event-timed */
+  double hist_ms;           /* summed event-timed histogram-kernel durations, milliseconds */
+} cofie_ngff_profile;
+
+/* Zeroes the counters; time_kernels != 0 turns event timing on, 0 off. */
+int cofie_ngff_profile_reset(cofie_ngff_t* h, int time_kernels);
+
+/* Waits for the timed launches and writes the counters to *out. */
+int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out);
 
 /* Text of the last error on this handle (empty string if none). Never NULL. */
 const char* cofie_ngff_last_error(const cofie_ngff_t* h);

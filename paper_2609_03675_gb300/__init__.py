@@ -1,0 +1,172 @@
+"""NGFF (CoFiE's Novelty-Guided Frame Filtering, Sec. 3.2) on GB300.
+
+Thin Python binding of libcofie_ngff.so. Every step of the method runs in the
+library's CUDA kernels; this module only marshals arguments. PyTorch provides
+device memory and the current CUDA stream.
+
+    from paper_2609_03675_gb300 import NGFF
+    f = NGFF(1920, 1080)                 # B=32, L_max=30, M_min=4, tau_h=0.30
+    scores, keep = f.push(frames_u8)     # frames: uint8 [n, H, W, 3], cuda or cpu
+"""
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from . import _abi
+from ._abi import (KEEP_DROP, KEEP_FIRST, KEEP_GAP, KEEP_NOVELTY, NGFFError)  # noqa: F401
+
+__all__ = ["NGFF", "NGFFError", "KEEP_DROP", "KEEP_NOVELTY", "KEEP_GAP", "KEEP_FIRST", "library_path"]
+
+
+def library_path() -> str:
+    return _abi.LIB_PATH
+
+
+def _ptr(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, torch.Tensor):
+        if not x.is_contiguous():
+            raise ValueError("tensors passed to the library must be contiguous")
+        return x.data_ptr()
+    return int(x)
+
+
+class NGFF:
+    """One library handle: max_streams independent streams of width x height frames."""
+
+    def __init__(self, width: int, height: int, *, bins: int = 32, l_max: int = 30, m_min: int = 4,
+                 tau: float = 0.30, luma_weights=(299, 587, 114), luma_den: int = 1000, max_streams: int = 1,
+                 max_frames_per_push: int = 4096, device: int | None = None, host_stage_bytes: int = 0):
+        lib = _abi.load()
+        p = _abi.Params()
+        lib.cofie_ngff_default_params(ctypes.byref(p), width, height)
+        p.bins, p.l_max, p.m_min, p.tau = bins, l_max, m_min, tau
+        p.luma_w[0], p.luma_w[1], p.luma_w[2] = luma_weights
+        p.luma_den = luma_den
+        p.max_streams, p.max_frames_per_push = max_streams, max_frames_per_push
+        if device is None:
+            device = torch.cuda.current_device()
+        p.device = device
+        p.host_stage_bytes = host_stage_bytes
+        h = ctypes.c_void_p()
+        rc = lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h))
+        if rc != _abi.OK:
+            raise NGFFError(rc, lib.cofie_ngff_global_error().decode())
+        self._lib, self._h, self.params = lib, h, p
+        self.width, self.height, self.bins, self.l_max, self.m_min, self.tau = width, height, bins, l_max, m_min, tau
+        self.device = torch.device("cuda", device)
+        self.frame_bytes = 3 * width * height
+
+    # ----------------------------------------------------------------- util --
+    def _check(self, rc: int):
+        if rc != _abi.OK:
+            raise NGFFError(rc, self._lib.cofie_ngff_last_error(self._h).decode())
+
+    def _stream(self, cuda_stream):
+        if cuda_stream is None:
+            return torch.cuda.current_stream(self.device).cuda_stream
+        if isinstance(cuda_stream, torch.cuda.Stream):
+            return cuda_stream.cuda_stream
+        return int(cuda_stream)
+
+    def _outputs(self, frames, n, scores, keep, hist, want_hist):
+        on_gpu = isinstance(frames, torch.Tensor) and frames.is_cuda
+        kw = dict(device=self.device) if on_gpu else dict(pin_memory=True)
+        if scores is None:
+            scores = torch.empty(n, dtype=torch.float32, **kw)
+        if keep is None:
+            keep = torch.empty(n, dtype=torch.uint8, **kw)
+        if want_hist and hist is None:
+            hist = torch.empty((n, self.bins), dtype=torch.int32, **kw)
+        return scores, keep, hist
+
+    def _frames(self, frames):
+        if isinstance(frames, torch.Tensor):
+            if frames.dtype != torch.uint8:
+                raise ValueError("frames must be uint8")
+            if frames.numel() % self.frame_bytes:
+                raise ValueError("frames must hold whole width x height x 3 frames")
+            return frames.numel() // self.frame_bytes
+        raise TypeError("frames must be a torch.uint8 tensor [n, H, W, 3] (cuda or cpu)")
+
+    # ------------------------------------------------------------------ API --
+    def push(self, frames, stream: int = 0, *, scores=None, keep=None, hist=None, return_hist: bool = False,
+             cuda_stream=None):
+        """Decides the next n frames of ``stream``; returns (scores, keep) or
+        (scores, keep, hist). Asynchronous on the current CUDA stream."""
+        n = self._frames(frames)
+        scores, keep, hist = self._outputs(frames, n, scores, keep, hist, return_hist or hist is not None)
+        st = self._stream(cuda_stream)
+        if hist is None:
+            rc = self._lib.cofie_ngff_push(self._h, stream, _ptr(frames), n, _ptr(scores), _ptr(keep), st)
+        else:
+            rc = self._lib.cofie_ngff_push_ex(self._h, stream, _ptr(frames), n, _ptr(scores), _ptr(keep),
+                                              _ptr(hist), st)
+        self._check(rc)
+        return (scores, keep, hist) if hist is not None else (scores, keep)
+
+    def push_raw(self, stream: int, frames_ptr: int, n: int, scores_ptr=None, keep_ptr=None, hist_ptr=None,
+                 cuda_stream=None):
+        """The C entry point with plain addresses (device or host)."""
+        st = self._stream(cuda_stream)
+        rc = self._lib.cofie_ngff_push_ex(self._h, stream, frames_ptr, n, scores_ptr, keep_ptr, hist_ptr, st)
+        self._check(rc)
+
+    def push_batch(self, items, cuda_stream=None):
+        """items: list of (stream, frames[cuda uint8], scores[cuda f32] | None, keep[cuda u8] | None)."""
+        arr = (_abi.PushDesc * max(1, len(items)))()
+        for i, (stream, frames, scores, keep) in enumerate(items):
+            n = self._frames(frames)
+            arr[i].stream, arr[i].n = stream, n
+            arr[i].frames, arr[i].scores_out, arr[i].keep_out = _ptr(frames), _ptr(scores), _ptr(keep)
+        self._check(self._lib.cofie_ngff_push_batch(self._h, arr, len(items), self._stream(cuda_stream)))
+
+    def reset(self, stream: int = 0, cuda_stream=None):
+        self._check(self._lib.cofie_ngff_reset(self._h, stream, self._stream(cuda_stream)))
+
+    def status(self, cuda_stream=None):
+        """Synchronises and raises NGFFError if a device-side wait ran out."""
+        self._check(self._lib.cofie_ngff_status(self._h, self._stream(cuda_stream)))
+
+    def frames_seen(self, stream: int = 0) -> int:
+        t = ctypes.c_uint64(0)
+        self._check(self._lib.cofie_ngff_frames_seen(self._h, stream, ctypes.byref(t)))
+        return t.value
+
+    def debug_bins(self, pixels: torch.Tensor, out: torch.Tensor | None = None, cuda_stream=None):
+        """Device bin index of every RGB triple in ``pixels`` (cuda uint8 [..., 3])."""
+        n = pixels.numel() // 3
+        if out is None:
+            out = torch.empty(n, dtype=torch.uint8, device=pixels.device)
+        self._check(self._lib.cofie_ngff_debug_bins(self._h, _ptr(pixels), n, _ptr(out), self._stream(cuda_stream)))
+        return out
+
+    def profile_reset(self, time_kernels: bool = False):
+        """Zeroes the launch counters; with time_kernels every histogram-kernel
+        launch is bracketed by CUDA events on its stream."""
+        self._check(self._lib.cofie_ngff_profile_reset(self._h, int(time_kernels)))
+
+    def profile_read(self) -> dict:
+        pr = _abi.Profile()
+        self._check(self._lib.cofie_ngff_profile_read(self._h, ctypes.byref(pr)))
+        return {k: getattr(pr, k) for k, _ in _abi.Profile._fields_}
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.cofie_ngff_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001 -- interpreter shutdown
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

@@ -1,0 +1,579 @@
+// C ABI of the NGFF library (declared in include/cofie_ngff.h).
+//
+// A push of n frames of one stream runs, in stream order:
+//   memset(hist) -> K1 histograms -> K2 windowed distances + gap masks ->
+//   K3 scan (scores, keep codes, stream state)
+// in pieces of at most max_frames_per_push frames. Frames in host memory are
+// copied into one of two device staging buffers on an internal copy stream,
+// overlapping the copy of piece i+1 with the kernels of piece i. Outputs in
+// host memory are written to device scratch and copied back on the caller's
+// stream.
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "cofie_ngff.h"
+#include "ngff_common.cuh"
+
+using namespace cofie;
+
+namespace {
+
+thread_local std::string g_global_error;
+
+enum MemKind { kNull = 0, kDevice = 1, kHostPinned = 2, kHostPageable = 3 };
+
+constexpr uint64_t kDefaultStageBytes = 256ull << 20;
+constexpr uint64_t kTimeoutNs = 2000000000ull;  // bounded device waits: 2 s
+constexpr size_t kMaxTimedEvents = 1u << 16;
+
+struct DeviceGuard {
+  int prev = -1;
+  bool ok = true;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+}  // namespace
+
+struct cofie_ngff {
+  cofie_ngff_params p{};
+  int device = 0;
+  int num_sms = 0;
+  uint64_t frame_bytes = 0;
+  uint32_t npix = 0;
+  uint32_t mask_words = 0;
+  LumaConsts lc{};
+  int bin_path = -1;  // kBinFast, kBinTwoStep, or -1 (generic kernel only)
+  bool size_fast = false;
+  int hist_grid = 0;
+  float two_n = 0.f;
+  uint32_t* d_hist = nullptr;
+  uint32_t* d_l1 = nullptr;
+  uint32_t* d_mask = nullptr;
+  uint32_t* d_ring = nullptr;
+  StreamState* d_state = nullptr;
+  float* d_scores = nullptr;
+  uint8_t* d_keep = nullptr;
+  uint32_t* d_err = nullptr;
+  uint8_t* d_stage[2] = {nullptr, nullptr};
+  uint64_t stage_bytes = 0;
+  uint32_t stage_frames = 0;
+  uint32_t stage_next = 0;
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t ev_copied[2] = {nullptr, nullptr};
+  cudaEvent_t ev_free[2] = {nullptr, nullptr};
+  std::vector<uint64_t> seen;
+  std::string err;
+  // launch counters and optional event timing of the histogram kernel
+  uint64_t n_hist = 0, n_select = 0, hist_bytes = 0;
+  bool time_kernels = false;
+  std::vector<cudaEvent_t> ev_pool;  // pairs: [2i] start, [2i+1] end
+  size_t ev_used = 0;
+
+  int fail(int code, const std::string& msg) {
+    err = msg;
+    return code;
+  }
+  int cuda_fail(cudaError_t e, const char* what) {
+    err = std::string(what) + ": " + cudaGetErrorString(e);
+    return COFIE_ECUDA;
+  }
+};
+
+namespace {
+
+MemKind classify(const void* ptr, int* dev_out = nullptr) {
+  if (!ptr) return kNull;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    cudaGetLastError();
+    return kHostPageable;
+  }
+  if (dev_out) *dev_out = a.device;
+  switch (a.type) {
+    case cudaMemoryTypeDevice:
+    case cudaMemoryTypeManaged:
+      return kDevice;
+    case cudaMemoryTypeHost:
+      return kHostPinned;
+    default:
+      return kHostPageable;
+  }
+}
+
+bool verify_magic(uint32_t magic, uint32_t vmax, uint32_t den, uint32_t bins, bool divide_only) {
+  for (uint32_t v = 0; v <= vmax; ++v) {
+    const uint32_t y = v / den;
+    const uint32_t want = divide_only ? y : (y * bins) / 256u;
+    const uint32_t got = static_cast<uint32_t>((static_cast<uint64_t>(v) * magic) >> 32);
+    if (got != want) return false;
+  }
+  return true;
+}
+
+int validate_params(const cofie_ngff_params* p, std::string& why) {
+  if (!p) return why = "params is NULL", COFIE_EINVAL;
+  if (p->width == 0 || p->height == 0) return why = "width and height must be >= 1", COFIE_EINVAL;
+  const uint64_t npix = static_cast<uint64_t>(p->width) * p->height;
+  if (npix > 0x7fffffffull) return why = "width * height must be < 2^31", COFIE_EINVAL;
+  if (p->bins < 1 || p->bins > COFIE_NGFF_MAX_BINS) return why = "bins must be in [1, 256]", COFIE_EINVAL;
+  if (p->l_max < 1 || p->l_max > COFIE_NGFF_MAX_LMAX) return why = "l_max must be in [1, 256]", COFIE_EINVAL;
+  if (p->tau != p->tau) return why = "tau is NaN", COFIE_EINVAL;
+  if (p->luma_den == 0 || p->luma_den > 65535) return why = "luma_den must be in [1, 65535]", COFIE_EINVAL;
+  if (static_cast<uint64_t>(p->luma_w[0]) + p->luma_w[1] + p->luma_w[2] != p->luma_den)
+    return why = "luma weights must sum to luma_den", COFIE_EINVAL;
+  if (p->max_streams < 1) return why = "max_streams must be >= 1", COFIE_EINVAL;
+  if (p->max_frames_per_push < 1) return why = "max_frames_per_push must be >= 1", COFIE_EINVAL;
+  return COFIE_OK;
+}
+
+template <typename T>
+cudaError_t dalloc(T** p, size_t count) {
+  return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) + 16);
+}
+
+// Runs K1-K3 over the rows described by segs (device frames).
+int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
+  if (segs.rows == 0) return COFIE_OK;
+  cudaError_t e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(segs.rows) * h->p.bins * 4, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+  bool fast = h->size_fast && h->bin_path >= 0;
+  for (uint32_t i = 0; i < segs.count && fast; ++i)
+    if (reinterpret_cast<uintptr_t>(segs.s[i].frames) % 16 != 0) fast = false;
+  HistArgs ha{};
+  ha.frame_bytes = h->frame_bytes;
+  ha.npix = h->npix;
+  ha.groups_per_frame = static_cast<uint32_t>(h->frame_bytes / 48);
+  ha.chunks_per_frame = (ha.groups_per_frame + hist_chunk_groups() - 1) / hist_chunk_groups();
+  ha.timeout_ns = kTimeoutNs;
+  cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+  if (h->time_kernels && h->ev_used + 2 <= kMaxTimedEvents) {
+    while (h->ev_pool.size() < h->ev_used + 2) {
+      cudaEvent_t ev;
+      if (cudaEventCreate(&ev) != cudaSuccess) break;
+      h->ev_pool.push_back(ev);
+    }
+    if (h->ev_pool.size() >= h->ev_used + 2) {
+      ev0 = h->ev_pool[h->ev_used];
+      ev1 = h->ev_pool[h->ev_used + 1];
+      h->ev_used += 2;
+      cudaEventRecord(ev0, st);
+    }
+  }
+  if (fast) {
+    const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
+    const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid);
+    e = launch_hist_fast(segs, ha, h->lc, h->bin_path, h->d_hist, h->d_err, grid, st);
+  } else {
+    e = launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
+  }
+  if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
+  if (ev1) cudaEventRecord(ev1, st);
+  h->n_hist += 1;
+  h->hist_bytes += static_cast<uint64_t>(segs.rows) * (h->frame_bytes + 4ull * h->p.bins);
+  SelectArgs sa{};
+  sa.bins = h->p.bins;
+  sa.l_max = h->p.l_max;
+  sa.mask_words = h->mask_words;
+  sa.tau = h->p.tau;
+  sa.two_n = h->two_n;
+  e = launch_window(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "window kernel launch");
+  e = launch_scan(segs, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "scan kernel launch");
+  h->n_select += 2;
+  return COFIE_OK;
+}
+
+// One piece of a single-stream push: n <= max_frames_per_push device frames.
+int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n, float* scores, MemKind ks,
+              uint8_t* keep, MemKind kk, uint32_t* hist_out, MemKind kh, cudaStream_t st) {
+  SegTable segs;
+  memset(&segs, 0, sizeof segs);
+  segs.count = 1;
+  segs.rows = n;
+  Segment& s = segs.s[0];
+  s.frames = dframes;
+  s.n = n;
+  s.row0 = 0;
+  s.stream = stream;
+  s.scores = ks == kDevice ? scores : (ks == kNull ? nullptr : h->d_scores);
+  s.keep = kk == kDevice ? keep : (kk == kNull ? nullptr : h->d_keep);
+  int rc = run_segments(h, segs, st);
+  if (rc != COFIE_OK) return rc;
+  cudaError_t e = cudaSuccess;
+  if (ks == kHostPinned || ks == kHostPageable)
+    e = cudaMemcpyAsync(scores, h->d_scores, n * sizeof(float), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess && (kk == kHostPinned || kk == kHostPageable))
+    e = cudaMemcpyAsync(keep, h->d_keep, n, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess && kh != kNull)
+    e = cudaMemcpyAsync(hist_out, h->d_hist, static_cast<size_t>(n) * h->p.bins * 4, cudaMemcpyDefault, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "output copy");
+  return COFIE_OK;
+}
+
+int ensure_staging(cofie_ngff* h) {
+  if (h->d_stage[0]) return COFIE_OK;
+  for (int i = 0; i < 2; ++i) {
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&h->d_stage[i]), h->stage_bytes);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      for (int j = 0; j < 2; ++j) {
+        if (h->d_stage[j]) cudaFree(h->d_stage[j]);
+        h->d_stage[j] = nullptr;
+      }
+      return h->fail(COFIE_ENOMEM, "staging buffer allocation failed");
+    }
+  }
+  return COFIE_OK;
+}
+
+int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n, float* scores, uint8_t* keep,
+              uint32_t* hist_out, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+  if (n == 0) return COFIE_OK;
+  if (!frames) return h->fail(COFIE_EINVAL, "frames is NULL");
+  DeviceGuard guard(h->device);
+  if (!guard.ok) return h->fail(COFIE_ECUDA, "cannot select the handle's device");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  int fdev = -1;
+  const MemKind kf = classify(frames, &fdev);
+  const MemKind ks = classify(scores), kk = classify(keep), kh = classify(hist_out);
+  if (kf == kDevice && fdev != h->device) return h->fail(COFIE_EINVAL, "frames live on another device");
+  const uint32_t B = h->p.bins;
+  if (kf == kDevice) {
+    const uint32_t step = h->p.max_frames_per_push;
+    for (uint32_t off = 0; off < n; off += step) {
+      const uint32_t m = n - off < step ? n - off : step;
+      int rc = run_piece(h, stream, frames + off * h->frame_bytes, m, scores ? scores + off : nullptr, ks,
+                         keep ? keep + off : nullptr, kk, hist_out ? hist_out + static_cast<size_t>(off) * B : nullptr,
+                         kh, st);
+      if (rc != COFIE_OK) return rc;
+    }
+  } else {
+    int rc = ensure_staging(h);
+    if (rc != COFIE_OK) return rc;
+    const uint32_t step = h->stage_frames < h->p.max_frames_per_push ? h->stage_frames : h->p.max_frames_per_push;
+    for (uint32_t off = 0; off < n; off += step) {
+      const uint32_t m = n - off < step ? n - off : step;
+      const uint32_t slot = h->stage_next;
+      h->stage_next ^= 1u;
+      cudaError_t e = cudaStreamWaitEvent(h->copy_stream, h->ev_free[slot], 0);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h->d_stage[slot], frames + off * h->frame_bytes, m * h->frame_bytes,
+                            cudaMemcpyHostToDevice, h->copy_stream);
+      if (e == cudaSuccess) e = cudaEventRecord(h->ev_copied[slot], h->copy_stream);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_copied[slot], 0);
+      if (e != cudaSuccess) return h->cuda_fail(e, "host frame staging");
+      rc = run_piece(h, stream, h->d_stage[slot], m, scores ? scores + off : nullptr, ks, keep ? keep + off : nullptr,
+                     kk, hist_out ? hist_out + static_cast<size_t>(off) * B : nullptr, kh, st);
+      if (rc != COFIE_OK) return rc;
+      e = cudaEventRecord(h->ev_free[slot], st);
+      if (e != cudaSuccess) return h->cuda_fail(e, "staging event");
+    }
+  }
+  h->seen[stream] += n;
+  h->err.clear();
+  return COFIE_OK;
+}
+
+void free_handle(cofie_ngff* h) {
+  if (!h) return;
+  DeviceGuard guard(h->device);
+  cudaDeviceSynchronize();
+  void* bufs[] = {h->d_hist, h->d_l1, h->d_mask, h->d_ring, h->d_state, h->d_scores,
+                  h->d_keep, h->d_err,  h->d_stage[0], h->d_stage[1]};
+  for (void* b : bufs)
+    if (b) cudaFree(b);
+  for (cudaEvent_t ev : h->ev_pool) cudaEventDestroy(ev);
+  for (int i = 0; i < 2; ++i) {
+    if (h->ev_copied[i]) cudaEventDestroy(h->ev_copied[i]);
+    if (h->ev_free[i]) cudaEventDestroy(h->ev_free[i]);
+  }
+  if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
+  delete h;
+}
+
+}  // namespace
+
+extern "C" {
+
+void cofie_ngff_default_params(cofie_ngff_params* p, uint32_t width, uint32_t height) {
+  if (!p) return;
+  memset(p, 0, sizeof *p);
+  p->width = width;
+  p->height = height;
+  p->bins = 32;     // App. A
+  p->l_max = 30;    // App. B.2
+  p->m_min = 4;     // App. B.2
+  p->tau = 0.30f;   // App. B.2
+  p->luma_w[0] = 299;
+  p->luma_w[1] = 587;
+  p->luma_w[2] = 114;
+  p->luma_den = 1000;
+  p->max_streams = 1;
+  p->max_frames_per_push = 4096;
+  p->device = -1;
+  p->host_stage_bytes = 0;
+}
+
+int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
+  std::string why;
+  if (!out) {
+    g_global_error = "out is NULL";
+    return COFIE_EINVAL;
+  }
+  int rc = validate_params(p, why);
+  if (rc != COFIE_OK) {
+    g_global_error = why;
+    return rc;
+  }
+  int dev = p->device;
+  if (dev < 0 && cudaGetDevice(&dev) != cudaSuccess) {
+    g_global_error = "no CUDA device";
+    return COFIE_ECUDA;
+  }
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess || dev >= ndev) {
+    cudaGetLastError();
+    g_global_error = "device ordinal out of range";
+    return COFIE_EINVAL;
+  }
+  DeviceGuard guard(dev);
+  if (!guard.ok) {
+    g_global_error = "cannot select the device";
+    return COFIE_ECUDA;
+  }
+  cofie_ngff* h = new (std::nothrow) cofie_ngff();
+  if (!h) {
+    g_global_error = "host allocation failed";
+    return COFIE_ENOMEM;
+  }
+  h->p = *p;
+  h->device = dev;
+  h->p.device = dev;
+  cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev);
+  h->npix = p->width * p->height;
+  h->frame_bytes = 3ull * h->npix;
+  h->mask_words = (p->l_max + 31) / 32;
+  h->two_n = static_cast<float>(2ull * h->npix);
+  h->size_fast = (h->npix % 16) == 0;
+  h->seen.assign(p->max_streams, 0);
+
+  LumaConsts& lc = h->lc;
+  const uint32_t wr = p->luma_w[0], wg = p->luma_w[1], wb = p->luma_w[2], den = p->luma_den;
+  lc.w_rg = (wg << 16) | wr;
+  lc.w_b0 = wb;
+  lc.w_0r = wr << 16;
+  lc.w_gb = (wb << 16) | wg;
+  lc.half = den / 2;
+  lc.bins = p->bins;
+  lc.w[0] = wr;
+  lc.w[1] = wg;
+  lc.w[2] = wb;
+  lc.den = den;
+  const uint32_t vmax = 255u * den + den / 2;
+  h->bin_path = -1;
+  if (256 % p->bins == 0) {
+    const uint64_t D = static_cast<uint64_t>(den) * (256 / p->bins);
+    const uint64_t M = ((1ull << 32) + D - 1) / D;
+    if (D >= 2 && M <= 0xffffffffull && verify_magic(static_cast<uint32_t>(M), vmax, den, p->bins, false)) {
+      lc.magic = static_cast<uint32_t>(M);
+      h->bin_path = kBinFast;
+    }
+  }
+  if (h->bin_path < 0 && den >= 2) {
+    const uint64_t M = ((1ull << 32) + den - 1) / den;
+    if (M <= 0xffffffffull && verify_magic(static_cast<uint32_t>(M), vmax, den, p->bins, true)) {
+      lc.magic_y = static_cast<uint32_t>(M);
+      h->bin_path = kBinTwoStep;
+    }
+  }
+
+  const uint64_t F = p->max_frames_per_push, S = p->max_streams;
+  cudaError_t e = cudaSuccess;
+  if (e == cudaSuccess) e = dalloc(&h->d_hist, F * p->bins);
+  if (e == cudaSuccess) e = dalloc(&h->d_l1, F * p->l_max);
+  if (e == cudaSuccess) e = dalloc(&h->d_mask, F * h->mask_words);
+  if (e == cudaSuccess) e = dalloc(&h->d_ring, S * p->l_max * p->bins);
+  if (e == cudaSuccess) e = dalloc(&h->d_state, S);
+  if (e == cudaSuccess) e = dalloc(&h->d_scores, F);
+  if (e == cudaSuccess) e = dalloc(&h->d_keep, F);
+  if (e == cudaSuccess) e = dalloc(&h->d_err, 1);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    free_handle(h);
+    g_global_error = "device allocation failed";
+    return COFIE_ENOMEM;
+  }
+  if (e == cudaSuccess) e = cudaMemset(h->d_state, 0, S * sizeof(StreamState));
+  if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
+  for (int i = 0; i < 2 && e == cudaSuccess; ++i) {
+    e = cudaEventCreateWithFlags(&h->ev_copied[i], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_free[i], cudaEventDisableTiming);
+  }
+  if (e == cudaSuccess) e = scan_prepare(h->mask_words, p->l_max);
+  if (e == cudaSuccess && h->bin_path >= 0) {
+    const int per_sm = hist_blocks_per_sm(h->bin_path, p->bins);
+    if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
+    h->hist_grid = h->num_sms * (per_sm > 0 ? per_sm : 1);
+  }
+  if (e != cudaSuccess) {
+    g_global_error = std::string("CUDA setup failed: ") + cudaGetErrorString(e);
+    cudaGetLastError();
+    free_handle(h);
+    return COFIE_ECUDA;
+  }
+  uint64_t sb = p->host_stage_bytes ? p->host_stage_bytes : kDefaultStageBytes;
+  if (sb < h->frame_bytes) sb = h->frame_bytes;
+  h->stage_frames = static_cast<uint32_t>(sb / h->frame_bytes);
+  h->stage_bytes = static_cast<uint64_t>(h->stage_frames) * h->frame_bytes;
+  *out = h;
+  return COFIE_OK;
+}
+
+void cofie_ngff_destroy(cofie_ngff_t* h) { free_handle(h); }
+
+int cofie_ngff_push(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n, float* scores_out,
+                    uint8_t* keep_out, void* cuda_stream) {
+  return push_impl(h, stream, frames, n, scores_out, keep_out, nullptr, cuda_stream);
+}
+
+int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n, float* scores_out,
+                       uint8_t* keep_out, uint32_t* hist_out, void* cuda_stream) {
+  return push_impl(h, stream, frames, n, scores_out, keep_out, hist_out, cuda_stream);
+}
+
+int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (nd == 0) return COFIE_OK;
+  if (!desc) return h->fail(COFIE_EINVAL, "desc is NULL");
+  if (nd > COFIE_NGFF_MAX_BATCH) return h->fail(COFIE_EINVAL, "more than COFIE_NGFF_MAX_BATCH descriptors");
+  DeviceGuard guard(h->device);
+  if (!guard.ok) return h->fail(COFIE_ECUDA, "cannot select the handle's device");
+  SegTable segs;
+  memset(&segs, 0, sizeof segs);
+  uint64_t rows = 0;
+  std::vector<uint8_t> used(h->p.max_streams, 0);
+  for (uint32_t i = 0; i < nd; ++i) {
+    const cofie_ngff_push_desc& d = desc[i];
+    if (d.stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+    if (used[d.stream]) return h->fail(COFIE_EINVAL, "a stream appears twice in one batch");
+    used[d.stream] = 1;
+    if (d.n > 0) {
+      int fdev = -1;
+      if (!d.frames || classify(d.frames, &fdev) != kDevice || fdev != h->device)
+        return h->fail(COFIE_EINVAL, "batched frames must be device memory on the handle's device");
+      if ((d.scores_out && classify(d.scores_out) != kDevice) || (d.keep_out && classify(d.keep_out) != kDevice))
+        return h->fail(COFIE_EINVAL, "batched outputs must be device memory");
+    }
+    Segment& s = segs.s[segs.count++];
+    s.frames = d.frames;
+    s.n = d.n;
+    s.row0 = static_cast<uint32_t>(rows);
+    s.stream = d.stream;
+    s.scores = d.scores_out;
+    s.keep = d.keep_out;
+    rows += d.n;
+  }
+  if (rows > h->p.max_frames_per_push) return h->fail(COFIE_EINVAL, "batch exceeds max_frames_per_push frames");
+  segs.rows = static_cast<uint32_t>(rows);
+  int rc = run_segments(h, segs, static_cast<cudaStream_t>(cuda_stream));
+  if (rc != COFIE_OK) return rc;
+  for (uint32_t i = 0; i < nd; ++i) h->seen[desc[i].stream] += desc[i].n;
+  h->err.clear();
+  return COFIE_OK;
+}
+
+int cofie_ngff_reset(cofie_ngff_t* h, uint32_t stream, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+  DeviceGuard guard(h->device);
+  cudaError_t e =
+      cudaMemsetAsync(h->d_state + stream, 0, sizeof(StreamState), static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return h->cuda_fail(e, "reset");
+  h->seen[stream] = 0;
+  return COFIE_OK;
+}
+
+int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  DeviceGuard guard(h->device);
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return h->cuda_fail(e, "stream synchronise");
+  uint32_t word = 0;
+  e = cudaMemcpy(&word, h->d_err, sizeof word, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return h->cuda_fail(e, "error word read");
+  if (word) {
+    cudaMemset(h->d_err, 0, sizeof word);
+    char buf[96];
+    snprintf(buf, sizeof buf, "device-side wait ran out (error bits 0x%x)", word);
+    return h->fail(COFIE_ETIMEOUT, buf);
+  }
+  return COFIE_OK;
+}
+
+int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_out) {
+  if (!h || !t_out || stream >= h->p.max_streams) return COFIE_EINVAL;
+  *t_out = h->seen[stream];
+  return COFIE_OK;
+}
+
+int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pixels, uint8_t* bins_out,
+                          void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (n_pixels == 0) return COFIE_OK;
+  if (!pixels || !bins_out || n_pixels % 4 != 0) return h->fail(COFIE_EINVAL, "pixels/bins_out NULL or n_pixels % 4");
+  if (h->bin_path < 0) return h->fail(COFIE_EINVAL, "these parameters use the generic histogram kernel only");
+  if (classify(pixels) != kDevice || classify(bins_out) != kDevice)
+    return h->fail(COFIE_EINVAL, "debug buffers must be device memory");
+  DeviceGuard guard(h->device);
+  cudaError_t e = launch_debug_bins(pixels, n_pixels / 4, h->lc, h->bin_path, bins_out,
+                                    static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return h->cuda_fail(e, "debug kernel launch");
+  return COFIE_OK;
+}
+
+int cofie_ngff_profile_reset(cofie_ngff_t* h, int time_kernels) {
+  if (!h) return COFIE_EINVAL;
+  h->n_hist = h->n_select = h->hist_bytes = 0;
+  h->ev_used = 0;
+  h->time_kernels = time_kernels != 0;
+  return COFIE_OK;
+}
+
+int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out) {
+  if (!h || !out) return COFIE_EINVAL;
+  DeviceGuard guard(h->device);
+  double ms = 0.0;
+  for (size_t i = 0; i + 1 < h->ev_used; i += 2) {
+    cudaError_t e = cudaEventSynchronize(h->ev_pool[i + 1]);
+    float t = 0.f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, h->ev_pool[i], h->ev_pool[i + 1]);
+    if (e != cudaSuccess) return h->cuda_fail(e, "kernel timing events");
+    ms += t;
+  }
+  out->hist_launches = h->n_hist;
+  out->select_launches = h->n_select;
+  out->hist_bytes = h->hist_bytes;
+  out->hist_timed = h->ev_used / 2;
+  out->hist_ms = ms;
+  return COFIE_OK;
+}
+
+const char* cofie_ngff_last_error(const cofie_ngff_t* h) { return h ? h->err.c_str() : ""; }
+
+const char* cofie_ngff_global_error(void) { return g_global_error.c_str(); }
+
+}  // extern "C"

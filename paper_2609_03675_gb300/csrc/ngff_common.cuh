@@ -1,0 +1,99 @@
+// Internal declarations shared by the NGFF kernels and the C ABI layer.
+//
+// Data layout in device memory (per handle):
+//   frames   uint8  [rows][H][W][3]   caller-owned (or a staging buffer)
+//   hist     uint32 [rows][B]         integer histograms of the push
+//   l1       uint32 [rows][L_max]     L1[t][k-1] = sum_b |c_t[b] - c_{t-k}[b]|
+//   mask     uint32 [rows][W_m]       bit g-1 of row t: keep decision of frame t
+//                                     if its gap t - r(t) were g (W_m = ceil(L_max/32))
+//   ring     uint32 [streams][L_max][B]  histogram of frame t at slot t mod L_max
+//   state    StreamState [streams]    frames seen and current gap
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace cofie {
+
+constexpr int kMaxSegs = 64;
+constexpr int kMaxBins = 256;
+constexpr int kMaxLmax = 256;
+
+// One stream's frames inside a push: rows [row0, row0 + n) of the tables.
+struct Segment {
+  const uint8_t* frames;  // device pointer of the first frame
+  float* scores;          // device, n entries, or nullptr
+  uint8_t* keep;          // device, n entries, or nullptr
+  uint32_t n;
+  uint32_t row0;
+  uint32_t stream;
+  uint32_t pad;
+};
+
+struct SegTable {
+  Segment s[kMaxSegs];
+  uint32_t count;
+  uint32_t rows;
+};
+
+// Grayscale weights packed for the two-way 16x8-bit dot product (dp2a):
+// dp2a.lo(a, b, c) = a.h0 * b.byte0 + a.h1 * b.byte1 + c, .hi uses bytes 2, 3.
+struct LumaConsts {
+  uint32_t w_rg;     // (wG << 16) | wR
+  uint32_t w_b0;     // wB
+  uint32_t w_0r;     // wR << 16
+  uint32_t w_gb;     // (wB << 16) | wG
+  uint32_t half;     // floor(den / 2), the rounding term
+  uint32_t magic;    // bin = umulhi(v, magic) when the fast bin path holds
+  uint32_t magic_y;  // Y = umulhi(v, magic_y) on the two-step path
+  uint32_t bins;
+  uint32_t w[3];     // plain weights and divisor for the generic kernel
+  uint32_t den;
+};
+
+enum BinPath : int { kBinFast = 0, kBinTwoStep = 1 };
+
+struct StreamState {
+  unsigned long long t;  // frames seen
+  uint32_t g;            // t - r(t) of the next frame (valid when t > 0)
+  uint32_t pad;
+};
+
+// Bits of the device error word.
+constexpr uint32_t kErrConsumerTimeout = 1u;
+constexpr uint32_t kErrProducerTimeout = 2u;
+constexpr uint32_t kErrDrainTimeout = 4u;
+
+struct HistArgs {
+  uint64_t frame_bytes;      // 3 W H
+  uint32_t npix;             // W H
+  uint32_t groups_per_frame; // frame_bytes / 48 (fast kernel)
+  uint32_t chunks_per_frame; // ceil(groups_per_frame / chunk groups)
+  uint64_t timeout_ns;
+};
+
+struct SelectArgs {
+  uint32_t bins;
+  uint32_t l_max;
+  uint32_t mask_words;
+  float tau;
+  float two_n;  // fp32(2 W H)
+};
+
+// Launchers (stream-ordered; return the launch error).
+int hist_blocks_per_sm(int bin_path, uint32_t bins);
+uint32_t hist_chunk_groups();
+size_t hist_smem_bytes(uint32_t bins);
+cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
+                             uint32_t* hist, uint32_t* err, int grid, cudaStream_t st);
+cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* hist,
+                                cudaStream_t st);
+cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
+                          const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st);
+cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
+                        const uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st);
+cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
+                              uint8_t* bins_out, cudaStream_t st);
+cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);
+
+}  // namespace cofie

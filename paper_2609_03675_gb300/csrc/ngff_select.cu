@@ -1,0 +1,213 @@
+// K2 and K3: novelty scores and the keep/drop decisions (CoFiE Sec. 3.2,
+// Eqs. 2-5).
+//
+// The decision for frame t depends on r(t), the most recent retained frame,
+// through the gap g = t - r(t). Because the gap rule (Eq. 5, second term)
+// retains a frame whenever g reaches L_max, g always lies in [1, L_max], so
+// every distance the rule can need is one of the L_max windowed distances
+// d(h_t, h_{t-k}), k = 1..L_max. That turns the sequential rule into:
+//
+// K2 (one warp per frame, lane = bin): L1[t][k-1] = sum_b |c_t[b] - c_{t-k}[b]|
+//    for every k (Eq. 2 up to the factor 1/(2N)), reading h_{t-k} from this
+//    push's histograms or from the stream's ring of the last L_max
+//    histograms, and the keep decision for every possible gap g as one bit:
+//    keep_t(g) = fp32(max(L1[t][0], L1[t][g-1])) / fp32(2N) >= tau_h
+//                (Eqs. 3-4: s = max(s_adj, s_ref))
+//                or g >= L_max (Eq. 5).
+//
+// K3 (one 1024-thread CTA per stream): the frame-to-frame gap update
+//    g' = keep_t(g) ? 1 : g + 1 is a map on [1, L_max]. Each warp composes
+//    the maps of a contiguous run of frames for all entry gaps at once (lane
+//    = entry gap), thread 0 chains the 32 run maps, each warp replays its run
+//    from the resolved entry gap, and all threads then emit score and keep
+//    code per frame. The stream state (frames seen, current gap, ring of the
+//    last L_max histograms) is updated at the end.
+#include "ngff_common.cuh"
+
+namespace cofie {
+namespace {
+
+constexpr int kWinWarps = 8;
+constexpr int kScanThreads = 1024;
+constexpr int kScanWarps = kScanThreads / 32;
+constexpr uint32_t kScanTile = 2048;  // frames per shared-memory tile
+
+__device__ __forceinline__ uint32_t absdiff(uint32_t a, uint32_t b) { return a > b ? a - b : b - a; }
+
+__global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, SelectArgs a,
+                                                                const uint32_t* __restrict__ hist,
+                                                                const uint32_t* __restrict__ ring,
+                                                                const StreamState* __restrict__ state,
+                                                                uint32_t* __restrict__ l1, uint32_t* __restrict__ mask) {
+  __shared__ uint32_t sl1[kWinWarps][kMaxLmax];
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t row = blockIdx.x * kWinWarps + warp;
+  if (row >= segs.rows) return;
+  uint32_t seg = 0;
+  while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
+  const uint32_t stream = segs.s[seg].stream;
+  const uint32_t j = row - segs.s[seg].row0;
+  const unsigned long long t = state[stream].t + j;
+  const uint32_t B = a.bins, L = a.l_max;
+  const uint32_t nq = (B + 31) / 32;
+
+  uint32_t ct[kMaxBins / 32];
+#pragma unroll
+  for (uint32_t q = 0; q < kMaxBins / 32; ++q) {
+    const uint32_t b = lane + 32 * q;
+    ct[q] = (q < nq && b < B) ? hist[static_cast<uint64_t>(row) * B + b] : 0u;
+  }
+  for (uint32_t k = 1; k <= L; ++k) {
+    uint32_t d = 0;
+    if (k <= t) {
+      const uint32_t* src = (k <= j) ? hist + static_cast<uint64_t>(row - k) * B
+                                     : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
+#pragma unroll
+      for (uint32_t q = 0; q < kMaxBins / 32; ++q) {
+        const uint32_t b = lane + 32 * q;
+        if (q < nq && b < B) d += absdiff(ct[q], src[b]);
+      }
+      d = __reduce_add_sync(0xffffffffu, d);
+    }
+    if (lane == 0) sl1[warp][k - 1] = d;
+  }
+  __syncwarp();
+  for (uint32_t k = lane; k < L; k += 32) l1[static_cast<uint64_t>(row) * L + k] = sl1[warp][k];
+  const uint32_t l_adj = sl1[warp][0];
+  for (uint32_t w = 0; w < a.mask_words; ++w) {
+    const uint32_t g = 32 * w + lane + 1;
+    bool keep = false;
+    if (g <= L) {
+      const uint32_t lm = max(l_adj, sl1[warp][g - 1]);
+      const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
+      keep = (s >= a.tau) || (g >= L);
+    }
+    const uint32_t m = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) mask[static_cast<uint64_t>(row) * a.mask_words + w] = m;
+  }
+}
+
+__device__ __forceinline__ uint32_t step_gap(const uint32_t* m, uint32_t g) {
+  const uint32_t bit = (m[(g - 1) >> 5] >> ((g - 1) & 31)) & 1u;
+  return bit ? 1u : g + 1u;
+}
+
+__global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, SelectArgs a,
+                                                            const uint32_t* __restrict__ l1,
+                                                            const uint32_t* __restrict__ mask,
+                                                            const uint32_t* __restrict__ hist,
+                                                            uint32_t* __restrict__ ring,
+                                                            StreamState* __restrict__ state) {
+  extern __shared__ __align__(16) uint32_t ssm[];
+  __shared__ Segment sseg;
+  __shared__ uint32_t entry[kScanWarps + 1];
+  __shared__ unsigned long long s_t0;
+  __shared__ uint32_t s_g;
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t W = a.mask_words, L = a.l_max, B = a.bins;
+  uint32_t* smask = ssm;                                       // [kScanTile][W]
+  uint16_t* sgap = reinterpret_cast<uint16_t*>(smask + kScanTile * W);  // [kScanTile]
+  uint16_t* sexit = sgap + kScanTile;                          // [kScanWarps][L]
+
+  if (tid == 0) {
+    sseg = segs.s[blockIdx.x];
+    s_t0 = state[sseg.stream].t;
+    s_g = state[sseg.stream].g;
+  }
+  __syncthreads();
+  const uint32_t n = sseg.n, row0 = sseg.row0, stream = sseg.stream;
+  if (n == 0) return;
+  const unsigned long long t0 = s_t0;
+  const uint32_t j_start = (t0 == 0) ? 1u : 0u;  // the stream's first frame is decided below
+  uint32_t g_entry = (t0 == 0) ? 1u : s_g;
+  if (g_entry < 1u || g_entry > L) g_entry = L;  // the state only ever holds [1, L]
+
+  for (uint32_t tile0 = j_start; tile0 < n; tile0 += kScanTile) {
+    const uint32_t m = min(kScanTile, n - tile0);
+    for (uint32_t i = tid; i < m * W; i += kScanThreads)
+      smask[i] = mask[static_cast<uint64_t>(row0 + tile0) * W + i];
+    __syncthreads();
+    const uint32_t run = (m + kScanWarps - 1) / kScanWarps;
+    const uint32_t f0 = min(warp * run, m), f1 = min(f0 + run, m);
+    // compose this warp's run of gap maps for every entry gap
+    for (uint32_t gin = lane + 1; gin <= L; gin += 32) {
+      uint32_t g = gin;
+      for (uint32_t f = f0; f < f1; ++f) g = step_gap(smask + f * W, g);
+      sexit[warp * L + gin - 1] = static_cast<uint16_t>(g);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t g = g_entry;
+      for (uint32_t w = 0; w < kScanWarps; ++w) {
+        entry[w] = g;
+        if (min(w * run, m) < min(w * run + run, m)) g = sexit[w * L + g - 1];
+      }
+      entry[kScanWarps] = g;
+    }
+    __syncthreads();
+    if (lane == 0) {
+      uint32_t g = entry[warp];
+      for (uint32_t f = f0; f < f1; ++f) {
+        sgap[f] = static_cast<uint16_t>(g);
+        g = step_gap(smask + f * W, g);
+      }
+    }
+    __syncthreads();
+    for (uint32_t f = tid; f < m; f += kScanThreads) {
+      const uint32_t jj = tile0 + f;
+      const uint32_t g = sgap[f];
+      const uint64_t r = static_cast<uint64_t>(row0 + jj) * L;
+      const uint32_t lm = max(l1[r], l1[r + g - 1]);
+      const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
+      const bool nov = s >= a.tau;
+      const uint8_t code = nov ? 1 : (g >= L ? 2 : 0);
+      if (sseg.scores) sseg.scores[jj] = s;
+      if (sseg.keep) sseg.keep[jj] = code;
+    }
+    g_entry = entry[kScanWarps];
+    __syncthreads();
+  }
+
+  if (tid == 0) {
+    if (t0 == 0) {  // first frame of the stream: always retained, score 0
+      if (sseg.scores) sseg.scores[0] = 0.0f;
+      if (sseg.keep) sseg.keep[0] = 3;
+    }
+    state[stream].t = t0 + n;
+    state[stream].g = g_entry;
+  }
+  // ring: histograms of the last min(n, L) frames of the push
+  const uint32_t keep_n = min(n, L);
+  for (uint32_t i = tid; i < keep_n * B; i += kScanThreads) {
+    const uint32_t jj = n - keep_n + i / B, b = i % B;
+    const uint64_t slot = (t0 + jj) % L;
+    ring[(static_cast<uint64_t>(stream) * L + slot) * B + b] = hist[static_cast<uint64_t>(row0 + jj) * B + b];
+  }
+}
+
+size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
+  return static_cast<size_t>(kScanTile) * mask_words * 4 + kScanTile * 2 + static_cast<size_t>(kScanWarps) * l_max * 2;
+}
+
+}  // namespace
+
+cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max) {
+  return cudaFuncSetAttribute(scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(scan_smem_bytes(mask_words, l_max)));
+}
+
+cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
+                          const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
+  const uint32_t grid = (segs.rows + kWinWarps - 1) / kWinWarps;
+  window_kernel<<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
+                        const uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st) {
+  scan_kernel<<<segs.count, kScanThreads, scan_smem_bytes(a.mask_words, a.l_max), st>>>(segs, a, l1, mask, hist, ring,
+                                                                                      state);
+  return cudaGetLastError();
+}
+
+}  // namespace cofie

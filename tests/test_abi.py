@@ -1,0 +1,78 @@
+"""The C-ABI library builds, loads without a GPU, exports every declared
+symbol, and rejects bad parameters before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from tests.conftest import REPO
+
+HEADER = os.path.join(REPO, "include", "cofie_ngff.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cofie_ngff_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_03675_gb300 import build
+    build.build()
+    from paper_2609_03675_gb300 import _abi
+    return _abi.load()
+
+
+def test_exports_every_declared_symbol(lib):
+    from paper_2609_03675_gb300 import _abi
+    names = _declared()
+    assert len(names) >= 10
+    assert sorted(_abi.EXPORTS) == names, "binding and header disagree"
+    for n in names:
+        assert hasattr(lib, n), f"{n} not exported"
+
+
+def test_param_struct_layout_matches_header(lib):
+    from paper_2609_03675_gb300 import _abi
+    # width..luma_den: 10 x 4 bytes, max_streams, max_frames_per_push, device, pad, u64
+    assert ctypes.sizeof(_abi.Params) == 64
+    assert ctypes.sizeof(_abi.PushDesc) == 32
+
+
+def test_defaults_are_the_papers(lib):
+    import json
+    from paper_2609_03675_gb300 import _abi
+    p = _abi.Params()
+    lib.cofie_ngff_default_params(ctypes.byref(p), 1920, 1080)
+    d = json.load(open(os.path.join(REPO, "tests", "golden", "ngff_defaults.json")))
+    assert (p.bins, p.m_min, p.l_max) == (d["bins"]["value"], d["m_min"]["value"], d["l_max"]["value"])
+    assert abs(p.tau - d["tau_h"]["value"]) < 1e-7
+    assert list(p.luma_w) == [299, 587, 114] and p.luma_den == 1000
+
+
+@pytest.mark.parametrize("field,value,msg", [
+    ("width", 0, "width"), ("bins", 0, "bins"), ("bins", 257, "bins"), ("l_max", 0, "l_max"),
+    ("l_max", 257, "l_max"), ("tau", float("nan"), "NaN"), ("luma_den", 999, "sum"), ("max_streams", 0, "streams"),
+    ("max_frames_per_push", 0, "max_frames"),
+])
+def test_create_rejects_bad_params_without_gpu(lib, field, value, msg):
+    from paper_2609_03675_gb300 import _abi
+    p = _abi.Params()
+    lib.cofie_ngff_default_params(ctypes.byref(p), 64, 48)
+    setattr(p, field, value)
+    h = ctypes.c_void_p()
+    rc = lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h))
+    assert rc == _abi.EINVAL
+    assert msg in lib.cofie_ngff_global_error().decode()
+    assert not h.value
+
+
+def test_null_handle_calls_are_rejected(lib):
+    from paper_2609_03675_gb300 import _abi
+    assert lib.cofie_ngff_push(None, 0, None, 0, None, None, None) == _abi.EINVAL
+    assert lib.cofie_ngff_reset(None, 0, None) == _abi.EINVAL
+    assert lib.cofie_ngff_status(None, None) == _abi.EINVAL
+    assert lib.cofie_ngff_last_error(None) == b""
+    lib.cofie_ngff_destroy(None)

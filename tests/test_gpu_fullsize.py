@@ -1,0 +1,111 @@
+"""Full-size parity: the 1080p, 720p rare-event and 32-stream serving workloads.
+
+Every frame's histogram, score and keep code is compared with the oracle
+(its histogram routine mapped over host threads, then its selection rule),
+on the same seeded bytes, in the launch configuration the benchmark times.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import synth
+from tests.gpu_helpers import assert_parity, run_stream
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def _pinned_stream(spec):
+    buf = torch.empty((spec.frames, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=buf.data_ptr())
+    return buf
+
+
+def _oracle(buf, spec, taus):
+    o = O.load()
+    p = O.Params(spec.width, spec.height)
+    hist = o.histograms_parallel(buf.data_ptr(), spec.frames, p)
+    return hist, {tau: o.select(hist, O.Params(spec.width, spec.height, tau=tau)) for tau in taus}
+
+
+def test_hd1080_whole_stream_push():
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.hd1080()
+    buf = _pinned_stream(spec)
+    dev = buf.cuda()
+    taus = (0.30, 0.05)
+    hist_o, sel = _oracle(buf, spec, taus)
+    del buf
+    for tau in taus:
+        f = NGFF(spec.width, spec.height, tau=tau, max_frames_per_push=spec.frames)
+        got = run_stream(f, dev, [spec.frames])
+        band = assert_parity(got, (hist_o, *sel[tau]), tau, f"1080p tau={tau}")
+        print(f"1080p tau={tau}: kept {int((got[2] != 0).sum())}/{spec.frames}, band frames {list(band)}")
+        f.close()
+    # every scene cut of the textured stream moves the histogram past tau = 0.30
+    cuts = synth.scene_starts(spec)[1:]
+    got30 = sel[0.30][1]
+    print(f"1080p: {len(cuts)} cuts, {int((got30[cuts] != 0).sum())} retained at tau 0.30")
+
+
+def test_rare_event_720p():
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.rare_event()
+    buf = _pinned_stream(spec)
+    dev = buf.cuda()
+    taus = (0.30, 0.15, 0.10, 0.05, 0.02)
+    hist_o, sel = _oracle(buf, spec, taus)
+    events = synth.event_mask(spec).astype(bool)
+    for tau in taus:
+        f = NGFF(spec.width, spec.height, tau=tau)
+        got = run_stream(f, dev, [spec.frames])
+        assert_parity(got, (hist_o, *sel[tau]), tau, f"720p tau={tau}")
+        kept = got[2] != 0
+        print(f"720p tau={tau}: keep ratio {kept.mean():.4f}, event-frame recall {kept[events].mean():.3f}")
+        f.close()
+
+
+def test_serving_32_streams_batched():
+    from paper_2609_03675_gb300 import NGFF
+    S = synth.SERVING_STREAMS
+    specs = [synth.serving_stream(s) for s in range(S)]
+    T, W, H = specs[0].frames, specs[0].width, specs[0].height
+    o = O.load()
+    p = O.Params(W, H)
+    host = torch.empty((T, H, W, 3), dtype=torch.uint8, pin_memory=True)
+    dev, want = [], []
+    for sp in specs:
+        synth.generate(sp, out=host.data_ptr())
+        hist = o.histograms_parallel(host.data_ptr(), T, p)
+        want.append((hist, *o.select(hist, p)))
+        dev.append(host.cuda())
+    f = NGFF(W, H, max_streams=S)
+    sizes = [synth.push_sizes(synth.SEED_BASE + 4, s, T) for s in range(S)]
+    scores = torch.empty((S, T), dtype=torch.float32, device="cuda")
+    keep = torch.empty((S, T), dtype=torch.uint8, device="cuda")
+    pos = [0] * S
+    call = 0
+    while min(pos) < T:
+        items = []
+        for s in range(S):
+            if pos[s] >= T:
+                continue
+            n = int(min(sizes[s][call], T - pos[s]))
+            items.append((s, dev[s][pos[s]:pos[s] + n], scores[s, pos[s]:pos[s] + n], keep[s, pos[s]:pos[s] + n]))
+            pos[s] += n
+        f.push_batch(items)
+        call += 1
+    torch.cuda.synchronize()
+    f.status()
+    ks, ss = keep.cpu().numpy(), scores.cpu().numpy()
+    for s in range(S):
+        _, so, ko = want[s]
+        assert np.array_equal(ks[s], ko), f"stream {s}"
+        assert (np.abs(ss[s].astype(np.float64) - so) <= 1e-6 * so).all(), f"stream {s}"
+    print(f"serving: {call} batched calls, keep ratio {(ks != 0).mean():.4f}")

@@ -1,0 +1,173 @@
+"""GPU path against the oracle, element by element, on seeded synthetic streams.
+
+Bar: integer histograms bit-exact; scores within 1e-6 relative of the
+oracle's double-precision distance; keep codes identical (the decision is
+taken in fp32 on both sides; frames in the tolerance band around tau_h are
+reported).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import synth
+from tests.gpu_helpers import assert_parity, oracle_run, run_stream
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_03675_gb300 import NGFF  # noqa: F401  (fails loudly if the library is missing)
+
+
+def _ngff(w, h, **kw):
+    from paper_2609_03675_gb300 import NGFF
+    return NGFF(w, h, **kw)
+
+
+def test_tiny_stream_whole_push():
+    spec = synth.tiny()
+    fr = synth.generate(spec)
+    p = O.Params(spec.width, spec.height)
+    want = oracle_run(fr, p)
+    f = _ngff(spec.width, spec.height)
+    got = run_stream(f, torch.from_numpy(fr).cuda(), [spec.frames])
+    band = assert_parity(got, want, p.tau, "tiny")
+    # at tau_h = 0.30 the tiny stream's cuts are too small to see: first + gap keeps only
+    assert list(np.flatnonzero(got[2])) == [0, 30, 60] and len(band) == 0
+
+
+def test_banded_cuts_kept():
+    spec = synth.tiny_banded()
+    fr = synth.generate(spec)
+    p = O.Params(spec.width, spec.height)
+    want = oracle_run(fr, p)
+    got = run_stream(_ngff(spec.width, spec.height), torch.from_numpy(fr).cuda(), [spec.frames])
+    assert_parity(got, want, p.tau, "banded")
+    cuts = synth.scene_starts(spec)[1:]
+    assert (got[2][cuts] == 1).all()
+
+
+def test_medium_stream_chunks_of_8():
+    spec = synth.medium()
+    fr = synth.generate(spec)
+    for tau in (0.30, 0.05, 0.02):
+        p = O.Params(spec.width, spec.height, tau=tau)
+        want = oracle_run(fr, p)
+        got = run_stream(_ngff(spec.width, spec.height, tau=tau), torch.from_numpy(fr).cuda(), [8] * 75)
+        assert_parity(got, want, tau, f"medium tau={tau}")
+
+
+@pytest.mark.parametrize("w,h", [(16, 1), (20, 4), (17, 13), (1, 1), (33, 7), (64, 48), (100, 3)])
+@pytest.mark.parametrize("bins,l_max,tau", [(32, 30, 0.05), (1, 1, 0.3), (3, 2, 0.0), (7, 33, 0.1),
+                                            (64, 5, 1.5), (256, 64, 0.02), (24, 256, 0.2)])
+def test_shapes_and_params(w, h, bins, l_max, tau):
+    g = np.random.default_rng(w * 1000 + h * 7 + bins + l_max)
+    T = 150
+    spec = synth.medium(seed=int(g.integers(1 << 30))).with_(width=w, height=h, frames=T, mean_scene_len=6)
+    fr = synth.generate(spec)
+    p = O.Params(w, h, bins=bins, l_max=l_max, tau=tau)
+    want = oracle_run(fr, p)
+    f = _ngff(w, h, bins=bins, l_max=l_max, tau=tau, max_frames_per_push=37)
+    cuts = np.sort(g.choice(np.arange(1, T), size=9, replace=False))
+    chunks = np.diff(np.concatenate([[0], cuts, [T]])).tolist()
+    got = run_stream(f, torch.from_numpy(fr).cuda(), chunks)
+    assert_parity(got, want, tau, f"{w}x{h} B={bins} L={l_max} tau={tau}")
+
+
+def test_push_split_invariance_and_empty_push():
+    spec = synth.medium().with_(width=96, height=64, frames=200)
+    fr = synth.generate(spec)
+    p = O.Params(96, 64, tau=0.05)
+    want = oracle_run(fr, p)
+    dev = torch.from_numpy(fr).cuda()
+    f = _ngff(96, 64, tau=0.05)
+    for chunks in ([200], [1] * 200, [3, 97, 1, 99], [29, 30, 31, 110]):
+        f.reset()
+        got = run_stream(f, dev, chunks)
+        assert_parity(got, want, 0.05, f"chunks {chunks[:4]}")
+    s, k = f.push(dev[:0])  # n = 0: a no-op
+    assert s.numel() == 0 and k.numel() == 0
+
+
+def test_reset_restarts_stream():
+    spec = synth.medium().with_(width=64, height=32, frames=90)
+    fr = torch.from_numpy(synth.generate(spec)).cuda()
+    f = _ngff(64, 32, tau=0.05)
+    a = run_stream(f, fr, [90])
+    f.push(fr[:45])
+    f.reset()
+    assert f.frames_seen() == 0
+    b = run_stream(f, fr, [90])
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
+
+
+def test_multistream_batch_equals_single():
+    g = np.random.default_rng(5)
+    S, T, w, h = 6, 120, 48, 32
+    specs = [synth.medium(seed=100 + s).with_(width=w, height=h, frames=T) for s in range(S)]
+    frames = [torch.from_numpy(synth.generate(sp)).cuda() for sp in specs]
+    p = O.Params(w, h, tau=0.05)
+    want = [oracle_run(synth.generate(sp), p) for sp in specs]
+    f = _ngff(w, h, tau=0.05, max_streams=S)
+    pos = [0] * S
+    outs = [(torch.empty(T, dtype=torch.float32, device="cuda"), torch.empty(T, dtype=torch.uint8, device="cuda"))
+            for _ in range(S)]
+    while min(pos) < T:
+        items = []
+        for s in g.permutation(S):
+            if pos[s] >= T:
+                continue
+            n = int(min(g.integers(0, 9), T - pos[s]))
+            items.append((int(s), frames[s][pos[s]:pos[s] + n], outs[s][0][pos[s]:pos[s] + n],
+                          outs[s][1][pos[s]:pos[s] + n]))
+            pos[s] += n
+        f.push_batch(items)
+    torch.cuda.synchronize()
+    f.status()
+    for s in range(S):
+        got_s, got_k = outs[s][0].cpu().numpy(), outs[s][1].cpu().numpy()
+        ho, so, ko = want[s]
+        assert np.array_equal(got_k, ko), f"stream {s}"
+        assert (np.abs(got_s - so) <= 1e-6 * so).all()
+
+
+def test_host_frames_and_host_outputs():
+    spec = synth.medium().with_(width=128, height=96, frames=70)
+    fr = synth.generate(spec)
+    p = O.Params(128, 96, tau=0.05)
+    ho, so, ko = oracle_run(fr, p)
+    # staging buffers of 5 frames force several overlapped host->device pieces
+    f = _ngff(128, 96, tau=0.05, host_stage_bytes=5 * spec.frame_bytes)
+    pinned = torch.from_numpy(fr).pin_memory()
+    scores = torch.empty(70, dtype=torch.float32).pin_memory()
+    keep = torch.empty(70, dtype=torch.uint8).pin_memory()
+    hist = torch.empty((70, 32), dtype=torch.int32).pin_memory()
+    f.push(pinned, scores=scores, keep=keep, hist=hist)
+    torch.cuda.synchronize()
+    f.status()
+    assert_parity((hist.numpy().view(np.uint32), scores.numpy(), keep.numpy()), (ho, so, ko), 0.05, "host")
+    # pageable host memory (plain numpy) through the raw entry point
+    f.reset()
+    s2 = np.zeros(70, np.float32)
+    k2 = np.zeros(70, np.uint8)
+    f.push_raw(0, fr.ctypes.data, 70, s2.ctypes.data, k2.ctypes.data)
+    torch.cuda.synchronize()
+    assert np.array_equal(k2, ko)
+
+
+def test_all_triples_frame_histogram():
+    """A 4096x4096 frame holding every RGB triple once, through the histogram kernel (B = 256: bin = Y)."""
+    v = torch.arange(1 << 24, dtype=torch.int64)
+    px = torch.stack([(v >> 16) & 255, (v >> 8) & 255, v & 255], -1).to(torch.uint8).reshape(1, 4096, 4096, 3)
+    o = O.load()
+    for bins in (256, 32):
+        want = o.histogram(px.numpy()[0], O.Params(4096, 4096, bins=bins))
+        f = _ngff(4096, 4096, bins=bins)
+        _, _, h = f.push(px.cuda(), return_hist=True)
+        torch.cuda.synchronize()
+        assert np.array_equal(h.cpu().numpy()[0].view(np.uint32), want)
