@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--frames", type=int, default=3600,
+                    help="use the first FRAMES frames of the stream (small cases for profiling; default all 3600)")
     return ap.parse_args()
 
 
@@ -162,6 +164,7 @@ def bench_gb300(args):
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     spec = synth.hd1080(seed=synth.SEED_BASE + 3 + rank)
+    spec = spec.with_(frames=min(spec.frames, max(1, args.frames)))
     T = spec.frames
     # inputs: generated on the host (pinned, kept for the end-to-end leg), resident in HBM for the timed region
     host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
@@ -250,7 +253,7 @@ def bench_gb300(args):
         fe.close()
 
     cpu = None
-    if rank == 0 and world == 1:
+    if rank == 0 and world == 1 and args.cpu_seconds > 0:
         k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds)
         cpu = {"value": k / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"first {k} frames of the 1080p stream, single-threaded C oracle (histograms + selection)"}
@@ -260,10 +263,10 @@ def bench_gb300(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u8", "data": "synthetic",
-            "config": {"workload": "1080p stream: 3600 uint8 RGB frames of 1920x1080 (HWC), one whole-stream push "
+            "config": {"workload": f"1080p stream: {T} uint8 RGB frames of 1920x1080 (HWC), one whole-stream push "
                                    "per step, B=32, L_max=30, tau_h=0.30",
                        "frames_per_step": T, "width": spec.width, "height": spec.height, "bins": 32, "l_max": 30,
-                       "tau": 0.30, "l2": "inputs larger than L2 (22.4 GB per step), no flush",
+                       "tau": 0.30, "l2": f"inputs larger than L2 ({T * spec.frame_bytes / 1e9:.1f} GB per step), no flush",
                        "parallelism": f"{world} independent stream(s), one per GPU"},
             "pixel_gbs": pixel_gbs,
             "frac_of_nominal_8tbs": pixel_gbs / NOMINAL_HBM_GBS,
