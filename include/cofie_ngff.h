@@ -203,6 +203,38 @@ int cofie_ngff_profile_reset(cofie_ngff_t* h, int time_kernels);
 /* Waits for the timed launches and writes the counters to *out. */
 int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out);
 
+/*
+ * Selection without device allocation (the paper has no counterpart: this is
+ * an interface for callers that may not allocate device memory, such as a
+ * process whose device memory belongs to another framework's pooling
+ * allocator under a hard cap, a media or ingest plugin that is handed buffers
+ * but may not allocate, or a latency-bound pipeline that fixes its memory at
+ * start-up because cudaMalloc can synchronise the device).
+ *
+ * Decides the first n frames of a fresh stream from their integer histograms
+ * and writes the same scores and keep codes cofie_ngff_push_ex gives on a new
+ * stream. Needs no handle and allocates nothing: its working tables live in a
+ * static device array of 1048576 32-bit words (4 MiB) that every GPU loading
+ * the library holds until the process exits.
+ *   p           width, height, bins, l_max and tau are used (the rest ignored).
+ *   hist        n * bins uint32 counts, row-major, device memory on the
+ *               current device (for example hist_out of cofie_ngff_push_ex).
+ *   n           frames; n * (l_max + ceil(l_max / 32)) must not exceed
+ *               1048576 (33825 frames at l_max = 30), else COFIE_EINVAL.
+ *   scores_out, keep_out
+ *               n floats / n bytes in device memory on the current device, or NULL.
+ *   err, err_cap  optional buffer that receives the error text (may be NULL).
+ * Runs on the calling thread's current device, asynchronously on cuda_stream.
+ * The first call on a device looks up the array's device address and sets
+ * the kernel's shared-memory limit (no allocation); make that first call
+ * before any stream capture. All calls share the array and it keeps the
+ * previous call's contents (each call overwrites every entry it reads), so
+ * calls that overlap on the GPU race: serialise them.
+ * Errors: COFIE_EINVAL, COFIE_ECUDA.
+ */
+int cofie_ngff_select_static(const cofie_ngff_params* p, const uint32_t* hist, uint32_t n, float* scores_out,
+                             uint8_t* keep_out, char* err, size_t err_cap, void* cuda_stream);
+
 /* Text of the last error on this handle (empty string if none). Never NULL. */
 const char* cofie_ngff_last_error(const cofie_ngff_t* h);
 

@@ -30,6 +30,7 @@ EXPORTS = (
     "cofie_ngff_debug_bins",
     "cofie_ngff_profile_reset",
     "cofie_ngff_profile_read",
+    "cofie_ngff_select_static",
     "cofie_ngff_last_error",
     "cofie_ngff_global_error",
 )
@@ -117,6 +118,8 @@ def load():
     lib.cofie_ngff_profile_reset.restype = ctypes.c_int
     lib.cofie_ngff_profile_read.argtypes = [H, ctypes.POINTER(Profile)]
     lib.cofie_ngff_profile_read.restype = ctypes.c_int
+    lib.cofie_ngff_select_static.argtypes = [P, vp, u32, vp, vp, ctypes.c_char_p, ctypes.c_size_t, vp]
+    lib.cofie_ngff_select_static.restype = ctypes.c_int
     lib.cofie_ngff_last_error.argtypes = [H]
     lib.cofie_ngff_last_error.restype = ctypes.c_char_p
     lib.cofie_ngff_global_error.argtypes = []
