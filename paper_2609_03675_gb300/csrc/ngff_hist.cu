@@ -11,7 +11,7 @@
 //   - one producer thread streams chunks HBM -> shared memory with 1-D bulk
 //     async copies (cp.async.bulk, the TMA engine) into a 4-stage ring
 //     guarded by mbarriers (full: transaction bytes, empty: consumer warps);
-//   - 8 consumer warps read 48-byte groups (16 RGB pixels) with three 128-bit
+//   - 4 consumer warps read 48-byte groups (16 RGB pixels) with three 128-bit
 //     shared loads at a 48-byte stride (conflict-free), form the luma sums
 //     with two dp2a per pixel, bin them with one multiply-high, and count
 //     into lane-private shared counters cnt[bin][lane] (bank = lane, so a
@@ -27,13 +27,32 @@
 namespace cofie {
 namespace {
 
-constexpr int kConsumerWarps = 8;
+// Tuning constants (compile-time overridable for sweeps). Measured on GB300
+// over the 1080p stream: 4 consumer warps (one per SM sub-partition) with two
+// CTAs per SM stream at ~7.59 TB/s; 3 or 5 warps (uneven over the
+// sub-partitions) lose 8-20 %, 8 warps lose 8 %, and any shape that leaves
+// one CTA per SM loses 25-40 %. The L2 evict-first hint makes no measurable
+// difference; the default policy is kept.
+#ifndef COFIE_K1_CONSUMER_WARPS
+#define COFIE_K1_CONSUMER_WARPS 4
+#endif
+#ifndef COFIE_K1_STAGES
+#define COFIE_K1_STAGES 4
+#endif
+#ifndef COFIE_K1_CHUNK_GROUPS
+#define COFIE_K1_CHUNK_GROUPS 512
+#endif
+#ifndef COFIE_K1_EVICT_FIRST
+#define COFIE_K1_EVICT_FIRST 0
+#endif
+
+constexpr int kConsumerWarps = COFIE_K1_CONSUMER_WARPS;
 constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kThreads = kConsumers + 32;  // + one producer warp
-constexpr int kStages = 4;
+constexpr int kStages = COFIE_K1_STAGES;
 constexpr int kGroupBytes = 48;            // 16 RGB pixels
-constexpr int kChunkGroups = 512;
-constexpr int kChunkBytes = kChunkGroups * kGroupBytes;  // 24 KiB
+constexpr int kChunkGroups = COFIE_K1_CHUNK_GROUPS;
+constexpr int kChunkBytes = kChunkGroups * kGroupBytes;  // 24 KiB by default
 
 struct SegLite {
   const uint8_t* frames;
@@ -87,9 +106,13 @@ __device__ __noinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, ui
   }
 }
 
-__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+__device__ __forceinline__ uint64_t l2_read_policy() {
   uint64_t pol;
+#if COFIE_K1_EVICT_FIRST
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+#else
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
+#endif
   return pol;
 }
 
@@ -196,7 +219,7 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
   if (warp == kConsumerWarps) {
     // ---------------------------------------------------------- producer --
     if (lane != 0) return;
-    const uint64_t pol = l2_evict_first_policy();
+    const uint64_t pol = l2_read_policy();
     const uint32_t ring0 = smem_u32(ring);
     ChunkCursor cur;
     cur.init(c0, cpf, sseg, nseg);

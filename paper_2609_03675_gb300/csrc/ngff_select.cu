@@ -30,7 +30,8 @@ namespace {
 constexpr int kWinWarps = 8;
 constexpr int kScanThreads = 1024;
 constexpr int kScanWarps = kScanThreads / 32;
-constexpr uint32_t kScanTile = 2048;  // frames per shared-memory tile
+constexpr uint32_t kScanTile = 4096;  // frames per shared-memory tile
+constexpr uint32_t kLagBatch = 8;     // lags whose loads K2 keeps in flight together
 
 __device__ __forceinline__ uint32_t absdiff(uint32_t a, uint32_t b) { return a > b ? a - b : b - a; }
 
@@ -57,19 +58,32 @@ __global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, S
     const uint32_t b = lane + 32 * q;
     ct[q] = (q < nq && b < B) ? hist[static_cast<uint64_t>(row) * B + b] : 0u;
   }
-  for (uint32_t k = 1; k <= L; ++k) {
-    uint32_t d = 0;
-    if (k <= t) {
-      const uint32_t* src = (k <= j) ? hist + static_cast<uint64_t>(row - k) * B
-                                     : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
+  // lags in groups of kLagBatch: the group's loads are independent and in
+  // flight together, then reduced one lag at a time
+  for (uint32_t k0 = 1; k0 <= L; k0 += kLagBatch) {
+    uint32_t dk[kLagBatch];
 #pragma unroll
-      for (uint32_t q = 0; q < kMaxBins / 32; ++q) {
-        const uint32_t b = lane + 32 * q;
-        if (q < nq && b < B) d += absdiff(ct[q], src[b]);
+    for (uint32_t u = 0; u < kLagBatch; ++u) {
+      const uint32_t k = k0 + u;
+      dk[u] = 0;
+      if (k <= L && k <= t) {
+        const uint32_t* src = (k <= j) ? hist + static_cast<uint64_t>(row - k) * B
+                                       : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
+#pragma unroll
+        for (uint32_t q = 0; q < kMaxBins / 32; ++q) {
+          const uint32_t b = lane + 32 * q;
+          if (q < nq && b < B) dk[u] += absdiff(ct[q], src[b]);
+        }
       }
-      d = __reduce_add_sync(0xffffffffu, d);
     }
-    if (lane == 0) sl1[warp][k - 1] = d;
+#pragma unroll
+    for (uint32_t u = 0; u < kLagBatch; ++u) {
+      const uint32_t k = k0 + u;
+      if (k <= L) {
+        const uint32_t d = (k <= t) ? __reduce_add_sync(0xffffffffu, dk[u]) : 0u;
+        if (lane == 0) sl1[warp][k - 1] = d;
+      }
+    }
   }
   __syncwarp();
   for (uint32_t k = lane; k < L; k += 32) l1[static_cast<uint64_t>(row) * L + k] = sl1[warp][k];
@@ -132,6 +146,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
     // compose this warp's run of gap maps for every entry gap
     for (uint32_t gin = lane + 1; gin <= L; gin += 32) {
       uint32_t g = gin;
+#pragma unroll 4
       for (uint32_t f = f0; f < f1; ++f) g = step_gap(smask + f * W, g);
       sexit[warp * L + gin - 1] = static_cast<uint16_t>(g);
     }
@@ -147,6 +162,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
     __syncthreads();
     if (lane == 0) {
       uint32_t g = entry[warp];
+#pragma unroll 4
       for (uint32_t f = f0; f < f1; ++f) {
         sgap[f] = static_cast<uint16_t>(g);
         g = step_gap(smask + f * W, g);
