@@ -234,6 +234,17 @@ def bench_gb300(args):
 
         estep()
         torch.cuda.synchronize()
+        # the raw host->device link, measured right before, to read the e2e figure against
+        nb = min(host.numel(), 4 << 30)
+        link_dst = torch.empty(nb, dtype=torch.uint8, device="cuda")
+        hflat = host.view(-1)[:nb]
+        link_dst.copy_(hflat, non_blocking=True)
+        torch.cuda.synchronize()
+        tl = time.perf_counter()
+        link_dst.copy_(hflat, non_blocking=True)
+        torch.cuda.synchronize()
+        link_gbs = nb / (time.perf_counter() - tl) / 1e9
+        del link_dst
         if world > 1:
             dist.barrier()
         t0 = time.perf_counter()
@@ -249,7 +260,8 @@ def bench_gb300(args):
         assert torch.equal(hk.to("cuda"), keep), "end-to-end keep codes differ from the device-resident run"
         e2e = {"value": args.e2e_steps * T * world / el, "unit": UNIT,
                "h2d_bytes_per_step": T * spec.frame_bytes, "d2h_bytes_per_step": T * (4 + 1),
-               "ms_per_step": el / args.e2e_steps * 1e3}
+               "ms_per_step": el / args.e2e_steps * 1e3, "h2d_link_gbs": link_gbs,
+               "h2d_achieved_gbs": T * spec.frame_bytes * args.e2e_steps / el / 1e9}
         fe.close()
 
     cpu = None
@@ -272,7 +284,8 @@ def bench_gb300(args):
             "frac_of_nominal_8tbs": pixel_gbs / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "peak_kind": f"{peak_kind} copy bandwidth", "traffic": traffic,
-                         "kernel": "ngff histogram (K1)", "launch_ms": k1_ms, "bytes_per_launch": k1_bytes},
+                         "kernel": "ngff histogram (K1)", "launch_ms": k1_ms, "bytes_per_launch": k1_bytes,
+                         "select_ms_per_step": prof["select_ms"] / max(prof["select_timed"], 1)},
             "e2e": e2e,
             "cpu_baseline": cpu,
             "gpu_launches": int(prof["hist_launches"] + prof["select_launches"]),

@@ -186,8 +186,9 @@ int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pix
 
 /*
  * Launch counters and kernel timing (a tracing aid). Counters run always;
- * with timing on, every launch of the histogram kernel is bracketed by two
- * CUDA events recorded on the stream it is launched on.
+ * with timing on, every launch of the histogram kernel, and every pair of
+ * distance + scan launches, is bracketed by two CUDA events recorded on the
+ * stream it is launched on.
  */
 typedef struct {
   uint64_t hist_launches;   /* histogram-kernel launches since the last reset */
@@ -195,6 +196,8 @@ typedef struct {
   uint64_t hist_bytes;      /* algorithmic bytes of those histogram launches: frame bytes read + counts written */
   uint64_t hist_timed;      /* histogram launches that were event-timed */
   double hist_ms;           /* summed event-timed histogram-kernel durations, milliseconds */
+  uint64_t select_timed;    /* distance + scan launch pairs that were event-timed */
+  double select_ms;         /* summed event-timed durations of those pairs, milliseconds */
 } cofie_ngff_profile;
 
 /* Zeroes the counters; time_kernels != 0 turns event timing on, 0 off. */

@@ -70,6 +70,8 @@ class Profile(ctypes.Structure):
         ("hist_bytes", ctypes.c_uint64),
         ("hist_timed", ctypes.c_uint64),
         ("hist_ms", ctypes.c_double),
+        ("select_timed", ctypes.c_uint64),
+        ("select_ms", ctypes.c_double),
     ]
 
 

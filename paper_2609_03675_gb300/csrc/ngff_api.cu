@@ -78,6 +78,8 @@ struct cofie_ngff {
   bool time_kernels = false;
   std::vector<cudaEvent_t> ev_pool;  // pairs: [2i] start, [2i+1] end
   size_t ev_used = 0;
+  std::vector<cudaEvent_t> ev_sel;  // the same for distance + scan pairs
+  size_t ev_sel_used = 0;
 
   int fail(int code, const std::string& msg) {
     err = msg;
@@ -141,6 +143,36 @@ cudaError_t dalloc(T** p, size_t count) {
   return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) + 16);
 }
 
+// Takes the next event pair from a pool (growing it up to kMaxTimedEvents).
+bool take_pair(std::vector<cudaEvent_t>& pool, size_t& used, cudaEvent_t* a, cudaEvent_t* b) {
+  if (used + 2 > kMaxTimedEvents) return false;
+  while (pool.size() < used + 2) {
+    cudaEvent_t ev;
+    if (cudaEventCreate(&ev) != cudaSuccess) return false;
+    pool.push_back(ev);
+  }
+  *a = pool[used];
+  *b = pool[used + 1];
+  used += 2;
+  return true;
+}
+
+double sum_pairs(const std::vector<cudaEvent_t>& pool, size_t used, cudaError_t* err) {
+  double ms = 0.0;
+  *err = cudaSuccess;
+  for (size_t i = 0; i + 1 < used; i += 2) {
+    cudaError_t e = cudaEventSynchronize(pool[i + 1]);
+    float t = 0.f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, pool[i], pool[i + 1]);
+    if (e != cudaSuccess) {
+      *err = e;
+      return 0.0;
+    }
+    ms += t;
+  }
+  return ms;
+}
+
 // Runs K1-K3 over the rows described by segs (device frames).
 int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
   if (segs.rows == 0) return COFIE_OK;
@@ -156,19 +188,7 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
   ha.chunks_per_frame = (ha.groups_per_frame + hist_chunk_groups() - 1) / hist_chunk_groups();
   ha.timeout_ns = kTimeoutNs;
   cudaEvent_t ev0 = nullptr, ev1 = nullptr;
-  if (h->time_kernels && h->ev_used + 2 <= kMaxTimedEvents) {
-    while (h->ev_pool.size() < h->ev_used + 2) {
-      cudaEvent_t ev;
-      if (cudaEventCreate(&ev) != cudaSuccess) break;
-      h->ev_pool.push_back(ev);
-    }
-    if (h->ev_pool.size() >= h->ev_used + 2) {
-      ev0 = h->ev_pool[h->ev_used];
-      ev1 = h->ev_pool[h->ev_used + 1];
-      h->ev_used += 2;
-      cudaEventRecord(ev0, st);
-    }
-  }
+  if (h->time_kernels && take_pair(h->ev_pool, h->ev_used, &ev0, &ev1)) cudaEventRecord(ev0, st);
   if (fast) {
     const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
     const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid);
@@ -186,10 +206,13 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
   sa.mask_words = h->mask_words;
   sa.tau = h->p.tau;
   sa.two_n = h->two_n;
+  cudaEvent_t es0 = nullptr, es1 = nullptr;
+  if (h->time_kernels && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
   e = launch_window(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "window kernel launch");
   e = launch_scan(segs, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "scan kernel launch");
+  if (es1) cudaEventRecord(es1, st);
   h->n_select += 2;
   return COFIE_OK;
 }
@@ -296,6 +319,7 @@ void free_handle(cofie_ngff* h) {
   for (void* b : bufs)
     if (b) cudaFree(b);
   for (cudaEvent_t ev : h->ev_pool) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : h->ev_sel) cudaEventDestroy(ev);
   for (int i = 0; i < 2; ++i) {
     if (h->ev_copied[i]) cudaEventDestroy(h->ev_copied[i]);
     if (h->ev_free[i]) cudaEventDestroy(h->ev_free[i]);
@@ -548,7 +572,7 @@ int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pix
 int cofie_ngff_profile_reset(cofie_ngff_t* h, int time_kernels) {
   if (!h) return COFIE_EINVAL;
   h->n_hist = h->n_select = h->hist_bytes = 0;
-  h->ev_used = 0;
+  h->ev_used = h->ev_sel_used = 0;
   h->time_kernels = time_kernels != 0;
   return COFIE_OK;
 }
@@ -556,19 +580,18 @@ int cofie_ngff_profile_reset(cofie_ngff_t* h, int time_kernels) {
 int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out) {
   if (!h || !out) return COFIE_EINVAL;
   DeviceGuard guard(h->device);
-  double ms = 0.0;
-  for (size_t i = 0; i + 1 < h->ev_used; i += 2) {
-    cudaError_t e = cudaEventSynchronize(h->ev_pool[i + 1]);
-    float t = 0.f;
-    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, h->ev_pool[i], h->ev_pool[i + 1]);
-    if (e != cudaSuccess) return h->cuda_fail(e, "kernel timing events");
-    ms += t;
-  }
+  cudaError_t e;
+  const double hist_ms = sum_pairs(h->ev_pool, h->ev_used, &e);
+  if (e != cudaSuccess) return h->cuda_fail(e, "kernel timing events");
+  const double sel_ms = sum_pairs(h->ev_sel, h->ev_sel_used, &e);
+  if (e != cudaSuccess) return h->cuda_fail(e, "kernel timing events");
   out->hist_launches = h->n_hist;
   out->select_launches = h->n_select;
   out->hist_bytes = h->hist_bytes;
   out->hist_timed = h->ev_used / 2;
-  out->hist_ms = ms;
+  out->hist_ms = hist_ms;
+  out->select_timed = h->ev_sel_used / 2;
+  out->select_ms = sel_ms;
   return COFIE_OK;
 }
 

@@ -7,7 +7,7 @@
 // every distance the rule can need is one of the L_max windowed distances
 // d(h_t, h_{t-k}), k = 1..L_max. That turns the sequential rule into:
 //
-// K2 (one warp per frame, lane = bin): L1[t][k-1] = sum_b |c_t[b] - c_{t-k}[b]|
+// K2 (one warp per frame, lane = lag): L1[t][k-1] = sum_b |c_t[b] - c_{t-k}[b]|
 //    for every k (Eq. 2 up to the factor 1/(2N)), reading h_{t-k} from this
 //    push's histograms or from the stream's ring of the last L_max
 //    histograms, and the keep decision for every possible gap g as one bit:
@@ -31,16 +31,19 @@ constexpr int kWinWarps = 8;
 constexpr int kScanThreads = 1024;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr uint32_t kScanTile = 4096;  // frames per shared-memory tile
-constexpr uint32_t kLagBatch = 8;     // lags whose loads K2 keeps in flight together
 
 __device__ __forceinline__ uint32_t absdiff(uint32_t a, uint32_t b) { return a > b ? a - b : b - a; }
 
+// One warp per frame; lane = lag: lane k-1 sums |c_t - c_{t-k}| over all
+// bins of row t-k (16-byte loads when B % 4 == 0), so the warp's loads are
+// independent and in flight together. The keep bit for gap g = k is decided
+// in the same lane.
+template <bool kVec4>
 __global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, SelectArgs a,
                                                                 const uint32_t* __restrict__ hist,
                                                                 const uint32_t* __restrict__ ring,
                                                                 const StreamState* __restrict__ state,
                                                                 uint32_t* __restrict__ l1, uint32_t* __restrict__ mask) {
-  __shared__ uint32_t sl1[kWinWarps][kMaxLmax];
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t row = blockIdx.x * kWinWarps + warp;
   if (row >= segs.rows) return;
@@ -50,62 +53,48 @@ __global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, S
   const uint32_t j = row - segs.s[seg].row0;
   const unsigned long long t = state[stream].t + j;
   const uint32_t B = a.bins, L = a.l_max;
-  const uint32_t nq = (B + 31) / 32;
-
-  uint32_t ct[kMaxBins / 32];
-#pragma unroll
-  for (uint32_t q = 0; q < kMaxBins / 32; ++q) {
-    const uint32_t b = lane + 32 * q;
-    ct[q] = (q < nq && b < B) ? hist[static_cast<uint64_t>(row) * B + b] : 0u;
-  }
-  // lags in groups of kLagBatch: the group's loads are independent and in
-  // flight together, then reduced one lag at a time
-  for (uint32_t k0 = 1; k0 <= L; k0 += kLagBatch) {
-    uint32_t dk[kLagBatch];
-#pragma unroll
-    for (uint32_t u = 0; u < kLagBatch; ++u) {
-      const uint32_t k = k0 + u;
-      dk[u] = 0;
-      if (k <= L && k <= t) {
-        const uint32_t* src = (k <= j) ? hist + static_cast<uint64_t>(row - k) * B
-                                       : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
-#pragma unroll
-        for (uint32_t q = 0; q < kMaxBins / 32; ++q) {
-          const uint32_t b = lane + 32 * q;
-          if (q < nq && b < B) dk[u] += absdiff(ct[q], src[b]);
-        }
-      }
-    }
-#pragma unroll
-    for (uint32_t u = 0; u < kLagBatch; ++u) {
-      const uint32_t k = k0 + u;
-      if (k <= L) {
-        const uint32_t d = (k <= t) ? __reduce_add_sync(0xffffffffu, dk[u]) : 0u;
-        if (lane == 0) sl1[warp][k - 1] = d;
-      }
-    }
-  }
-  __syncwarp();
-  for (uint32_t k = lane; k < L; k += 32) l1[static_cast<uint64_t>(row) * L + k] = sl1[warp][k];
-  const uint32_t l_adj = sl1[warp][0];
+  const uint32_t* ct = hist + static_cast<uint64_t>(row) * B;
+  uint32_t l_adj = 0;
   for (uint32_t w = 0; w < a.mask_words; ++w) {
-    const uint32_t g = 32 * w + lane + 1;
+    const uint32_t k = 32 * w + lane + 1;  // this lane's lag, and the gap it decides
+    const bool valid = k <= L && k <= t;
+    const uint32_t* src = ct;
+    if (valid)
+      src = (k <= j) ? hist + static_cast<uint64_t>(row - k) * B
+                     : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
+    uint32_t d = 0;
+    if (kVec4) {
+      const uint4* c4 = reinterpret_cast<const uint4*>(ct);
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+#pragma unroll 8
+      for (uint32_t q = 0; q < B / 4; ++q) {
+        const uint4 x = c4[q], y = s4[q];
+        d += absdiff(x.x, y.x) + absdiff(x.y, y.y) + absdiff(x.z, y.z) + absdiff(x.w, y.w);
+      }
+    } else {
+#pragma unroll 4
+      for (uint32_t b = 0; b < B; ++b) d += absdiff(ct[b], src[b]);
+    }
+    if (!valid) d = 0;
+    if (w == 0) l_adj = __shfl_sync(0xffffffffu, d, 0);  // lag 1
+    if (k <= L) l1[static_cast<uint64_t>(row) * L + k - 1] = d;
     bool keep = false;
-    if (g <= L) {
-      const uint32_t lm = max(l_adj, sl1[warp][g - 1]);
-      const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
-      keep = (s >= a.tau) || (g >= L);
+    if (k <= L) {
+      const float s = __fdiv_rn(static_cast<float>(max(l_adj, d)), a.two_n);
+      keep = (s >= a.tau) || (k >= L);
     }
     const uint32_t m = __ballot_sync(0xffffffffu, keep);
     if (lane == 0) mask[static_cast<uint64_t>(row) * a.mask_words + w] = m;
   }
 }
 
+template <bool kOneWord>
 __device__ __forceinline__ uint32_t step_gap(const uint32_t* m, uint32_t g) {
-  const uint32_t bit = (m[(g - 1) >> 5] >> ((g - 1) & 31)) & 1u;
-  return bit ? 1u : g + 1u;
+  const uint32_t word = kOneWord ? m[0] : m[(g - 1) >> 5];
+  return ((word >> ((g - 1) & 31)) & 1u) ? 1u : g + 1u;
 }
 
+template <bool kOneWord>
 __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, SelectArgs a,
                                                             const uint32_t* __restrict__ l1,
                                                             const uint32_t* __restrict__ mask,
@@ -147,7 +136,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
     for (uint32_t gin = lane + 1; gin <= L; gin += 32) {
       uint32_t g = gin;
 #pragma unroll 4
-      for (uint32_t f = f0; f < f1; ++f) g = step_gap(smask + f * W, g);
+      for (uint32_t f = f0; f < f1; ++f) g = step_gap<kOneWord>(smask + f * W, g);
       sexit[warp * L + gin - 1] = static_cast<uint16_t>(g);
     }
     __syncthreads();
@@ -165,10 +154,11 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
 #pragma unroll 4
       for (uint32_t f = f0; f < f1; ++f) {
         sgap[f] = static_cast<uint16_t>(g);
-        g = step_gap(smask + f * W, g);
+        g = step_gap<kOneWord>(smask + f * W, g);
       }
     }
     __syncthreads();
+#pragma unroll 4
     for (uint32_t f = tid; f < m; f += kScanThreads) {
       const uint32_t jj = tile0 + f;
       const uint32_t g = sgap[f];
@@ -208,21 +198,28 @@ size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
 }  // namespace
 
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max) {
-  return cudaFuncSetAttribute(scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(scan_smem_bytes(mask_words, l_max)));
+  const int smem = static_cast<int>(scan_smem_bytes(mask_words, l_max));
+  return mask_words == 1 ? cudaFuncSetAttribute(scan_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)
+                         : cudaFuncSetAttribute(scan_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
 }
 
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
                           const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
   const uint32_t grid = (segs.rows + kWinWarps - 1) / kWinWarps;
-  window_kernel<<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
+  if (a.bins % 4 == 0)
+    window_kernel<true><<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
+  else
+    window_kernel<false><<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
   return cudaGetLastError();
 }
 
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
                         const uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st) {
-  scan_kernel<<<segs.count, kScanThreads, scan_smem_bytes(a.mask_words, a.l_max), st>>>(segs, a, l1, mask, hist, ring,
-                                                                                      state);
+  const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
+  if (a.mask_words == 1)
+    scan_kernel<true><<<segs.count, kScanThreads, smem, st>>>(segs, a, l1, mask, hist, ring, state);
+  else
+    scan_kernel<false><<<segs.count, kScanThreads, smem, st>>>(segs, a, l1, mask, hist, ring, state);
   return cudaGetLastError();
 }
 
