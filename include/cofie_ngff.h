@@ -55,6 +55,7 @@ extern "C" {
 #define COFIE_ENOMEM 2   /* a device or pinned-host allocation failed */
 #define COFIE_ECUDA 3    /* a CUDA runtime call failed */
 #define COFIE_ETIMEOUT 4 /* a device-side bounded wait ran out (cofie_ngff_status) */
+#define COFIE_EDEVICE 5  /* a device-side check failed: a gather index outside the frames (cofie_ngff_status) */
 
 /* Keep codes written to keep_out. Nonzero means retained (a candidate). */
 #define COFIE_KEEP_DROP 0
@@ -156,14 +157,45 @@ int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, 
  */
 int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream);
 
+/*
+ * Closes a prefix of T frames (Sec. 3.2, the safeguards that need the end of
+ * the prefix) and writes its candidate set S_c as ascending frame indices:
+ * every frame with a nonzero keep code, the last frame T-1, and -- when that
+ * leaves fewer than M_min frames -- the uniformly spaced frames
+ * round(i (T-1) / (M_min - 1)), i = 0..M_min-1, rounded half up.
+ *   keep     T keep codes of frames 0..T-1 (the concatenated keep_out of the
+ *            stream's pushes), device memory.
+ *   idx_out  room for T uint32 indices, device memory.
+ *   m_out    |S_c|, device memory (asynchronous) or host memory (the call then
+ *            synchronises cuda_stream).
+ * M_min is the handle's m_min. T == 0 gives |S_c| = 0. Errors: COFIE_EINVAL,
+ * COFIE_ECUDA.
+ */
+int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out, uint32_t* m_out,
+                          void* cuda_stream);
+
+/*
+ * Copies the m frames idx[0..m) of `frames` back to back into `out`: the
+ * frames S_c that go on to the vision encoder (Sec. 3.2, "only these m frames
+ * are sent to the encoder").
+ *   frames   n_frames frames of 3 W H bytes, device memory.
+ *   idx      m frame indices, device memory (for example cofie_ngff_candidates' idx_out).
+ *   out      m * 3 W H bytes, device memory, not overlapping frames.
+ * An index >= n_frames is skipped and reported as COFIE_EDEVICE by
+ * cofie_ngff_status. Errors: COFIE_EINVAL, COFIE_ECUDA.
+ */
+int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames, const uint32_t* idx, uint32_t m,
+                      uint8_t* out, void* cuda_stream);
+
 /* Restarts stream `stream` at t = 0 (its next frame is a first frame). */
 int cofie_ngff_reset(cofie_ngff_t* h, uint32_t stream, void* cuda_stream);
 
 /*
  * Synchronises cuda_stream and reports device-side failures of earlier
  * calls on the handle: COFIE_ETIMEOUT if a bounded wait inside a kernel ran
- * out (the affected results are invalid), COFIE_ECUDA on a CUDA error,
- * COFIE_OK otherwise. Clears the device error word.
+ * out (the affected results are invalid), COFIE_EDEVICE if a gather index
+ * was outside its frames, COFIE_ECUDA on a CUDA error, COFIE_OK otherwise.
+ * Clears the device error word.
  */
 int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream);
 

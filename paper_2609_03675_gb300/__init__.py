@@ -124,6 +124,27 @@ class NGFF:
             arr[i].frames, arr[i].scores_out, arr[i].keep_out = _ptr(frames), _ptr(scores), _ptr(keep)
         self._check(self._lib.cofie_ngff_push_batch(self._h, arr, len(items), self._stream(cuda_stream)))
 
+    def candidates(self, keep: torch.Tensor, cuda_stream=None) -> torch.Tensor:
+        """S_c of a closed prefix: ascending indices of the retained frames, the
+        last frame, and the M_min uniform fill (cuda uint8 keep codes in, cuda
+        int32 indices out; synchronises to read the count)."""
+        T = keep.numel()
+        idx = torch.empty(max(T, 1), dtype=torch.int32, device=self.device)
+        m = ctypes.c_uint32(0)
+        self._check(self._lib.cofie_ngff_candidates(self._h, _ptr(keep), T, _ptr(idx), ctypes.addressof(m),
+                                                    self._stream(cuda_stream)))
+        return idx[: m.value]
+
+    def gather(self, frames: torch.Tensor, idx: torch.Tensor, out: torch.Tensor | None = None, cuda_stream=None):
+        """frames[idx] back to back (cuda uint8 [m, H, W, 3]): the encoder's input."""
+        n = self._frames(frames)
+        m = idx.numel()
+        if out is None:
+            out = torch.empty((m, self.height, self.width, 3), dtype=torch.uint8, device=self.device)
+        self._check(self._lib.cofie_ngff_gather(self._h, _ptr(frames), n, _ptr(idx), m, _ptr(out),
+                                                self._stream(cuda_stream)))
+        return out
+
     def reset(self, stream: int = 0, cuda_stream=None):
         self._check(self._lib.cofie_ngff_reset(self._h, stream, self._stream(cuda_stream)))
 

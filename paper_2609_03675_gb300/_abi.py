@@ -12,7 +12,7 @@ import os
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libcofie_ngff.so")
 
-OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT = 0, 1, 2, 3, 4
+OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE = 0, 1, 2, 3, 4, 5
 KEEP_DROP, KEEP_NOVELTY, KEEP_GAP, KEEP_FIRST = 0, 1, 2, 3
 MAX_BINS, MAX_LMAX, MAX_BATCH = 256, 256, 64
 
@@ -24,6 +24,8 @@ EXPORTS = (
     "cofie_ngff_push",
     "cofie_ngff_push_ex",
     "cofie_ngff_push_batch",
+    "cofie_ngff_candidates",
+    "cofie_ngff_gather",
     "cofie_ngff_reset",
     "cofie_ngff_status",
     "cofie_ngff_frames_seen",
@@ -108,6 +110,10 @@ def load():
     lib.cofie_ngff_push_ex.restype = ctypes.c_int
     lib.cofie_ngff_push_batch.argtypes = [H, ctypes.POINTER(PushDesc), u32, vp]
     lib.cofie_ngff_push_batch.restype = ctypes.c_int
+    lib.cofie_ngff_candidates.argtypes = [H, vp, u32, vp, vp, vp]
+    lib.cofie_ngff_candidates.restype = ctypes.c_int
+    lib.cofie_ngff_gather.argtypes = [H, vp, u32, vp, u32, vp, vp]
+    lib.cofie_ngff_gather.restype = ctypes.c_int
     lib.cofie_ngff_reset.argtypes = [H, u32, vp]
     lib.cofie_ngff_reset.restype = ctypes.c_int
     lib.cofie_ngff_status.argtypes = [H, vp]

@@ -64,6 +64,7 @@ struct cofie_ngff {
   float* d_scores = nullptr;
   uint8_t* d_keep = nullptr;
   uint32_t* d_err = nullptr;
+  uint32_t* d_count = nullptr;  // candidate count when the caller's m_out is host memory
   uint8_t* d_stage[2] = {nullptr, nullptr};
   uint64_t stage_bytes = 0;
   uint32_t stage_frames = 0;
@@ -315,7 +316,7 @@ void free_handle(cofie_ngff* h) {
   DeviceGuard guard(h->device);
   cudaDeviceSynchronize();
   void* bufs[] = {h->d_hist, h->d_l1, h->d_mask, h->d_ring, h->d_state, h->d_scores,
-                  h->d_keep, h->d_err,  h->d_stage[0], h->d_stage[1]};
+                  h->d_keep, h->d_err,  h->d_stage[0], h->d_stage[1], h->d_count};
   for (void* b : bufs)
     if (b) cudaFree(b);
   for (cudaEvent_t ev : h->ev_pool) cudaEventDestroy(ev);
@@ -434,6 +435,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   if (e == cudaSuccess) e = dalloc(&h->d_scores, F);
   if (e == cudaSuccess) e = dalloc(&h->d_keep, F);
   if (e == cudaSuccess) e = dalloc(&h->d_err, 1);
+  if (e == cudaSuccess) e = dalloc(&h->d_count, 1);
   if (e != cudaSuccess) {
     cudaGetLastError();
     free_handle(h);
@@ -541,9 +543,12 @@ int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream) {
   if (e != cudaSuccess) return h->cuda_fail(e, "error word read");
   if (word) {
     cudaMemset(h->d_err, 0, sizeof word);
-    char buf[96];
-    snprintf(buf, sizeof buf, "device-side wait ran out (error bits 0x%x)", word);
-    return h->fail(COFIE_ETIMEOUT, buf);
+    char buf[128];
+    snprintf(buf, sizeof buf, "device-side failure (error bits 0x%x: 1/2/4 a wait ran out, 8 a bad gather index)",
+             word);
+    return h->fail((word & (kErrConsumerTimeout | kErrProducerTimeout | kErrDrainTimeout)) ? COFIE_ETIMEOUT
+                                                                                          : COFIE_EDEVICE,
+                   buf);
   }
   return COFIE_OK;
 }
@@ -566,6 +571,51 @@ int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pix
   cudaError_t e = launch_debug_bins(pixels, n_pixels / 4, h->lc, h->bin_path, bins_out,
                                     static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return h->cuda_fail(e, "debug kernel launch");
+  return COFIE_OK;
+}
+
+int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out, uint32_t* m_out,
+                          void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (!m_out) return h->fail(COFIE_EINVAL, "m_out is NULL");
+  DeviceGuard guard(h->device);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const MemKind km = classify(m_out);
+  if (T == 0) {
+    if (km == kDevice) {
+      cudaError_t e = cudaMemsetAsync(m_out, 0, sizeof(uint32_t), st);
+      return e == cudaSuccess ? COFIE_OK : h->cuda_fail(e, "candidates count");
+    }
+    *m_out = 0;
+    return COFIE_OK;
+  }
+  int dk = -1, di = -1;
+  if (!keep || !idx_out || classify(keep, &dk) != kDevice || classify(idx_out, &di) != kDevice || dk != h->device ||
+      di != h->device)
+    return h->fail(COFIE_EINVAL, "keep and idx_out must be device memory on the handle's device");
+  uint32_t* count = km == kDevice ? m_out : h->d_count;
+  cudaError_t e = launch_candidates(keep, T, h->p.m_min, idx_out, count, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "candidates kernel launch");
+  if (km != kDevice) {
+    e = cudaMemcpyAsync(m_out, count, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "candidates count");
+  }
+  return COFIE_OK;
+}
+
+int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames, const uint32_t* idx, uint32_t m,
+                      uint8_t* out, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (m == 0) return COFIE_OK;
+  int d0 = -1, d1 = -1, d2 = -1;
+  if (!frames || !idx || !out || classify(frames, &d0) != kDevice || classify(idx, &d1) != kDevice ||
+      classify(out, &d2) != kDevice || d0 != h->device || d1 != h->device || d2 != h->device)
+    return h->fail(COFIE_EINVAL, "frames, idx and out must be device memory on the handle's device");
+  DeviceGuard guard(h->device);
+  cudaError_t e = launch_gather(frames, n_frames, h->frame_bytes, idx, m, out, h->d_err,
+                                static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return h->cuda_fail(e, "gather kernel launch");
   return COFIE_OK;
 }
 

@@ -63,6 +63,7 @@ struct StreamState {
 constexpr uint32_t kErrConsumerTimeout = 1u;
 constexpr uint32_t kErrProducerTimeout = 2u;
 constexpr uint32_t kErrDrainTimeout = 4u;
+constexpr uint32_t kErrBadIndex = 8u;  // a gather index outside the frame buffer
 
 struct HistArgs {
   uint64_t frame_bytes;      // 3 W H
@@ -95,5 +96,9 @@ cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);
+cudaError_t launch_candidates(const uint8_t* keep, uint32_t T, uint32_t m_min, uint32_t* idx, uint32_t* m_out,
+                              cudaStream_t st);
+cudaError_t launch_gather(const uint8_t* frames, uint32_t n_frames, uint64_t frame_bytes, const uint32_t* idx, uint32_t m,
+                          uint8_t* out, uint32_t* err, cudaStream_t st);
 
 }  // namespace cofie

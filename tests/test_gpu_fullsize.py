@@ -41,13 +41,22 @@ def test_hd1080_whole_stream_push():
     dev = buf.cuda()
     taus = (0.30, 0.05)
     hist_o, sel = _oracle(buf, spec, taus)
-    del buf
     for tau in taus:
         f = NGFF(spec.width, spec.height, tau=tau, max_frames_per_push=spec.frames)
         got = run_stream(f, dev, [spec.frames])
         band = assert_parity(got, (hist_o, *sel[tau]), tau, f"1080p tau={tau}")
         print(f"1080p tau={tau}: kept {int((got[2] != 0).sum())}/{spec.frames}, band frames {list(band)}")
+        # close the prefix and gather the encoder's input
+        idx = f.candidates(torch.from_numpy(got[2]).cuda())
+        want_idx = O.load().candidates(sel[tau][1], 4)
+        assert np.array_equal(idx.cpu().numpy().astype(np.uint32), want_idx)
+        out = f.gather(dev, idx)
+        torch.cuda.synchronize()
+        f.status()
+        assert torch.equal(out.cpu(), buf[torch.from_numpy(want_idx.astype(np.int64))])
+        del out
         f.close()
+    del buf
     # every scene cut of the textured stream moves the histogram past tau = 0.30
     cuts = synth.scene_starts(spec)[1:]
     got30 = sel[0.30][1]
