@@ -45,6 +45,9 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather"], default="hd1080",
+                    help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
+                         "finalize + gather bandwidth)")
     ap.add_argument("--frames", type=int, default=3600,
                     help="use the first FRAMES frames of the stream (small cases for profiling; default all 3600)")
     return ap.parse_args()
@@ -52,6 +55,28 @@ def parse():
 
 def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def stream_seed(rank: int) -> int:
+    """Each rank filters its own independently seeded 1080p stream."""
+    import synth
+    return synth.SEED_BASE + 3 + rank
+
+
+def max_over_ranks(x: float, device="cuda") -> float:
+    """The largest value of x over all ranks (a no-op without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, world: int, seconds_max: float) -> float:
+    """Whole-job throughput: the units all ranks processed over the slowest rank's time."""
+    return units_per_rank * world / seconds_max
 
 
 def peaks():
@@ -163,7 +188,7 @@ def bench_gb300(args):
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    spec = synth.hd1080(seed=synth.SEED_BASE + 3 + rank)
+    spec = synth.hd1080(seed=stream_seed(rank))
     spec = spec.with_(frames=min(spec.frames, max(1, args.frames)))
     T = spec.frames
     # inputs: generated on the host (pinned, kept for the end-to-end leg), resident in HBM for the timed region
@@ -201,16 +226,13 @@ def bench_gb300(args):
             dist.barrier()
     f.status()
     prof = f.profile_read()
-    ms = start.elapsed_time(end)
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(start.elapsed_time(end))
     clocks = clk.summary()
+    clocks["gpu_uuid"] = gpu_id
     kept = int((keep != 0).sum().item())
 
     frames_total = args.steps * T * world
-    value = frames_total / (ms / 1e3)
+    value = whole_job_rate(args.steps * T, world, ms / 1e3)
     pixel_gbs = frames_total * spec.frame_bytes / (ms / 1e3) / 1e9
 
     # roofline of the dominant kernel (histogram): algorithmic bytes per launch / mean event-timed duration
@@ -234,33 +256,31 @@ def bench_gb300(args):
 
         estep()
         torch.cuda.synchronize()
-        # the raw host->device link, measured right before, to read the e2e figure against
-        nb = min(host.numel(), 4 << 30)
-        link_dst = torch.empty(nb, dtype=torch.uint8, device="cuda")
-        hflat = host.view(-1)[:nb]
-        link_dst.copy_(hflat, non_blocking=True)
-        torch.cuda.synchronize()
-        tl = time.perf_counter()
-        link_dst.copy_(hflat, non_blocking=True)
-        torch.cuda.synchronize()
-        link_gbs = nb / (time.perf_counter() - tl) / 1e9
-        del link_dst
+        # the raw host->device link over the same bytes (one plain copy of the
+        # whole pinned stream into the device frame tensor), measured right
+        # before and right after the end-to-end steps, to read the e2e figure against
+        def link():
+            torch.cuda.synchronize()
+            tl = time.perf_counter()
+            dev.copy_(host, non_blocking=True)
+            torch.cuda.synchronize()
+            return host.numel() / (time.perf_counter() - tl) / 1e9
+
+        link_before = link()
         if world > 1:
             dist.barrier()
         t0 = time.perf_counter()
         for _ in range(args.e2e_steps):
             estep()
         torch.cuda.synchronize()
-        el = time.perf_counter() - t0
-        if world > 1:
-            tt = torch.tensor([el], device="cuda")
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            el = float(tt.item())
+        el = max_over_ranks(time.perf_counter() - t0)
+        link_after = link()
         fe.status()
         assert torch.equal(hk.to("cuda"), keep), "end-to-end keep codes differ from the device-resident run"
-        e2e = {"value": args.e2e_steps * T * world / el, "unit": UNIT,
+        e2e = {"value": whole_job_rate(args.e2e_steps * T, world, el), "unit": UNIT,
                "h2d_bytes_per_step": T * spec.frame_bytes, "d2h_bytes_per_step": T * (4 + 1),
-               "ms_per_step": el / args.e2e_steps * 1e3, "h2d_link_gbs": link_gbs,
+               "ms_per_step": el / args.e2e_steps * 1e3, "h2d_link_gbs_before": link_before,
+               "h2d_link_gbs_after": link_after,
                "h2d_achieved_gbs": T * spec.frame_bytes * args.e2e_steps / el / 1e9}
         fe.close()
 
@@ -335,10 +355,236 @@ def bench_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def _pct(xs, q):
+    import numpy as np
+    return float(np.percentile(np.asarray(xs), q))
+
+
+def bench_serving(args):
+    """32 concurrent 640x360 streams, each call pushing U{1..8} new frames per
+    stream in one batched launch sequence: per-call latency (synchronised
+    calls) and pipelined aggregate frames/s."""
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    S = synth.SERVING_STREAMS
+    specs = [synth.serving_stream(s) for s in range(S)]
+    T, W, H = specs[0].frames, specs[0].width, specs[0].height
+    host = torch.empty((T, H, W, 3), dtype=torch.uint8, pin_memory=True)
+    dev = []
+    for sp in specs:
+        synth.generate(sp, out=host.data_ptr())
+        dev.append(host.cuda())
+    sizes = [synth.push_sizes(synth.SEED_BASE + 4, s, T) for s in range(S)]
+    scores = torch.empty((S, T), dtype=torch.float32, device="cuda")
+    keep = torch.empty((S, T), dtype=torch.uint8, device="cuda")
+    f = NGFF(W, H, max_streams=S)
+
+    def calls():
+        pos, call, out = [0] * S, 0, []
+        while min(pos) < T:
+            items = []
+            for s in range(S):
+                if pos[s] >= T:
+                    continue
+                n = int(min(sizes[s][call], T - pos[s]))
+                items.append((s, dev[s][pos[s]:pos[s] + n], scores[s, pos[s]:pos[s] + n], keep[s, pos[s]:pos[s] + n]))
+                pos[s] += n
+            out.append(items)
+            call += 1
+        return out
+
+    plan = [f.make_batch(items) for items in calls()]  # descriptors marshalled once, outside the timing
+    frames_total = S * T
+    st = torch.cuda.current_stream().cuda_stream
+
+    def run(sync_each):
+        for s in range(S):
+            f.reset(s)
+        lat = []
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for arr, nd in plan:
+            c0 = time.perf_counter()
+            f.push_batch_raw(arr, nd, st)
+            if sync_each:
+                torch.cuda.synchronize()
+                lat.append((time.perf_counter() - c0) * 1e3)
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0, lat
+
+    for _ in range(max(1, args.warmup // 3)):
+        run(False)
+    el_pipe, _ = run(False)
+    el_sync, lat = run(True)
+    f.status()
+    line = {"workload": "serving: 32 streams x 1800 frames of 640x360, U{1..8} frames per stream per batched call",
+            "calls": len(plan), "frames": frames_total,
+            "pipelined_frames_per_s": frames_total / el_pipe, "pipelined_ms_per_call": el_pipe / len(plan) * 1e3,
+            "sync_frames_per_s": frames_total / el_sync,
+            "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99), "latency_ms_max": max(lat),
+            "latency": "host wall time of one push_batch call plus a device synchronise",
+            "keep_ratio": float((keep != 0).float().mean().item())}
+    print(json.dumps(line), flush=True)
+
+
+def bench_medium(args):
+    """600 frames of 448x448 pushed 8 at a time: per-push latency and frames/s."""
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.medium()
+    dev = torch.from_numpy(synth.generate(spec)).cuda()
+    scores = torch.empty(spec.frames, dtype=torch.float32, device="cuda")
+    keep = torch.empty(spec.frames, dtype=torch.uint8, device="cuda")
+    f = NGFF(spec.width, spec.height)
+    st = torch.cuda.current_stream().cuda_stream
+    fb = spec.frame_bytes
+    ptrs = [(dev.data_ptr() + i * fb, scores.data_ptr() + 4 * i, keep.data_ptr() + i) for i in range(0, spec.frames, 8)]
+
+    def run(sync_each):
+        f.reset()
+        lat = []
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for fp, sp, kp in ptrs:
+            c0 = time.perf_counter()
+            f.push_raw(0, fp, 8, sp, kp, None, st)
+            if sync_each:
+                torch.cuda.synchronize()
+                lat.append((time.perf_counter() - c0) * 1e3)
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0, lat
+
+    for _ in range(max(1, args.warmup)):
+        run(False)
+    el_pipe, _ = run(False)
+    el_sync, lat = run(True)
+    f.status()
+    print(json.dumps({"workload": "medium: 600 frames of 448x448 pushed in chunks of 8", "pushes": len(lat),
+                      "pipelined_frames_per_s": spec.frames / el_pipe, "sync_frames_per_s": spec.frames / el_sync,
+                      "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99),
+                      "latency": "host wall time of one push plus a device synchronise",
+                      "kept": int((keep != 0).sum().item())}), flush=True)
+
+
+def bench_rare_event(args):
+    """3600 frames of 1280x720 with 40 injected events: frames/s, keep ratio
+    and event-frame recall across tau_h."""
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.rare_event()
+    host = torch.empty((spec.frames, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.cuda()
+    events = torch.from_numpy(synth.event_mask(spec).astype(bool)).cuda()
+    starts = synth.event_mask(spec)
+    out = {"workload": "rare-event: 3600 frames of 1280x720, 40 events of 1-3 frames", "taus": {}}
+    for tau in (0.30, 0.15, 0.10, 0.05, 0.02):
+        f = NGFF(spec.width, spec.height, tau=tau)
+        scores = torch.empty(spec.frames, dtype=torch.float32, device="cuda")
+        keep = torch.empty(spec.frames, dtype=torch.uint8, device="cuda")
+
+        def step():
+            f.reset()
+            f.push(dev, scores=scores, keep=keep)
+
+        for _ in range(3):
+            step()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(20):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+        f.status()
+        kept = keep != 0
+        # per-event recall: an event counts as caught if any of its frames is kept
+        ev = starts.astype(bool)
+        runs, t = [], 0
+        while t < spec.frames:
+            if ev[t]:
+                u = t
+                while u < spec.frames and ev[u]:
+                    u += 1
+                runs.append((t, u))
+                t = u
+            else:
+                t += 1
+        kc = kept.cpu().numpy()
+        caught = sum(1 for a, b in runs if kc[a:b].any())
+        out["taus"][str(tau)] = {"frames_per_s": 20 * spec.frames / (e0.elapsed_time(e1) / 1e3),
+                                 "keep_ratio": float(kept.float().mean().item()),
+                                 "event_frame_recall": float(kept[events].float().mean().item()),
+                                 "event_recall": caught / max(1, len(runs))}
+        f.close()
+    print(json.dumps(out), flush=True)
+
+
+def bench_gather(args):
+    """Closing the 1080p prefix: candidate set S_c, then the gather of S_c into
+    one buffer. Bandwidth of the gather (bytes read + written) against the
+    measured copy peak."""
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.hd1080()
+    spec = spec.with_(frames=min(spec.frames, max(1, args.frames)))
+    host = torch.empty((spec.frames, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.cuda()
+    del host
+    f = NGFF(spec.width, spec.height, max_frames_per_push=spec.frames)
+    _, keep = f.push(dev)
+    idx = f.candidates(keep)
+    m = idx.numel()
+    out = torch.empty((m, spec.height, spec.width, 3), dtype=torch.uint8, device="cuda")
+    m_dev = torch.empty(1, dtype=torch.int32, device="cuda")
+    idx_buf = torch.empty(spec.frames, dtype=torch.int32, device="cuda")
+    from paper_2609_03675_gb300 import _abi
+    st = torch.cuda.current_stream().cuda_stream
+    for _ in range(3):
+        f.gather(dev, idx, out=out)
+    torch.cuda.synchronize()
+    reps = 50
+    e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+    e0.record()
+    for _ in range(reps):
+        f._check(f._lib.cofie_ngff_candidates(f._h, keep.data_ptr(), spec.frames, idx_buf.data_ptr(),
+                                              m_dev.data_ptr(), st))
+    e1.record()
+    for _ in range(reps):
+        f.gather(dev, idx, out=out)
+    e2.record()
+    torch.cuda.synchronize()
+    f.status()
+    del _abi
+    peak, kind = peaks()
+    g_ms = e1.elapsed_time(e2) / reps
+    gbs = 2 * m * spec.frame_bytes / (g_ms / 1e3) / 1e9
+    print(json.dumps({"workload": f"finalize + gather of the 1080p stream ({spec.frames} frames, {m} candidates)",
+                      "candidates_us": e0.elapsed_time(e1) / reps * 1e3, "gather_ms": g_ms,
+                      "gather_bytes": 2 * m * spec.frame_bytes, "gather_gbs": gbs, "peak_gbs": peak,
+                      "frac": gbs / peak, "peak_kind": f"{kind} copy bandwidth (read + write)"}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         bench_reference(args)
+    elif args.workload == "serving":
+        bench_serving(args)
+    elif args.workload == "medium":
+        bench_medium(args)
+    elif args.workload == "rare_event":
+        bench_rare_event(args)
+    elif args.workload == "gather":
+        bench_gather(args)
     else:
         bench_gb300(args)
 

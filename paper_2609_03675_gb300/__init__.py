@@ -115,14 +115,24 @@ class NGFF:
         rc = self._lib.cofie_ngff_push_ex(self._h, stream, frames_ptr, n, scores_ptr, keep_ptr, hist_ptr, st)
         self._check(rc)
 
-    def push_batch(self, items, cuda_stream=None):
-        """items: list of (stream, frames[cuda uint8], scores[cuda f32] | None, keep[cuda u8] | None)."""
+    def make_batch(self, items):
+        """Descriptor array for push_batch_raw from a list of
+        (stream, frames[cuda uint8], scores[cuda f32] | None, keep[cuda u8] | None)."""
         arr = (_abi.PushDesc * max(1, len(items)))()
         for i, (stream, frames, scores, keep) in enumerate(items):
             n = self._frames(frames)
             arr[i].stream, arr[i].n = stream, n
             arr[i].frames, arr[i].scores_out, arr[i].keep_out = _ptr(frames), _ptr(scores), _ptr(keep)
-        self._check(self._lib.cofie_ngff_push_batch(self._h, arr, len(items), self._stream(cuda_stream)))
+        return arr, len(items)
+
+    def push_batch(self, items, cuda_stream=None):
+        """items: list of (stream, frames[cuda uint8], scores[cuda f32] | None, keep[cuda u8] | None)."""
+        arr, nd = self.make_batch(items)
+        self.push_batch_raw(arr, nd, cuda_stream)
+
+    def push_batch_raw(self, arr, nd: int, cuda_stream=None):
+        """The batched C entry point on a prebuilt descriptor array."""
+        self._check(self._lib.cofie_ngff_push_batch(self._h, arr, nd, self._stream(cuda_stream)))
 
     def candidates(self, keep: torch.Tensor, cuda_stream=None) -> torch.Tensor:
         """S_c of a closed prefix: ascending indices of the retained frames, the

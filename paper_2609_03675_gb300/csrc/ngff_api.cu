@@ -65,6 +65,7 @@ struct cofie_ngff {
   uint8_t* d_keep = nullptr;
   uint32_t* d_err = nullptr;
   uint32_t* d_count = nullptr;  // candidate count when the caller's m_out is host memory
+  uint64_t dirty_rows = 0;      // histogram rows [0, dirty_rows) may be nonzero
   uint8_t* d_stage[2] = {nullptr, nullptr};
   uint64_t stage_bytes = 0;
   uint32_t stage_frames = 0;
@@ -174,11 +175,19 @@ double sum_pairs(const std::vector<cudaEvent_t>& pool, size_t used, cudaError_t*
   return ms;
 }
 
-// Runs K1-K3 over the rows described by segs (device frames).
-int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
+// Runs K1-K3 over the rows described by segs (device frames). Histogram rows
+// must be zero when K1 starts: the fused small-push kernel clears its rows
+// after use (unless keep_hist: the caller copies them out afterwards);
+// otherwise the rows are marked dirty and the next push clears them first.
+int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep_hist = false) {
   if (segs.rows == 0) return COFIE_OK;
-  cudaError_t e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(segs.rows) * h->p.bins * 4, st);
-  if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+  cudaError_t e = cudaSuccess;
+  if (h->dirty_rows) {
+    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->p.bins * 4, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+    h->dirty_rows = 0;
+  }
+  h->dirty_rows = h->p.max_frames_per_push;  // until the whole sequence is enqueued
   bool fast = h->size_fast && h->bin_path >= 0;
   for (uint32_t i = 0; i < segs.count && fast; ++i)
     if (reinterpret_cast<uintptr_t>(segs.s[i].frames) % 16 != 0) fast = false;
@@ -207,14 +216,27 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
   sa.mask_words = h->mask_words;
   sa.tau = h->p.tau;
   sa.two_n = h->two_n;
+  uint32_t longest = 0;
+  for (uint32_t i = 0; i < segs.count; ++i) longest = segs.s[i].n > longest ? segs.s[i].n : longest;
+  // small pushes clear their rows inside the fused kernel (saving a launch);
+  // large ones leave that to one device-wide memset before the next push
+  const bool fused = longest <= select_small_max();
+  sa.zero_hist = (fused && !keep_hist) ? 1u : 0u;
   cudaEvent_t es0 = nullptr, es1 = nullptr;
   if (h->time_kernels && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
-  e = launch_window(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
-  if (e != cudaSuccess) return h->cuda_fail(e, "window kernel launch");
-  e = launch_scan(segs, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st);
-  if (e != cudaSuccess) return h->cuda_fail(e, "scan kernel launch");
+  if (fused) {  // distances and scan in one launch
+    e = launch_select_small(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "selection kernel launch");
+    h->n_select += 1;
+  } else {
+    e = launch_window(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "window kernel launch");
+    e = launch_scan(segs, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "scan kernel launch");
+    h->n_select += 2;
+  }
   if (es1) cudaEventRecord(es1, st);
-  h->n_select += 2;
+  h->dirty_rows = sa.zero_hist ? 0 : segs.rows;
   return COFIE_OK;
 }
 
@@ -232,7 +254,7 @@ int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n
   s.stream = stream;
   s.scores = ks == kDevice ? scores : (ks == kNull ? nullptr : h->d_scores);
   s.keep = kk == kDevice ? keep : (kk == kNull ? nullptr : h->d_keep);
-  int rc = run_segments(h, segs, st);
+  int rc = run_segments(h, segs, st, kh != kNull);
   if (rc != COFIE_OK) return rc;
   cudaError_t e = cudaSuccess;
   if (ks == kHostPinned || ks == kHostPageable)
@@ -443,6 +465,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     return COFIE_ENOMEM;
   }
   if (e == cudaSuccess) e = cudaMemset(h->d_state, 0, S * sizeof(StreamState));
+  if (e == cudaSuccess) e = cudaMemset(h->d_hist, 0, F * p->bins * sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
   for (int i = 0; i < 2 && e == cudaSuccess; ++i) {

@@ -2,7 +2,8 @@
 //
 // Data layout in device memory (per handle):
 //   frames   uint8  [rows][H][W][3]   caller-owned (or a staging buffer)
-//   hist     uint32 [rows][B]         integer histograms of the push
+//   hist     uint32 [rows][B]         integer histograms of the push (kept zero
+//                                     between pushes: the scan clears its rows)
 //   l1       uint32 [rows][L_max]     L1[t][k-1] = sum_b |c_t[b] - c_{t-k}[b]|
 //   mask     uint32 [rows][W_m]       bit g-1 of row t: keep decision of frame t
 //                                     if its gap t - r(t) were g (W_m = ceil(L_max/32))
@@ -78,7 +79,8 @@ struct SelectArgs {
   uint32_t l_max;
   uint32_t mask_words;
   float tau;
-  float two_n;  // fp32(2 W H)
+  float two_n;        // fp32(2 W H)
+  uint32_t zero_hist;  // the scan zeroes the push's histogram rows after use
 };
 
 // Launchers (stream-ordered; return the launch error).
@@ -92,7 +94,10 @@ cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const L
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
                           const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st);
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
-                        const uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st);
+                        uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st);
+uint32_t select_small_max();
+cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
+                                StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st);
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);

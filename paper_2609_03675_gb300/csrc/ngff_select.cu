@@ -21,7 +21,11 @@
 //    = entry gap), thread 0 chains the 32 run maps, each warp replays its run
 //    from the resolved entry gap, and all threads then emit score and keep
 //    code per frame. The stream state (frames seen, current gap, ring of the
-//    last L_max histograms) is updated at the end.
+//    last L_max histograms) is updated at the end, and the push's histogram
+//    rows are zeroed for the next push unless the caller asked for them.
+//
+// Small pushes (at most kSmallMax frames per stream) run K2 and K3 as one
+// kernel: the same CTA first computes its stream's distances, then scans.
 #include "ngff_common.cuh"
 
 namespace cofie {
@@ -31,27 +35,22 @@ constexpr int kWinWarps = 8;
 constexpr int kScanThreads = 1024;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr uint32_t kScanTile = 4096;  // frames per shared-memory tile
+constexpr uint32_t kSmallMax = 64;    // frames per stream segment for the fused small-push kernel
 
 __device__ __forceinline__ uint32_t absdiff(uint32_t a, uint32_t b) { return a > b ? a - b : b - a; }
 
-// One warp per frame; lane = lag: lane k-1 sums |c_t - c_{t-k}| over all
-// bins of row t-k (16-byte loads when B % 4 == 0), so the warp's loads are
-// independent and in flight together. The keep bit for gap g = k is decided
-// in the same lane.
+// K2's work for one frame (row of the push), done by one warp. Lane k-1 sums
+// |c_t - c_{t-k}| over all bins of row t-k (16-byte loads when B % 4 == 0),
+// so the warp's loads are independent and in flight together; the keep bit
+// for gap g = k is decided in the same lane.
 template <bool kVec4>
-__global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, SelectArgs a,
-                                                                const uint32_t* __restrict__ hist,
-                                                                const uint32_t* __restrict__ ring,
-                                                                const StreamState* __restrict__ state,
-                                                                uint32_t* __restrict__ l1, uint32_t* __restrict__ mask) {
-  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t row = blockIdx.x * kWinWarps + warp;
-  if (row >= segs.rows) return;
-  uint32_t seg = 0;
-  while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
-  const uint32_t stream = segs.s[seg].stream;
-  const uint32_t j = row - segs.s[seg].row0;
-  const unsigned long long t = state[stream].t + j;
+__device__ __forceinline__ void window_row(uint32_t row, uint32_t lane, const Segment& sg, const SelectArgs& a,
+                                           const uint32_t* __restrict__ hist, const uint32_t* __restrict__ ring,
+                                           unsigned long long t0, uint32_t* __restrict__ l1,
+                                           uint32_t* __restrict__ mask) {
+  const uint32_t stream = sg.stream;
+  const uint32_t j = row - sg.row0;
+  const unsigned long long t = t0 + j;
   const uint32_t B = a.bins, L = a.l_max;
   const uint32_t* ct = hist + static_cast<uint64_t>(row) * B;
   uint32_t l_adj = 0;
@@ -88,41 +87,44 @@ __global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, S
   }
 }
 
+template <bool kVec4>
+__global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, SelectArgs a,
+                                                                const uint32_t* __restrict__ hist,
+                                                                const uint32_t* __restrict__ ring,
+                                                                const StreamState* __restrict__ state,
+                                                                uint32_t* __restrict__ l1, uint32_t* __restrict__ mask) {
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t row = blockIdx.x * kWinWarps + warp;
+  if (row >= segs.rows) return;
+  uint32_t seg = 0;
+  while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
+  const Segment sg = segs.s[seg];
+  window_row<kVec4>(row, lane, sg, a, hist, ring, state[sg.stream].t, l1, mask);
+}
+
 template <bool kOneWord>
 __device__ __forceinline__ uint32_t step_gap(const uint32_t* m, uint32_t g) {
   const uint32_t word = kOneWord ? m[0] : m[(g - 1) >> 5];
   return ((word >> ((g - 1) & 31)) & 1u) ? 1u : g + 1u;
 }
 
+// K3's work for one stream segment, done by a whole 1024-thread CTA. sseg,
+// t0 and g0 are the segment and its stream's state on entry (shared memory).
 template <bool kOneWord>
-__global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, SelectArgs a,
-                                                            const uint32_t* __restrict__ l1,
-                                                            const uint32_t* __restrict__ mask,
-                                                            const uint32_t* __restrict__ hist,
-                                                            uint32_t* __restrict__ ring,
-                                                            StreamState* __restrict__ state) {
-  extern __shared__ __align__(16) uint32_t ssm[];
-  __shared__ Segment sseg;
-  __shared__ uint32_t entry[kScanWarps + 1];
-  __shared__ unsigned long long s_t0;
-  __shared__ uint32_t s_g;
+__device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long long t0, uint32_t g0,
+                                             const SelectArgs& a, const uint32_t* __restrict__ l1,
+                                             const uint32_t* __restrict__ mask, uint32_t* __restrict__ hist,
+                                             uint32_t* __restrict__ ring, StreamState* __restrict__ state,
+                                             uint32_t* ssm, uint32_t* entry) {
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t W = a.mask_words, L = a.l_max, B = a.bins;
-  uint32_t* smask = ssm;                                       // [kScanTile][W]
+  uint32_t* smask = ssm;                                                // [kScanTile][W]
   uint16_t* sgap = reinterpret_cast<uint16_t*>(smask + kScanTile * W);  // [kScanTile]
-  uint16_t* sexit = sgap + kScanTile;                          // [kScanWarps][L]
-
-  if (tid == 0) {
-    sseg = segs.s[blockIdx.x];
-    s_t0 = state[sseg.stream].t;
-    s_g = state[sseg.stream].g;
-  }
-  __syncthreads();
+  uint16_t* sexit = sgap + kScanTile;                                   // [kScanWarps][L]
   const uint32_t n = sseg.n, row0 = sseg.row0, stream = sseg.stream;
   if (n == 0) return;
-  const unsigned long long t0 = s_t0;
   const uint32_t j_start = (t0 == 0) ? 1u : 0u;  // the stream's first frame is decided below
-  uint32_t g_entry = (t0 == 0) ? 1u : s_g;
+  uint32_t g_entry = (t0 == 0) ? 1u : g0;
   if (g_entry < 1u || g_entry > L) g_entry = L;  // the state only ever holds [1, L]
 
   for (uint32_t tile0 = j_start; tile0 < n; tile0 += kScanTile) {
@@ -189,6 +191,58 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
     const uint64_t slot = (t0 + jj) % L;
     ring[(static_cast<uint64_t>(stream) * L + slot) * B + b] = hist[static_cast<uint64_t>(row0 + jj) * B + b];
   }
+  if (a.zero_hist) {  // leave the push's histogram rows zeroed for the next push
+    __syncthreads();
+    for (uint64_t i = tid; i < static_cast<uint64_t>(n) * B; i += kScanThreads)
+      hist[static_cast<uint64_t>(row0) * B + i] = 0;
+  }
+}
+
+template <bool kOneWord>
+__global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, SelectArgs a,
+                                                            const uint32_t* __restrict__ l1,
+                                                            const uint32_t* __restrict__ mask,
+                                                            uint32_t* __restrict__ hist, uint32_t* __restrict__ ring,
+                                                            StreamState* __restrict__ state) {
+  extern __shared__ __align__(16) uint32_t ssm[];
+  __shared__ Segment sseg;
+  __shared__ uint32_t entry[kScanWarps + 1];
+  __shared__ unsigned long long s_t0;
+  __shared__ uint32_t s_g;
+  if (threadIdx.x == 0) {
+    sseg = segs.s[blockIdx.x];
+    s_t0 = state[sseg.stream].t;
+    s_g = state[sseg.stream].g;
+  }
+  __syncthreads();
+  scan_segment<kOneWord>(sseg, s_t0, s_g, a, l1, mask, hist, ring, state, ssm, entry);
+}
+
+// Small pushes: one CTA per stream segment computes the segment's windowed
+// distances (one warp per frame) and then scans them.
+template <bool kVec4, bool kOneWord>
+__global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable segs, SelectArgs a,
+                                                                    uint32_t* __restrict__ hist,
+                                                                    uint32_t* __restrict__ ring,
+                                                                    StreamState* __restrict__ state,
+                                                                    uint32_t* __restrict__ l1,
+                                                                    uint32_t* __restrict__ mask) {
+  extern __shared__ __align__(16) uint32_t ssm[];
+  __shared__ Segment sseg;
+  __shared__ uint32_t entry[kScanWarps + 1];
+  __shared__ unsigned long long s_t0;
+  __shared__ uint32_t s_g;
+  if (threadIdx.x == 0) {
+    sseg = segs.s[blockIdx.x];
+    s_t0 = state[sseg.stream].t;
+    s_g = state[sseg.stream].g;
+  }
+  __syncthreads();
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (uint32_t j = warp; j < sseg.n; j += kScanWarps)
+    window_row<kVec4>(sseg.row0 + j, lane, sseg, a, hist, ring, s_t0, l1, mask);
+  __syncthreads();  // this CTA's distance and mask rows are visible to all its threads
+  scan_segment<kOneWord>(sseg, s_t0, s_g, a, l1, mask, hist, ring, state, ssm, entry);
 }
 
 size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
@@ -197,10 +251,25 @@ size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
 
 }  // namespace
 
+uint32_t select_small_max() { return kSmallMax; }
+
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max) {
   const int smem = static_cast<int>(scan_smem_bytes(mask_words, l_max));
-  return mask_words == 1 ? cudaFuncSetAttribute(scan_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)
-                         : cudaFuncSetAttribute(scan_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  cudaError_t e;
+  if (mask_words == 1) {
+    e = cudaFuncSetAttribute(scan_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(select_small_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(select_small_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  } else {
+    e = cudaFuncSetAttribute(scan_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(select_small_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(select_small_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  }
+  return e;
 }
 
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
@@ -214,12 +283,27 @@ cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint3
 }
 
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
-                        const uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st) {
+                        uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st) {
   const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
   if (a.mask_words == 1)
     scan_kernel<true><<<segs.count, kScanThreads, smem, st>>>(segs, a, l1, mask, hist, ring, state);
   else
     scan_kernel<false><<<segs.count, kScanThreads, smem, st>>>(segs, a, l1, mask, hist, ring, state);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
+                                StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
+  const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
+  const bool vec = a.bins % 4 == 0, one = a.mask_words == 1;
+  if (vec && one)
+    select_small_kernel<true, true><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
+  else if (vec)
+    select_small_kernel<true, false><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
+  else if (one)
+    select_small_kernel<false, true><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
+  else
+    select_small_kernel<false, false><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
   return cudaGetLastError();
 }
 

@@ -171,3 +171,35 @@ def test_all_triples_frame_histogram():
         _, _, h = f.push(px.cuda(), return_hist=True)
         torch.cuda.synchronize()
         assert np.array_equal(h.cpu().numpy()[0].view(np.uint32), want)
+
+
+def test_histogram_rows_cleared_between_pushes():
+    """Pushes that return their histograms and pushes that do not, small
+    (fused selection kernel) and large (separate kernels), interleaved on one
+    stream and across two handles' streams, all match the oracle."""
+    spec = synth.medium(seed=41).with_(width=80, height=48, frames=400, mean_scene_len=12)
+    fr = synth.generate(spec)
+    ho, so, ko = oracle_run(fr, O.Params(80, 48, tau=0.05))
+    dev = torch.from_numpy(fr).cuda()
+    f = _ngff(80, 48, tau=0.05, max_streams=2)
+    chunks = [5, 130, 64, 65, 1, 100, 8, 27]  # sums to 400
+    want_hist = [True, False, False, True, False, True, True, False]
+    got_s, got_k = [], []
+    off = 0
+    for c, wh in zip(chunks, want_hist):
+        if wh:
+            s, k, h = f.push(dev[off:off + c], return_hist=True)
+            torch.cuda.synchronize()
+            assert np.array_equal(h.cpu().numpy().view(np.uint32), ho[off:off + c])
+        else:
+            s, k = f.push(dev[off:off + c])
+        # a second stream interleaved, always without histograms
+        f.push(dev[off:off + c], stream=1)
+        got_s.append(s)
+        got_k.append(k)
+        off += c
+    torch.cuda.synchronize()
+    f.status()
+    assert np.array_equal(torch.cat(got_k).cpu().numpy(), ko)
+    s = torch.cat(got_s).cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(s - so) <= 1e-6 * so)
