@@ -270,6 +270,59 @@ int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out);
 int cofie_ngff_select_static(const cofie_ngff_params* p, const uint32_t* hist, uint32_t n, float* scores_out,
                              uint8_t* keep_out, char* err, size_t err_cap, void* cuda_stream);
 
+/* ------------------------------------------------------------------------
+ * Query-specific evidence refinement (QER, CoFiE Sec. 3.3, Eqs. 6-8): the
+ * fine stage that ranks the NGFF candidates by text-to-vision attention.
+ *
+ *   a_ij = (1/H) sum_h <q_i^h, k_j^h> / sqrt(d_h)        (Eq. 6)
+ *   w_f  = mean over the frame's tokens of max_i a_ij    (Eq. 7)
+ *   S_e  = the max(1, round(rho m)) best frames by w_f   (Eq. 8)
+ *
+ * Query head h reads key head h / (H / H_kv) (grouped key/value heads, as in
+ * the attention). The query heads of each group are summed in fp32 and
+ * rounded to bf16; the contraction runs on the tensor cores in bf16 with fp32
+ * accumulation. round() rounds half to even; equal scores rank by lower
+ * frame index; S_e is returned in time order.
+ * ------------------------------------------------------------------------ */
+typedef struct cofie_qer cofie_qer_t;
+
+typedef struct {
+  uint32_t n_text;           /* text tokens |Q|, 1..256 */
+  uint32_t n_heads;          /* H query heads */
+  uint32_t n_kv_heads;       /* H_kv key heads, divides H */
+  uint32_t head_dim;         /* d_h; H_kv * d_h a multiple of 64, at most 16384 */
+  uint32_t max_frames;       /* largest |S_c| per call */
+  uint32_t tokens_per_frame; /* |V_f|, the same for every frame */
+  float rho;                 /* keep ratio, [0, 1] */
+  int32_t device;            /* CUDA device ordinal, or -1 for the current device */
+} cofie_qer_params;
+
+/* Validates *p and allocates the scratch (group-summed queries, per-token
+ * maxima, frame scores). Synchronous. Errors: COFIE_EINVAL, COFIE_ENOMEM, COFIE_ECUDA. */
+int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out);
+
+void cofie_qer_destroy(cofie_qer_t* h);
+
+/*
+ * Ranks n_frames candidate frames (Eqs. 6-8).
+ *   q        bf16 [n_text][H][d_h], device memory.
+ *   k        bf16 [n_frames * tokens_per_frame][H_kv][d_h], device memory,
+ *            16-byte aligned; frame f owns tokens [f T, (f+1) T).
+ *   w_out    n_frames floats (w_f), device memory, or NULL.
+ *   sel_out  room for n_frames uint32 frame indices (S_e, ascending), device memory.
+ *   k_out    |S_e|: device memory (asynchronous) or host memory (synchronises).
+ * Errors: COFIE_EINVAL, COFIE_ECUDA; device-side waits are reported by
+ * cofie_qer_status.
+ */
+int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t n_frames, float* w_out,
+                  uint32_t* sel_out, uint32_t* k_out, void* cuda_stream);
+
+/* Synchronises cuda_stream; COFIE_ETIMEOUT if a bounded device wait ran out. */
+int cofie_qer_status(cofie_qer_t* h, void* cuda_stream);
+
+/* Last error of h, or of the last failed cofie_qer_create when h is NULL. Never NULL. */
+const char* cofie_qer_last_error(const cofie_qer_t* h);
+
 /* Text of the last error on this handle (empty string if none). Never NULL. */
 const char* cofie_ngff_last_error(const cofie_ngff_t* h);
 

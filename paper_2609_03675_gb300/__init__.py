@@ -17,7 +17,7 @@ import torch
 from . import _abi
 from ._abi import (KEEP_DROP, KEEP_FIRST, KEEP_GAP, KEEP_NOVELTY, NGFFError)  # noqa: F401
 
-__all__ = ["NGFF", "NGFFError", "KEEP_DROP", "KEEP_NOVELTY", "KEEP_GAP", "KEEP_FIRST", "library_path"]
+__all__ = ["NGFF", "QER", "NGFFError", "KEEP_DROP", "KEEP_NOVELTY", "KEEP_GAP", "KEEP_FIRST", "library_path"]
 
 
 def library_path() -> str:
@@ -201,3 +201,53 @@ class NGFF:
 
     def __exit__(self, *exc):
         self.close()
+
+
+class QER:
+    """Query-specific evidence refinement (CoFiE Sec. 3.3) on the tensor cores:
+    ranks candidate frames by text-to-vision attention and keeps the best
+    max(1, round(rho m)) of them."""
+
+    def __init__(self, n_text: int, n_heads: int, n_kv_heads: int, head_dim: int, max_frames: int,
+                 tokens_per_frame: int, rho: float, device: int | None = None):
+        lib = _abi.load()
+        p = _abi.QerParams(n_text, n_heads, n_kv_heads, head_dim, max_frames, tokens_per_frame, rho,
+                           torch.cuda.current_device() if device is None else device)
+        h = ctypes.c_void_p()
+        rc = lib.cofie_qer_create(ctypes.byref(p), ctypes.byref(h))
+        if rc != _abi.OK:
+            raise NGFFError(rc, lib.cofie_qer_last_error(None).decode())
+        self._lib, self._h, self.params = lib, h, p
+        self.device = torch.device("cuda", p.device)
+
+    def _check(self, rc):
+        if rc != _abi.OK:
+            raise NGFFError(rc, self._lib.cofie_qer_last_error(self._h).decode())
+
+    def run(self, q: torch.Tensor, k: torch.Tensor, n_frames: int | None = None, cuda_stream=None):
+        """q: bf16 bits (int16/uint16 or bfloat16) [n_text, H, d]; k: [n_frames * T, H_kv, d].
+        Returns (w [n_frames] float32, selected frame indices int32, time order)."""
+        T = self.params.tokens_per_frame
+        n = k.shape[0] // T if n_frames is None else n_frames
+        w = torch.empty(n, dtype=torch.float32, device=self.device)
+        sel = torch.empty(n, dtype=torch.int32, device=self.device)
+        kk = ctypes.c_uint32(0)
+        st = torch.cuda.current_stream(self.device).cuda_stream if cuda_stream is None else int(cuda_stream)
+        self._check(self._lib.cofie_qer_run(self._h, _ptr(q), _ptr(k), n, _ptr(w), _ptr(sel),
+                                            ctypes.addressof(kk), st))
+        return w, sel[: kk.value]
+
+    def status(self, cuda_stream=None):
+        st = torch.cuda.current_stream(self.device).cuda_stream if cuda_stream is None else int(cuda_stream)
+        self._check(self._lib.cofie_qer_status(self._h, st))
+
+    def close(self):
+        if getattr(self, "_h", None):
+            self._lib.cofie_qer_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:  # noqa: BLE001 -- interpreter shutdown
+            pass

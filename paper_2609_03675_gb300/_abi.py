@@ -35,6 +35,11 @@ EXPORTS = (
     "cofie_ngff_select_static",
     "cofie_ngff_last_error",
     "cofie_ngff_global_error",
+    "cofie_qer_create",
+    "cofie_qer_destroy",
+    "cofie_qer_run",
+    "cofie_qer_status",
+    "cofie_qer_last_error",
 )
 
 
@@ -74,6 +79,19 @@ class Profile(ctypes.Structure):
         ("hist_ms", ctypes.c_double),
         ("select_timed", ctypes.c_uint64),
         ("select_ms", ctypes.c_double),
+    ]
+
+
+class QerParams(ctypes.Structure):
+    _fields_ = [
+        ("n_text", ctypes.c_uint32),
+        ("n_heads", ctypes.c_uint32),
+        ("n_kv_heads", ctypes.c_uint32),
+        ("head_dim", ctypes.c_uint32),
+        ("max_frames", ctypes.c_uint32),
+        ("tokens_per_frame", ctypes.c_uint32),
+        ("rho", ctypes.c_float),
+        ("device", ctypes.c_int32),
     ]
 
 
@@ -128,6 +146,16 @@ def load():
     lib.cofie_ngff_profile_read.restype = ctypes.c_int
     lib.cofie_ngff_select_static.argtypes = [P, vp, u32, vp, vp, ctypes.c_char_p, ctypes.c_size_t, vp]
     lib.cofie_ngff_select_static.restype = ctypes.c_int
+    lib.cofie_qer_create.argtypes = [ctypes.POINTER(QerParams), ctypes.POINTER(H)]
+    lib.cofie_qer_create.restype = ctypes.c_int
+    lib.cofie_qer_destroy.argtypes = [H]
+    lib.cofie_qer_destroy.restype = None
+    lib.cofie_qer_run.argtypes = [H, vp, vp, u32, vp, vp, vp, vp]
+    lib.cofie_qer_run.restype = ctypes.c_int
+    lib.cofie_qer_status.argtypes = [H, vp]
+    lib.cofie_qer_status.restype = ctypes.c_int
+    lib.cofie_qer_last_error.argtypes = [H]
+    lib.cofie_qer_last_error.restype = ctypes.c_char_p
     lib.cofie_ngff_last_error.argtypes = [H]
     lib.cofie_ngff_last_error.restype = ctypes.c_char_p
     lib.cofie_ngff_global_error.argtypes = []

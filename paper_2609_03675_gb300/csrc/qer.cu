@@ -1,0 +1,515 @@
+// Query-specific evidence refinement (QER), CoFiE Sec. 3.3, Eqs. 6-8, on the
+// GB300 tensor cores.
+//
+//   a_ij = (1/H) sum_h <q_i^h, k_j^h> / sqrt(d_h)            (Eq. 6)
+//   w_f  = mean_{j in V_f} max_{i in Q} a_ij                  (Eq. 7)
+//   S_e  = TopK_f(w_f, max(1, round(rho |S_c|))), in time order (Eq. 8)
+//
+// With grouped key/value heads (query head h reads key head h / G, G = H/H_kv)
+// the head mean of Eq. 6 is one dot product over D = H_kv * d_h once the G
+// query heads of each group are summed:
+//   a_ij = <q~_i, k_j> / (H sqrt(d_h)),  q~_i[g, c] = sum_{h in group g} q_i^h[c].
+// So Eq. 6 is a single bf16 GEMM-shaped contraction, Q~ [N x D] times K^T
+// [D x n_visual], whose column maxima over text (Eq. 7, inner max) are all
+// that is kept: the text-by-vision score matrix is never written to memory,
+// which is the point of the paper's tiled computation.
+//
+// Kernels:
+//   qer_prepare_q   q [n_text][H][d] -> q~ [N][D] bf16 (fp32 sums rounded to
+//                   nearest even; rows n_text..N-1 zero, N = n_text rounded up to 16)
+//   qer_score       one CTA per 128 visual tokens: TMA (cp.async.bulk.tensor,
+//                   128-byte swizzle) streams 64-wide K chunks of the token
+//                   tile and of q~ into a 4-stage shared-memory ring; one thread
+//                   issues tcgen05.mma (kind::f16, M = 128, N, K = 16) into a
+//                   TMEM accumulator (128 lanes x N fp32 columns) and commits
+//                   each stage back to the producer; four warps then read their
+//                   32 TMEM lanes (tcgen05.ld) and keep each token's max over
+//                   the n_text real columns.
+//   qer_select      one CTA: w_f = (sum of the frame's token maxima) / (|V_f| H sqrt(d)),
+//                   then the k best frames by rank (ties to the lower index),
+//                   compacted in time order.
+// Every mbarrier wait is bounded by the global timer; a wait that runs out
+// sets an error bit, stops issuing, lets the work already issued finish
+// (bounded) and frees TMEM before the CTA exits.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <string>
+
+#include "cofie_ngff.h"
+#include "ngff_common.cuh"
+
+namespace cofie {
+namespace {
+
+constexpr int kQerM = 128;          // visual tokens per CTA (MMA M)
+constexpr int kQerKChunk = 64;      // bf16 elements per 128-byte swizzled row
+constexpr int kQerStages = 4;
+constexpr int kQerUmmaK = 16;       // K of one tcgen05.mma for 16-bit inputs
+constexpr int kQerThreads = 128;    // four warps: TMEM lanes 0..127
+constexpr uint32_t kQerMaxN = 256;  // text tokens (MMA N) per CTA
+constexpr int kSelThreads = 1024;
+
+constexpr uint32_t kQerErrProducer = 16u, kQerErrMma = 32u, kQerErrEpilogue = 64u, kQerErrDrain = 128u;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t gtimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __noinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  if (mbar_try(bar, parity)) return true;
+  const uint64_t t0 = gtimer();
+  for (;;) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try(bar, parity)) return true;
+    if (gtimer() - t0 > timeout_ns) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t x, int32_t y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major, 128-byte-swizzled tile whose
+// rows are 128 bytes and whose 8-row swizzle atoms are 1024 bytes apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((addr >> 4) & 0x3FFFu);  // start address
+  d |= static_cast<uint64_t>(1u) << 16;                // leading byte offset (unused for swizzled K-major)
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;        // stride byte offset: 8 rows x 128 B
+  d |= static_cast<uint64_t>(1u) << 46;                // descriptor version
+  d |= static_cast<uint64_t>(2u) << 61;                // swizzle: 128 B
+  return d;
+}
+
+// Instruction descriptor: bf16 x bf16 -> fp32, both operands K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((n >> 3) << 17) | ((m >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H,
+                              uint32_t H_kv, uint32_t d, __nv_bfloat16_raw* __restrict__ qg) {
+  const uint32_t D = H_kv * d, G = H / H_kv;
+  const uint64_t total = static_cast<uint64_t>(n_pad) * D;
+  for (uint64_t e = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<uint64_t>(gridDim.x) * blockDim.x) {
+    const uint32_t i = static_cast<uint32_t>(e / D), r = static_cast<uint32_t>(e % D);
+    const uint32_t g = r / d, c = r % d;
+    float s = 0.f;
+    if (i < n_text)
+      for (uint32_t h = g * G; h < (g + 1) * G; ++h)
+        s += __uint_as_float(static_cast<uint32_t>(q[(static_cast<uint64_t>(i) * H + h) * d + c]) << 16);
+    qg[e] = static_cast<__nv_bfloat16_raw>(__float2bfloat16_rn(s));
+  }
+}
+
+__global__ void __launch_bounds__(kQerThreads, 1) qer_score(const __grid_constant__ CUtensorMap map_k,
+                                                             const __grid_constant__ CUtensorMap map_q,
+                                                             uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
+                                                             uint32_t tmem_cols, uint32_t n_chunks,
+                                                             float* __restrict__ colmax, uint32_t* __restrict__ err,
+                                                             uint64_t timeout_ns) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kQerStages];
+  __shared__ __align__(8) uint64_t empty_bar[kQerStages];
+  __shared__ __align__(8) uint64_t accum_bar;
+  __shared__ uint32_t tmem_slot;
+
+  // 1024-byte aligned stage buffers (the 128-byte swizzle repeats every 1024 bytes)
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t a_bytes = kQerM * 128, b_bytes = n_pad * 128;
+  const uint32_t stage_bytes = a_bytes + ((b_bytes + 1023) & ~1023u);
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t row0 = blockIdx.x * kQerM;
+
+  if (warp == 0) {  // the whole warp allocates the accumulator columns
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(tmem_cols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  if (threadIdx.x == 32) {
+    for (int s = 0; s < kQerStages; ++s) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full_bar[s])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&empty_bar[s])) : "memory");
+    }
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&accum_bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------- TMA producer
+    uint32_t issued = 0;
+    for (uint32_t kc = 0; kc < n_chunks; ++kc) {
+      const uint32_t s = kc % kQerStages, use = kc / kQerStages;
+      if (use > 0 && !mbar_wait_for(smem_u32(&empty_bar[s]), (use - 1) & 1, timeout_ns)) {
+        atomicOr(err, kQerErrProducer);
+        break;
+      }
+      const uint32_t fb = smem_u32(&full_bar[s]);
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(a_bytes + b_bytes)
+                   : "memory");
+      const uint32_t base = smem_u32(smem + s * stage_bytes);
+      tma_load_2d(base, &map_k, static_cast<int32_t>(kc * kQerKChunk), static_cast<int32_t>(row0), fb);
+      tma_load_2d(base + a_bytes, &map_q, static_cast<int32_t>(kc * kQerKChunk), 0, fb);
+      ++issued;
+    }
+    // no copy may still be writing shared memory when the CTA exits
+    for (uint32_t j = issued > kQerStages ? issued - kQerStages : 0; j < issued; ++j)
+      if (!mbar_wait_for(smem_u32(&full_bar[j % kQerStages]), (j / kQerStages) & 1, timeout_ns))
+        atomicOr(err, kQerErrDrain);
+  } else if (warp == 1 && lane == 0) {
+    // ----------------------------------------------------------- MMA issuer
+    const uint32_t idesc = idesc_bf16_f32(kQerM, n_pad);
+    for (uint32_t kc = 0; kc < n_chunks; ++kc) {
+      const uint32_t s = kc % kQerStages, use = kc / kQerStages;
+      if (!mbar_wait_for(smem_u32(&full_bar[s]), use & 1, timeout_ns)) {
+        atomicOr(err, kQerErrMma);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t a0 = smem_u32(smem + s * stage_bytes), b0 = a0 + a_bytes;
+#pragma unroll
+      for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk)
+        umma_bf16(tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), idesc, (kc | kk) != 0);
+      umma_commit(smem_u32(&empty_bar[s]));  // the stage is free once these MMAs have read it
+    }
+    umma_commit(smem_u32(&accum_bar));  // every MMA issued so far is complete
+  }
+  __syncwarp();
+
+  // ------------------------------------------------------------- epilogue
+  const bool ok = mbar_wait_for(smem_u32(&accum_bar), 0, timeout_ns);
+  if (!ok && lane == 0) atomicOr(err, kQerErrEpilogue);
+  tc_fence_after();
+  float best = -INFINITY;
+  const uint32_t taddr = tmem + ((warp * 32u) << 16);
+  for (uint32_t c0 = 0; c0 < n_pad; c0 += 32) {
+    float v[32];
+    tmem_ld32(taddr + c0, v);
+#pragma unroll
+    for (uint32_t c = 0; c < 32; ++c)
+      if (c0 + c < n_text) best = fmaxf(best, v[c]);
+  }
+  const uint32_t j = row0 + warp * 32 + lane;
+  if (ok && j < n_visual) colmax[j] = best;
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols) : "memory");
+  }
+}
+
+__global__ void __launch_bounds__(kSelThreads) qer_select(const float* __restrict__ colmax, uint32_t n_frames,
+                                                          uint32_t tpf, float scale, uint32_t k,
+                                                          float* __restrict__ w, uint32_t* __restrict__ sel,
+                                                          uint32_t* __restrict__ k_out) {
+  __shared__ uint32_t wsum[32];
+  __shared__ uint32_t s_total;
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // Eq. 7: mean over the frame's tokens of their max over text (then the 1/(H sqrt(d)) of Eq. 6)
+  for (uint32_t f = warp; f < n_frames; f += kSelThreads / 32) {
+    float s = 0.f;
+    for (uint32_t t = lane; t < tpf; t += 32) s += colmax[static_cast<uint64_t>(f) * tpf + t];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) w[f] = s / static_cast<float>(tpf) * scale;
+  }
+  __syncthreads();
+  // Eq. 8: frame f is kept when fewer than k frames rank above it (ties: lower index first)
+  uint32_t base = 0;
+  for (uint32_t f0 = 0; f0 < n_frames; f0 += kSelThreads) {
+    const uint32_t f = f0 + tid;
+    bool in = false;
+    if (f < n_frames) {
+      const float wf = w[f];
+      uint32_t above = 0;
+      for (uint32_t g = 0; g < n_frames && above < k; ++g) {
+        const float wg = w[g];
+        above += (wg > wf) || (wg == wf && g < f);
+      }
+      in = above < k;
+    }
+    const uint32_t bal = __ballot_sync(0xffffffffu, in);
+    const uint32_t before = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) wsum[warp] = __popc(bal);
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t v = wsum[lane];
+      uint32_t x = v;
+#pragma unroll
+      for (int dd = 1; dd < 32; dd <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, x, dd);
+        if (lane >= static_cast<uint32_t>(dd)) x += y;
+      }
+      wsum[lane] = x - v;
+      if (lane == 31) s_total = x;
+    }
+    __syncthreads();
+    if (in) sel[base + wsum[warp] + before] = f;
+    base += s_total;
+    __syncthreads();
+  }
+  if (tid == 0) *k_out = base;
+}
+
+size_t qer_smem_bytes(uint32_t n_pad) {
+  const uint32_t stage = kQerM * 128 + ((n_pad * 128 + 1023) & ~1023u);
+  return static_cast<size_t>(kQerStages) * stage + 1024;  // + slack for the 1024-byte alignment
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor [rows][cols] (cols contiguous), boxes of 64 columns x box_rows.
+bool make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kQerKChunk), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace
+}  // namespace cofie
+
+using namespace cofie;
+
+struct cofie_qer {
+  cofie_qer_params p{};
+  int device = 0;
+  uint32_t n_pad = 0, D = 0, tmem_cols = 0;
+  __nv_bfloat16_raw* d_qg = nullptr;
+  float* d_colmax = nullptr;
+  float* d_w = nullptr;
+  uint32_t* d_k = nullptr;
+  uint32_t* d_err = nullptr;
+  std::string err;
+  int fail(int code, const std::string& m) {
+    err = m;
+    return code;
+  }
+};
+
+namespace {
+
+bool is_device(const void* p, int dev) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) && a.device == dev;
+}
+
+void qer_free(cofie_qer* h) {
+  if (!h) return;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  void* bufs[] = {h->d_qg, h->d_colmax, h->d_w, h->d_k, h->d_err};
+  for (void* b : bufs)
+    if (b) cudaFree(b);
+  if (prev >= 0) cudaSetDevice(prev);
+  delete h;
+}
+
+thread_local std::string g_qer_error;
+
+}  // namespace
+
+extern "C" {
+
+int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
+  if (!p || !out) return g_qer_error = "params or out is NULL", COFIE_EINVAL;
+  if (p->n_text < 1 || p->n_text > kQerMaxN) return g_qer_error = "n_text must be in [1, 256]", COFIE_EINVAL;
+  if (p->n_heads < 1 || p->n_kv_heads < 1 || p->n_heads % p->n_kv_heads != 0)
+    return g_qer_error = "n_kv_heads must divide n_heads", COFIE_EINVAL;
+  const uint64_t D = static_cast<uint64_t>(p->n_kv_heads) * p->head_dim;
+  if (p->head_dim < 1 || D % kQerKChunk != 0 || D > 16384)
+    return g_qer_error = "n_kv_heads * head_dim must be a multiple of 64, at most 16384", COFIE_EINVAL;
+  if (p->max_frames < 1 || p->tokens_per_frame < 1 ||
+      static_cast<uint64_t>(p->max_frames) * p->tokens_per_frame > 0x7fffffffull)
+    return g_qer_error = "max_frames and tokens_per_frame must be >= 1 (product < 2^31)", COFIE_EINVAL;
+  if (!(p->rho >= 0.f && p->rho <= 1.f)) return g_qer_error = "rho must be in [0, 1]", COFIE_EINVAL;
+  int dev = p->device;
+  if (dev < 0 && cudaGetDevice(&dev) != cudaSuccess) return g_qer_error = "no CUDA device", COFIE_ECUDA;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (cudaSetDevice(dev) != cudaSuccess) return g_qer_error = "cannot select the device", COFIE_ECUDA;
+  if (!tensor_map_encoder()) {
+    if (prev >= 0) cudaSetDevice(prev);
+    return g_qer_error = "cuTensorMapEncodeTiled is not available", COFIE_ECUDA;
+  }
+  cofie_qer* h = new (std::nothrow) cofie_qer();
+  if (!h) return g_qer_error = "host allocation failed", COFIE_ENOMEM;
+  h->p = *p;
+  h->device = dev;
+  h->D = static_cast<uint32_t>(D);
+  h->n_pad = (p->n_text + 15) / 16 * 16;
+  h->tmem_cols = 32;
+  while (h->tmem_cols < h->n_pad) h->tmem_cols <<= 1;
+  const uint64_t nv = static_cast<uint64_t>(p->max_frames) * p->tokens_per_frame;
+  cudaError_t e = cudaMalloc(&h->d_qg, static_cast<size_t>(h->n_pad) * D * 2);
+  if (e == cudaSuccess) e = cudaMalloc(&h->d_colmax, nv * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&h->d_w, static_cast<size_t>(p->max_frames) * sizeof(float));
+  if (e == cudaSuccess) e = cudaMalloc(&h->d_k, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMalloc(&h->d_err, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(qer_score, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(qer_smem_bytes(h->n_pad)));
+  if (prev >= 0) cudaSetDevice(prev);
+  if (e != cudaSuccess) {
+    g_qer_error = std::string("QER set-up failed: ") + cudaGetErrorString(e);
+    cudaGetLastError();
+    qer_free(h);
+    return e == cudaErrorMemoryAllocation ? COFIE_ENOMEM : COFIE_ECUDA;
+  }
+  *out = h;
+  return COFIE_OK;
+}
+
+void cofie_qer_destroy(cofie_qer_t* h) { qer_free(h); }
+
+int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t n_frames, float* w_out,
+                  uint32_t* sel_out, uint32_t* k_out, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (n_frames < 1 || n_frames > h->p.max_frames) return h->fail(COFIE_EINVAL, "n_frames must be in [1, max_frames]");
+  if (!q || !k || !sel_out || !k_out) return h->fail(COFIE_EINVAL, "q, k, sel_out and k_out are required");
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != h->device) cudaSetDevice(h->device);
+  struct Restore {
+    int prev, dev;
+    ~Restore() {
+      if (prev >= 0 && prev != dev) cudaSetDevice(prev);
+    }
+  } restore{prev, h->device};
+  if (!is_device(q, h->device) || !is_device(k, h->device) || !is_device(sel_out, h->device) ||
+      (w_out && !is_device(w_out, h->device)))
+    return h->fail(COFIE_EINVAL, "q, k, w_out and sel_out must be device memory on the handle's device");
+  if (reinterpret_cast<uintptr_t>(k) % 16 != 0) return h->fail(COFIE_EINVAL, "k must be 16-byte aligned");
+  const cofie_qer_params& p = h->p;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const uint64_t nv = static_cast<uint64_t>(n_frames) * p.tokens_per_frame;
+  CUtensorMap map_k, map_q;
+  if (!make_map(&map_k, k, nv, h->D, kQerM) || !make_map(&map_q, h->d_qg, h->n_pad, h->D, h->n_pad))
+    return h->fail(COFIE_ECUDA, "tensor map encoding failed");
+  qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, h->n_pad, p.n_heads, p.n_kv_heads, p.head_dim, h->d_qg);
+  const uint32_t tiles = static_cast<uint32_t>((nv + kQerM - 1) / kQerM);
+  qer_score<<<tiles, kQerThreads, qer_smem_bytes(h->n_pad), st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text,
+                                                                   h->n_pad, h->tmem_cols, h->D / kQerKChunk,
+                                                                   h->d_colmax, h->d_err, 2000000000ull);
+  const uint32_t kk = static_cast<uint32_t>(std::max(1.0, std::nearbyint(static_cast<double>(p.rho) * n_frames)));
+  const float scale = static_cast<float>(1.0 / (static_cast<double>(p.n_heads) * std::sqrt(static_cast<double>(p.head_dim))));
+  float* w = w_out ? w_out : h->d_w;
+  uint32_t* kdev = is_device(k_out, h->device) ? k_out : h->d_k;
+  qer_select<<<1, kSelThreads, 0, st>>>(h->d_colmax, n_frames, p.tokens_per_frame, scale, kk, w, sel_out, kdev);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess && kdev != k_out) {
+    e = cudaMemcpyAsync(k_out, kdev, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  }
+  if (e != cudaSuccess) return h->fail(COFIE_ECUDA, std::string("QER launch: ") + cudaGetErrorString(e));
+  return COFIE_OK;
+}
+
+int cofie_qer_status(cofie_qer_t* h, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  int prev = -1;
+  cudaGetDevice(&prev);
+  cudaSetDevice(h->device);
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(cuda_stream));
+  uint32_t word = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&word, h->d_err, sizeof word, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && word) cudaMemset(h->d_err, 0, sizeof word);
+  if (prev >= 0) cudaSetDevice(prev);
+  if (e != cudaSuccess) return h->fail(COFIE_ECUDA, cudaGetErrorString(e));
+  if (word) return h->fail(COFIE_ETIMEOUT, "a device-side wait of the QER kernels ran out");
+  return COFIE_OK;
+}
+
+const char* cofie_qer_last_error(const cofie_qer_t* h) { return h ? h->err.c_str() : g_qer_error.c_str(); }
+
+}  // extern "C"

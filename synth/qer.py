@@ -26,6 +26,7 @@ class QerSpec:
     tokens_per_frame: int = 256
     n_evidence: int = 8
     seed: int = 0xC0F1E0A0
+    integer: bool = False  # small integers in [-4, 4]: every product and sum is exact in fp32
 
     @property
     def n_visual(self) -> int:
@@ -53,6 +54,10 @@ def generate(spec: QerSpec):
     """Returns (q_bits [n_text, H, d] uint16, k_bits [n_visual, H_kv, d] uint16,
     evidence_frames sorted int array)."""
     g = np.random.Generator(np.random.Philox(spec.seed))
+    if spec.integer:
+        q = g.integers(-4, 5, size=(spec.n_text, spec.n_heads, spec.head_dim)).astype(np.float32)
+        k = g.integers(-4, 5, size=(spec.n_visual, spec.n_kv_heads, spec.head_dim)).astype(np.float32)
+        return to_bf16_bits(q), to_bf16_bits(k), np.zeros(0, dtype=np.int64)
     q = g.standard_normal((spec.n_text, spec.n_heads, spec.head_dim), dtype=np.float32)
     k = g.standard_normal((spec.n_visual, spec.n_kv_heads, spec.head_dim), dtype=np.float32)
     ev = np.sort(g.choice(spec.n_frames, size=min(spec.n_evidence, spec.n_frames), replace=False))

@@ -14,7 +14,7 @@ HEADER = os.path.join(REPO, "include", "cofie_ngff.h")
 def _declared():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(cofie_ngff_[a-z_]+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(cofie_(?:ngff|qer)_[a-z_]+)\s*\(", text)))
 
 
 @pytest.fixture(scope="module")

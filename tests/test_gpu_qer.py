@@ -1,0 +1,100 @@
+"""QER on the tensor cores (tcgen05) against the float64 oracle of Eqs. 6-8.
+
+Frame scores w_f must lie within the oracle's error bound for a bf16
+group-sum + fp32 accumulation computation (plus fp32 rounding of the frame
+mean). The selection must be a valid TopK of the GPU's own scores (exact),
+and equal to the oracle's selection for every frame that is not within the
+bound of the cut (near ties may go either way)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import qer_oracle as Q
+from synth import qer as S
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def _run_gpu(spec, rho):
+    from paper_2609_03675_gb300 import QER
+    q, k, ev = S.generate(spec)
+    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, rho)
+    qd = torch.from_numpy(q.view(np.int16)).cuda()
+    kd = torch.from_numpy(k.view(np.int16)).cuda()
+    w, sel = f.run(qd, kd)
+    torch.cuda.synchronize()
+    f.status()
+    return q, k, ev, w.cpu().numpy().astype(np.float64), sel.cpu().numpy().astype(np.int64)
+
+
+def check(spec, rho, frames=None):
+    q, k, ev, w_gpu, sel_gpu = _run_gpu(spec, rho)
+    rho32 = float(np.float32(rho))
+    m = spec.n_frames
+    kk = Q.keep_count(m, rho32)
+    # selection is a valid TopK of the GPU's own scores (ties: lower index)
+    assert list(sel_gpu) == list(Q.select(w_gpu, rho32)), "GPU selection is not the TopK of its own scores"
+    frames = np.arange(m) if frames is None else np.asarray(frames)
+    w_o = Q.frame_relevance_subset(q, k, spec.tokens_per_frame, frames)
+    bound = Q.score_bound(q, k, spec.tokens_per_frame, frames) + 2.0 ** -18 * np.abs(w_o)
+    err = np.abs(w_gpu[frames] - w_o)
+    assert np.all(err <= bound), f"scores off by {err.max():.3e} > bound {bound[np.argmax(err - bound)]:.3e}"
+    if len(frames) == m:
+        sel_o = Q.select(w_o, rho32)
+        cut = np.sort(w_o)[::-1][kk - 1]
+        clear = np.abs(w_o - cut) > 2 * bound.max()
+        in_o = np.isin(np.arange(m), sel_o)
+        in_g = np.isin(np.arange(m), sel_gpu)
+        assert np.array_equal(in_o[clear], in_g[clear]), "selection differs away from the cut"
+    return w_gpu, sel_gpu, ev, err.max(), bound.min()
+
+
+@pytest.mark.parametrize("spec,rho", [
+    (S.QerSpec(n_text=40, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=6, tokens_per_frame=40, n_evidence=2,
+               seed=1), 0.5),
+    (S.QerSpec(n_text=16, n_heads=4, n_kv_heads=4, head_dim=64, n_frames=5, tokens_per_frame=64, n_evidence=1,
+               seed=2), 0.2),
+    (S.QerSpec(n_text=1, n_heads=2, n_kv_heads=1, head_dim=64, n_frames=9, tokens_per_frame=16, n_evidence=3,
+               seed=3), 0.34),
+    (S.QerSpec(n_text=129, n_heads=16, n_kv_heads=4, head_dim=64, n_frames=7, tokens_per_frame=100, n_evidence=2,
+               seed=4), 0.3),
+    (S.QerSpec(n_text=256, n_heads=32, n_kv_heads=8, head_dim=128, n_frames=16, tokens_per_frame=256, n_evidence=4,
+               seed=5), 0.25),
+])
+def test_qer_small_and_ragged(spec, rho):
+    check(spec, rho)
+
+
+@pytest.mark.parametrize("spec", [
+    S.QerSpec(n_text=256, n_heads=32, n_kv_heads=8, head_dim=128, n_frames=12, tokens_per_frame=256, integer=True,
+              seed=7),
+    S.QerSpec(n_text=37, n_heads=8, n_kv_heads=2, head_dim=96, n_frames=5, tokens_per_frame=52, integer=True, seed=8),
+])
+def test_qer_exact_on_integer_inputs(spec):
+    """Integer inputs in [-4, 4]: head-group sums, products and the fp32
+    accumulation are all exact, so only the final scaling and the frame mean
+    round (a few fp32 ulps of w)."""
+    q, k, _, w_gpu, _ = _run_gpu(spec, 0.5)
+    w_o = Q.frame_relevance(Q.token_scores(q, k), spec.tokens_per_frame)
+    assert np.all(np.abs(w_gpu - w_o) <= 2.0 ** -21 * np.abs(w_o)), np.abs(w_gpu - w_o).max()
+
+
+def test_qer_planted_evidence_found():
+    spec = S.QerSpec(n_text=64, n_heads=32, n_kv_heads=8, head_dim=128, n_frames=32, tokens_per_frame=64,
+                     n_evidence=4, seed=6)
+    w, sel, ev, _, _ = check(spec, 4 / 32)
+    assert list(sel) == list(ev)
+
+
+def test_qer_full_size_sampled():
+    """The benchmark's geometry: 256 text tokens, 128 frames x 256 tokens,
+    32/8 heads of 128; the oracle checks 12 sampled frames."""
+    spec = S.QerSpec()
+    frames = np.linspace(0, spec.n_frames - 1, 12).astype(int)
+    check(spec, 0.3, frames=frames)
