@@ -45,9 +45,11 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather"], default="hd1080",
+    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer"],
+                    default="hd1080",
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
+    ap.add_argument("--qer-frames", type=int, default=128, help="candidate frames of the qer workload")
     ap.add_argument("--frames", type=int, default=3600,
                     help="use the first FRAMES frames of the stream (small cases for profiling; default all 3600)")
     return ap.parse_args()
@@ -573,6 +575,66 @@ def bench_gather(args):
                       "frac": gbs / peak, "peak_kind": f"{kind} copy bandwidth (read + write)"}), flush=True)
 
 
+def peaks_bf16():
+    try:
+        with open(os.path.join(REPO, "MEASURED_PEAKS.json")) as fh:
+            d = json.load(fh)
+        return float(d["bf16_tflops"]), "measured"
+    except Exception:  # noqa: BLE001
+        return 1900.0, "fallback"
+
+
+def bench_qer(args):
+    """QER frame scoring (Eqs. 6-8) on the Qwen3-VL-8B last-layer geometry:
+    256 text tokens, 32 query / 8 key heads of 128, 256 tokens per frame.
+    Roofline of the tensor-core scoring kernel against both the measured
+    bf16 dense peak and the measured copy bandwidth."""
+    import numpy as np
+    import torch
+
+    from paper_2609_03675_gb300 import QER
+    from synth import qer as SQ
+    spec = SQ.QerSpec(n_frames=args.qer_frames)
+    q, k, ev = SQ.generate(spec)
+    qd = torch.from_numpy(q.view(np.int16)).cuda()
+    kd = torch.from_numpy(k.view(np.int16)).cuda()
+    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3)
+    w = torch.empty(spec.n_frames, dtype=torch.float32, device="cuda")
+    sel_all = torch.empty(spec.n_frames, dtype=torch.int32, device="cuda")
+    k_dev = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for _ in range(5):
+        f.run_async(qd, kd, w, sel_all, k_dev)
+    torch.cuda.synchronize()
+    f.profile_reset(time_kernels=True)
+    reps = 200
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        f.run_async(qd, kd, w, sel_all, k_dev)
+    e1.record()
+    torch.cuda.synchronize()
+    f.status()
+    sel = sel_all[: int(k_dev.item())]
+    pr = f.profile_read()
+    k_ms = pr["score_ms"] / max(pr["timed"], 1)
+    tflops = pr["flops"] / pr["launches"] / (k_ms / 1e3) / 1e12
+    gbs = pr["key_bytes"] / pr["launches"] / (k_ms / 1e3) / 1e9
+    tc_peak, tc_kind = peaks_bf16()
+    hbm_peak, hbm_kind = peaks()
+    print(json.dumps({
+        "workload": f"qer: {spec.n_text} text tokens, {spec.n_frames} frames x {spec.tokens_per_frame} tokens, "
+                    f"{spec.n_heads}/{spec.n_kv_heads} heads of {spec.head_dim}, rho 0.3",
+        "call_us": e0.elapsed_time(e1) / reps * 1e3, "score_kernel_us": k_ms * 1e3,
+        "frames_per_s": spec.n_frames / (e0.elapsed_time(e1) / reps / 1e3),
+        "tensor": {"achieved": tflops, "peak": tc_peak, "unit": "TFLOP/s", "frac": tflops / tc_peak,
+                   "peak_kind": f"{tc_kind} bf16 dense (burst)",
+                   "flops_per_launch": pr["flops"] / pr["launches"]},
+        "hbm": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                "peak_kind": f"{hbm_kind} copy bandwidth", "key_bytes_per_launch": pr["key_bytes"] / pr["launches"]},
+        "selected": int(sel.numel()), "evidence_recovered": int(np.isin(ev, sel.cpu().numpy()).sum()),
+        "n_evidence": int(len(ev))}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -585,6 +647,8 @@ def main():
         bench_rare_event(args)
     elif args.workload == "gather":
         bench_gather(args)
+    elif args.workload == "qer":
+        bench_qer(args)
     else:
         bench_gb300(args)
 

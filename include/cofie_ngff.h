@@ -320,6 +320,15 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
 /* Synchronises cuda_stream; COFIE_ETIMEOUT if a bounded device wait ran out. */
 int cofie_qer_status(cofie_qer_t* h, void* cuda_stream);
 
+/* Launch counter and CUDA-event timing of the scoring (tensor-core) kernel:
+ * reset zeroes the counters (time_kernels != 0 brackets every launch with two
+ * events on its stream); read waits for the timed launches and reports the
+ * launches, the timed launches, their summed milliseconds, the contraction's
+ * FLOPs (2 N n_visual D, N the padded text count) and the key bytes read. */
+int cofie_qer_profile_reset(cofie_qer_t* h, int time_kernels);
+int cofie_qer_profile_read(cofie_qer_t* h, uint64_t* launches, uint64_t* timed, double* score_ms, double* flops,
+                           double* key_bytes);
+
 /* Last error of h, or of the last failed cofie_qer_create when h is NULL. Never NULL. */
 const char* cofie_qer_last_error(const cofie_qer_t* h);
 

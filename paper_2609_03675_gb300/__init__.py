@@ -237,9 +237,29 @@ class QER:
                                             ctypes.addressof(kk), st))
         return w, sel[: kk.value]
 
+    def run_async(self, q: torch.Tensor, k: torch.Tensor, w: torch.Tensor, sel: torch.Tensor, k_dev: torch.Tensor,
+                  n_frames: int | None = None, cuda_stream=None):
+        """run() with every output in device memory (no synchronisation):
+        w [n_frames] float32, sel [n_frames] int32 (first k_dev[0] entries valid)."""
+        T = self.params.tokens_per_frame
+        n = k.shape[0] // T if n_frames is None else n_frames
+        st = torch.cuda.current_stream(self.device).cuda_stream if cuda_stream is None else int(cuda_stream)
+        self._check(self._lib.cofie_qer_run(self._h, _ptr(q), _ptr(k), n, _ptr(w), _ptr(sel), _ptr(k_dev), st))
+
     def status(self, cuda_stream=None):
         st = torch.cuda.current_stream(self.device).cuda_stream if cuda_stream is None else int(cuda_stream)
         self._check(self._lib.cofie_qer_status(self._h, st))
+
+    def profile_reset(self, time_kernels: bool = False):
+        self._check(self._lib.cofie_qer_profile_reset(self._h, int(time_kernels)))
+
+    def profile_read(self) -> dict:
+        la, ti = ctypes.c_uint64(0), ctypes.c_uint64(0)
+        ms, fl, kb = ctypes.c_double(0), ctypes.c_double(0), ctypes.c_double(0)
+        self._check(self._lib.cofie_qer_profile_read(self._h, ctypes.byref(la), ctypes.byref(ti), ctypes.byref(ms),
+                                                     ctypes.byref(fl), ctypes.byref(kb)))
+        return {"launches": la.value, "timed": ti.value, "score_ms": ms.value, "flops": fl.value,
+                "key_bytes": kb.value}
 
     def close(self):
         if getattr(self, "_h", None):

@@ -39,6 +39,8 @@ EXPORTS = (
     "cofie_qer_destroy",
     "cofie_qer_run",
     "cofie_qer_status",
+    "cofie_qer_profile_reset",
+    "cofie_qer_profile_read",
     "cofie_qer_last_error",
 )
 
@@ -154,6 +156,12 @@ def load():
     lib.cofie_qer_run.restype = ctypes.c_int
     lib.cofie_qer_status.argtypes = [H, vp]
     lib.cofie_qer_status.restype = ctypes.c_int
+    lib.cofie_qer_profile_reset.argtypes = [H, ctypes.c_int]
+    lib.cofie_qer_profile_reset.restype = ctypes.c_int
+    pu64 = ctypes.POINTER(ctypes.c_uint64)
+    pdbl = ctypes.POINTER(ctypes.c_double)
+    lib.cofie_qer_profile_read.argtypes = [H, pu64, pu64, pdbl, pdbl, pdbl]
+    lib.cofie_qer_profile_read.restype = ctypes.c_int
     lib.cofie_qer_last_error.argtypes = [H]
     lib.cofie_qer_last_error.restype = ctypes.c_char_p
     lib.cofie_ngff_last_error.argtypes = [H]

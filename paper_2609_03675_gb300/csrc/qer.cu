@@ -17,17 +17,20 @@
 // Kernels:
 //   qer_prepare_q   q [n_text][H][d] -> q~ [N][D] bf16 (fp32 sums rounded to
 //                   nearest even; rows n_text..N-1 zero, N = n_text rounded up to 16)
-//   qer_score       one CTA per 128 visual tokens: TMA (cp.async.bulk.tensor,
-//                   128-byte swizzle) streams 64-wide K chunks of the token
-//                   tile and of q~ into a 4-stage shared-memory ring; one thread
-//                   issues tcgen05.mma (kind::f16, M = 128, N, K = 16) into a
-//                   TMEM accumulator (128 lanes x N fp32 columns) and commits
-//                   each stage back to the producer; four warps then read their
-//                   32 TMEM lanes (tcgen05.ld) and keep each token's max over
-//                   the n_text real columns.
-//   qer_select      one CTA: w_f = (sum of the frame's token maxima) / (|V_f| H sqrt(d)),
-//                   then the k best frames by rank (ties to the lower index),
-//                   compacted in time order.
+//   qer_score       persistent CTAs over tiles of 256 visual tokens: TMA
+//                   (cp.async.bulk.tensor, 128-byte swizzle) streams 64-wide K
+//                   chunks of the token tile and of q~ into a shared-memory
+//                   ring; one thread issues tcgen05.mma (kind::f16, M = 128 per
+//                   half tile, N, K = 16) into TMEM accumulators (128 lanes x N
+//                   fp32 columns per half) and commits each stage back to the
+//                   producer; four epilogue warps read the accumulators
+//                   (tcgen05.ld) and keep each token's max over the n_text real
+//                   columns.
+//   qer_mean        w_f = (sum of the frame's token maxima) / (|V_f| H sqrt(d)),
+//                   a warp per frame;
+//   qer_rank        the k best frames by rank (ties to the lower index), a
+//                   thread per frame against all scores staged in shared memory;
+//   qer_compact     the kept frames in time order (one CTA).
 // Every mbarrier wait is bounded by the global timer; a wait that runs out
 // sets an error bit, stops issuing, lets the work already issued finish
 // (bounded) and frees TMEM before the CTA exits.
@@ -40,6 +43,7 @@
 #include <cstring>
 #include <new>
 #include <string>
+#include <vector>
 
 #include "cofie_ngff.h"
 #include "ngff_common.cuh"
@@ -47,13 +51,18 @@
 namespace cofie {
 namespace {
 
-constexpr int kQerM = 128;          // visual tokens per CTA (MMA M)
+constexpr int kQerM = 128;          // visual tokens per MMA (M)
+constexpr int kQerTile = 2 * kQerM; // visual tokens per tile: two MMAs share each q~ chunk
 constexpr int kQerKChunk = 64;      // bf16 elements per 128-byte swizzled row
-constexpr int kQerStages = 4;
+constexpr uint32_t kQerMaxStages = 8;
+constexpr size_t kQerStageBudget = 200 * 1024;  // shared memory for the ring
 constexpr int kQerUmmaK = 16;       // K of one tcgen05.mma for 16-bit inputs
-constexpr int kQerThreads = 128;    // four warps: TMEM lanes 0..127
+constexpr int kQerEpiWarps = 4;    // epilogue warps: TMEM lanes 0..127
+constexpr int kQerThreads = 32 * (2 + kQerEpiWarps);  // + TMA producer warp + MMA issuer warp
 constexpr uint32_t kQerMaxN = 256;  // text tokens (MMA N) per CTA
 constexpr int kSelThreads = 1024;
+constexpr int kRankThreads = 64;  // few warps per CTA: the O(m^2) ranking spreads over many SMs
+constexpr uint32_t kSelSmemFrames = 11264;  // frame scores staged in 44 KiB of shared memory (within the default limit)
 
 constexpr uint32_t kQerErrProducer = 16u, kQerErrMma = 32u, kQerErrEpilogue = 64u, kQerErrDrain = 128u;
 
@@ -131,9 +140,8 @@ __device__ __forceinline__ void umma_commit(uint32_t bar) {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
+// 32 consecutive fp32 columns of this thread's TMEM lane, without waiting.
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t* r) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
       "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
@@ -142,9 +150,30 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
         "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
         "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Max over the first n_text columns of this thread's TMEM lane (n_pad columns,
+// a multiple of 16), reading 64 columns per wait.
+__device__ __forceinline__ float tmem_row_max(uint32_t taddr, uint32_t n_pad, uint32_t n_text) {
+  float best = -INFINITY;
+  for (uint32_t c0 = 0; c0 < n_pad; c0 += 64) {
+    uint32_t r0[32], r1[32];
+    tmem_ld32_nowait(taddr + c0, r0);
+    const bool two = c0 + 32 < n_pad;
+    if (two) tmem_ld32_nowait(taddr + c0 + 32, r1);
+    tmem_wait_ld();
 #pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+    for (uint32_t c = 0; c < 32; ++c)
+      if (c0 + c < n_text) best = fmaxf(best, __uint_as_float(r0[c]));
+    if (two) {
+#pragma unroll
+      for (uint32_t c = 0; c < 32; ++c)
+        if (c0 + 32 + c < n_text) best = fmaxf(best, __uint_as_float(r1[c]));
+    }
+  }
+  return best;
 }
 
 __global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H,
@@ -163,138 +192,249 @@ __global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, u
   }
 }
 
-__global__ void __launch_bounds__(kQerThreads, 1) qer_score(const __grid_constant__ CUtensorMap map_k,
-                                                             const __grid_constant__ CUtensorMap map_q,
-                                                             uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
-                                                             uint32_t tmem_cols, uint32_t n_chunks,
-                                                             float* __restrict__ colmax, uint32_t* __restrict__ err,
-                                                             uint64_t timeout_ns) {
-  extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full_bar[kQerStages];
-  __shared__ __align__(8) uint64_t empty_bar[kQerStages];
-  __shared__ __align__(8) uint64_t accum_bar;
-  __shared__ uint32_t tmem_slot;
+// The same with 8 consecutive channels per thread (d % 8 == 0, 16-byte aligned q).
+__global__ void qer_prepare_q8(const uint4* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H, uint32_t H_kv,
+                               uint32_t d, uint4* __restrict__ qg) {
+  const uint32_t d8 = d / 8, D8 = H_kv * d8, G = H / H_kv;
+  const uint64_t total = static_cast<uint64_t>(n_pad) * D8;
+  for (uint64_t e = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<uint64_t>(gridDim.x) * blockDim.x) {
+    const uint32_t i = static_cast<uint32_t>(e / D8), r = static_cast<uint32_t>(e % D8);
+    const uint32_t g = r / d8, c8 = r % d8;
+    float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (i < n_text)
+      for (uint32_t h = g * G; h < (g + 1) * G; ++h) {
+        const uint4 v = q[(static_cast<uint64_t>(i) * H + h) * d8 + c8];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          s[2 * k] += __uint_as_float(w[k] << 16);
+          s[2 * k + 1] += __uint_as_float(w[k] & 0xFFFF0000u);
+        }
+      }
+    uint32_t out[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint32_t lo = static_cast<__nv_bfloat16_raw>(__float2bfloat16_rn(s[2 * k])).x;
+      const uint32_t hi = static_cast<__nv_bfloat16_raw>(__float2bfloat16_rn(s[2 * k + 1])).x;
+      out[k] = lo | (hi << 16);
+    }
+    qg[e] = make_uint4(out[0], out[1], out[2], out[3]);
+  }
+}
 
-  // 1024-byte aligned stage buffers (the 128-byte swizzle repeats every 1024 bytes)
+// Persistent, warp-specialised scoring kernel over tiles of 256 visual
+// tokens (two M = 128 halves sharing every q~ chunk, which halves the q~
+// traffic per token). Warp 0 (one thread) streams TMA chunks of the CTA's
+// tiles into an n_stages ring (per stage: two 16 KiB key halves + the q~
+// chunk); warp 1 (one thread) issues, per 16-wide K step, one MMA per half
+// into accumulator pair t % n_buf (two blocks of acc_cols TMEM columns);
+// warps 2..5 read the pair (warp w owns TMEM lanes 32 (w % 4) ..), so with
+// two buffers the epilogue of tile t overlaps the MMAs of tile t + 1.
+// Barriers: full/empty per ring stage (TMA bytes / MMA completion),
+// tfull/tempty per accumulator pair (MMA completion / the epilogue warps).
+__global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__ CUtensorMap map_k,
+                                                         const __grid_constant__ CUtensorMap map_q,
+                                                         uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
+                                                         uint32_t acc_cols, uint32_t n_buf, uint32_t n_stages,
+                                                         uint32_t n_chunks, uint32_t n_tiles,
+                                                         float* __restrict__ colmax, uint32_t* __restrict__ err,
+                                                         uint64_t timeout_ns) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t tfull_bar[2];
+  __shared__ __align__(8) uint64_t tempty_bar[2];
+  __shared__ __align__(8) uint64_t done_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile uint32_t abort_flag;
+
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t a_bytes = kQerM * 128, b_bytes = n_pad * 128;
+  const uint32_t half_bytes = kQerM * 128, a_bytes = 2 * half_bytes, b_bytes = n_pad * 128;
   const uint32_t stage_bytes = a_bytes + ((b_bytes + 1023) & ~1023u);
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const uint32_t row0 = blockIdx.x * kQerM;
+  const uint32_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+  const uint32_t tmem_total = 2 * acc_cols * n_buf;
 
-  if (warp == 0) {  // the whole warp allocates the accumulator columns
+  if (warp == 0) {  // the whole warp allocates the accumulators
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
-                 "r"(tmem_cols)
+                 "r"(tmem_total)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   if (threadIdx.x == 32) {
-    for (int s = 0; s < kQerStages; ++s) {
+    for (uint32_t s = 0; s < n_stages; ++s) {
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full_bar[s])) : "memory");
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&empty_bar[s])) : "memory");
     }
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&accum_bar)) : "memory");
+    for (int b = 0; b < 2; ++b) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&tfull_bar[b])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&tempty_bar[b])), "r"(kQerEpiWarps)
+                   : "memory");
+    }
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&done_bar)) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    abort_flag = 0;
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
-  if (warp == 0 && lane == 0) {
-    // ------------------------------------------------------------- TMA producer
-    uint32_t issued = 0;
-    for (uint32_t kc = 0; kc < n_chunks; ++kc) {
-      const uint32_t s = kc % kQerStages, use = kc / kQerStages;
-      if (use > 0 && !mbar_wait_for(smem_u32(&empty_bar[s]), (use - 1) & 1, timeout_ns)) {
-        atomicOr(err, kQerErrProducer);
-        break;
+  if (warp == 0) {
+    if (lane == 0) {
+      // --------------------------------------------------------- TMA producer
+      uint32_t g = 0;  // chunk counter over all of this CTA's tiles
+      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
+        const uint32_t row0 = (blockIdx.x + t * gridDim.x) * kQerTile;
+        for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
+          const uint32_t s = g % n_stages, use = g / n_stages;
+          if (use > 0 && !mbar_wait_for(smem_u32(&empty_bar[s]), (use - 1) & 1, timeout_ns)) {
+            atomicOr(err, kQerErrProducer);
+            abort_flag = 1;
+            break;
+          }
+          if (abort_flag) break;
+          const uint32_t fb = smem_u32(&full_bar[s]);
+          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(a_bytes + b_bytes)
+                       : "memory");
+          const uint32_t base = smem_u32(smem + s * stage_bytes);
+          const int32_t x = static_cast<int32_t>(kc * kQerKChunk);
+          tma_load_2d(base, &map_k, x, static_cast<int32_t>(row0), fb);
+          tma_load_2d(base + half_bytes, &map_k, x, static_cast<int32_t>(row0 + kQerM), fb);
+          tma_load_2d(base + a_bytes, &map_q, x, 0, fb);
+        }
       }
-      const uint32_t fb = smem_u32(&full_bar[s]);
-      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(a_bytes + b_bytes)
-                   : "memory");
-      const uint32_t base = smem_u32(smem + s * stage_bytes);
-      tma_load_2d(base, &map_k, static_cast<int32_t>(kc * kQerKChunk), static_cast<int32_t>(row0), fb);
-      tma_load_2d(base + a_bytes, &map_q, static_cast<int32_t>(kc * kQerKChunk), 0, fb);
-      ++issued;
+      // no copy may still be writing shared memory when the CTA exits
+      for (uint32_t j = g > n_stages ? g - n_stages : 0; j < g; ++j)
+        if (!mbar_wait_for(smem_u32(&full_bar[j % n_stages]), (j / n_stages) & 1, timeout_ns))
+          atomicOr(err, kQerErrDrain);
     }
-    // no copy may still be writing shared memory when the CTA exits
-    for (uint32_t j = issued > kQerStages ? issued - kQerStages : 0; j < issued; ++j)
-      if (!mbar_wait_for(smem_u32(&full_bar[j % kQerStages]), (j / kQerStages) & 1, timeout_ns))
-        atomicOr(err, kQerErrDrain);
-  } else if (warp == 1 && lane == 0) {
-    // ----------------------------------------------------------- MMA issuer
-    const uint32_t idesc = idesc_bf16_f32(kQerM, n_pad);
-    for (uint32_t kc = 0; kc < n_chunks; ++kc) {
-      const uint32_t s = kc % kQerStages, use = kc / kQerStages;
-      if (!mbar_wait_for(smem_u32(&full_bar[s]), use & 1, timeout_ns)) {
-        atomicOr(err, kQerErrMma);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ----------------------------------------------------------- MMA issuer
+      const uint32_t idesc = idesc_bf16_f32(kQerM, n_pad);
+      uint32_t g = 0;
+      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
+        const uint32_t b = t % n_buf, ub = t / n_buf;
+        if (ub > 0 && !mbar_wait_for(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
+          atomicOr(err, kQerErrMma);
+          abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc0 = tmem + b * 2 * acc_cols, acc1 = acc0 + acc_cols;
+        bool stop = false;
+        for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
+          const uint32_t s = g % n_stages, use = g / n_stages;
+          if (!mbar_wait_for(smem_u32(&full_bar[s]), use & 1, timeout_ns) || abort_flag) {
+            atomicOr(err, kQerErrMma);
+            abort_flag = 1;
+            stop = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(smem + s * stage_bytes), a1 = a0 + half_bytes, b0 = a0 + a_bytes;
+#pragma unroll
+          for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk) {
+            const uint64_t bd = sw128_desc(b0 + kk * 32);
+            umma_bf16(acc0, sw128_desc(a0 + kk * 32), bd, idesc, (kc | kk) != 0);
+            umma_bf16(acc1, sw128_desc(a1 + kk * 32), bd, idesc, (kc | kk) != 0);
+          }
+          umma_commit(smem_u32(&empty_bar[s]));  // the stage is free once these MMAs have read it
+        }
+        if (stop) break;
+        umma_commit(smem_u32(&tfull_bar[b]));  // accumulator pair b holds tile t
+      }
+      umma_commit(smem_u32(&done_bar));  // every MMA this CTA issued is complete
+    }
+  } else {
+    // --------------------------------------------------------------- epilogue
+    const uint32_t quarter = warp & 3;  // TMEM lanes this warp may read
+    for (uint32_t t = 0; t < my_tiles; ++t) {
+      const uint32_t b = t % n_buf, ub = t / n_buf;
+      bool ok = !abort_flag && mbar_wait_for(smem_u32(&tfull_bar[b]), ub & 1, timeout_ns);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) {
+        if (lane == 0) atomicOr(err, kQerErrEpilogue);
+        abort_flag = 1;
         break;
       }
       tc_fence_after();
-      const uint32_t a0 = smem_u32(smem + s * stage_bytes), b0 = a0 + a_bytes;
-#pragma unroll
-      for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk)
-        umma_bf16(tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), idesc, (kc | kk) != 0);
-      umma_commit(smem_u32(&empty_bar[s]));  // the stage is free once these MMAs have read it
+      const uint32_t row0 = (blockIdx.x + t * gridDim.x) * kQerTile;
+#pragma unroll 1
+      for (uint32_t half = 0; half < 2; ++half) {
+        const uint32_t taddr = tmem + (b * 2 + half) * acc_cols + ((quarter * 32u) << 16);
+        const float best = tmem_row_max(taddr, n_pad, n_text);
+        const uint32_t j = row0 + half * kQerM + quarter * 32 + lane;
+        if (j < n_visual) colmax[j] = best;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&tempty_bar[b])) : "memory");
     }
-    umma_commit(smem_u32(&accum_bar));  // every MMA issued so far is complete
   }
   __syncwarp();
-
-  // ------------------------------------------------------------- epilogue
-  const bool ok = mbar_wait_for(smem_u32(&accum_bar), 0, timeout_ns);
-  if (!ok && lane == 0) atomicOr(err, kQerErrEpilogue);
-  tc_fence_after();
-  float best = -INFINITY;
-  const uint32_t taddr = tmem + ((warp * 32u) << 16);
-  for (uint32_t c0 = 0; c0 < n_pad; c0 += 32) {
-    float v[32];
-    tmem_ld32(taddr + c0, v);
-#pragma unroll
-    for (uint32_t c = 0; c < 32; ++c)
-      if (c0 + c < n_text) best = fmaxf(best, v[c]);
+  // TMEM is freed only after every MMA this CTA issued has completed
+  if (warp == 0) {
+    const bool ok = mbar_wait_for(smem_u32(&done_bar), 0, timeout_ns);
+    if (!ok && lane == 0) atomicOr(err, kQerErrDrain);
   }
-  const uint32_t j = row0 + warp * 32 + lane;
-  if (ok && j < n_visual) colmax[j] = best;
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_cols) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_total) : "memory");
   }
 }
 
-__global__ void __launch_bounds__(kSelThreads) qer_select(const float* __restrict__ colmax, uint32_t n_frames,
-                                                          uint32_t tpf, float scale, uint32_t k,
-                                                          float* __restrict__ w, uint32_t* __restrict__ sel,
-                                                          uint32_t* __restrict__ k_out) {
+// Eq. 7: w_f = mean over the frame's tokens of their max over text, times the
+// 1/(H sqrt(d)) of Eq. 6. One warp per frame.
+__global__ void __launch_bounds__(256) qer_mean(const float* __restrict__ colmax, uint32_t n_frames, uint32_t tpf,
+                                                float scale, float* __restrict__ w) {
+  const uint32_t f = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (f >= n_frames) return;
+  float s = 0.f;
+  for (uint32_t t = lane; t < tpf; t += 32) s += colmax[static_cast<uint64_t>(f) * tpf + t];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) w[f] = s / static_cast<float>(tpf) * scale;
+}
+
+// Eq. 8: flag[f] = 1 when fewer than k frames rank above frame f (higher w,
+// or equal w and lower index). Each CTA stages all scores in shared memory
+// (or reads them from global memory when they do not fit); a thread per frame.
+__global__ void __launch_bounds__(kRankThreads) qer_rank(const float* __restrict__ w, uint32_t n_frames, uint32_t k,
+                                                uint8_t* __restrict__ flag) {
+  extern __shared__ float sw[];
+  const bool in_smem = n_frames <= kSelSmemFrames;
+  if (in_smem)
+    for (uint32_t g = threadIdx.x; g < n_frames; g += blockDim.x) sw[g] = w[g];
+  __syncthreads();
+  const float* ws = in_smem ? sw : w;
+  const uint32_t f = blockIdx.x * blockDim.x + threadIdx.x;
+  if (f >= n_frames) return;
+  const float wf = ws[f];
+  uint32_t above = 0;
+#pragma unroll 8
+  for (uint32_t g = 0; g < n_frames; ++g) {
+    const float wg = ws[g];  // the same word for the whole warp: a broadcast
+    above += (wg > wf) | ((wg == wf) & (g < f));
+  }
+  flag[f] = above < k;
+}
+
+// The flagged frames, in time order: block-wide compaction (ballot,
+// popcount, a scan of the 32 warp totals), 1024 frames per pass.
+__global__ void __launch_bounds__(kSelThreads) qer_compact(const uint8_t* __restrict__ flag, uint32_t n_frames,
+                                                           uint32_t* __restrict__ sel, uint32_t* __restrict__ k_out) {
   __shared__ uint32_t wsum[32];
   __shared__ uint32_t s_total;
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  // Eq. 7: mean over the frame's tokens of their max over text (then the 1/(H sqrt(d)) of Eq. 6)
-  for (uint32_t f = warp; f < n_frames; f += kSelThreads / 32) {
-    float s = 0.f;
-    for (uint32_t t = lane; t < tpf; t += 32) s += colmax[static_cast<uint64_t>(f) * tpf + t];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) w[f] = s / static_cast<float>(tpf) * scale;
-  }
-  __syncthreads();
-  // Eq. 8: frame f is kept when fewer than k frames rank above it (ties: lower index first)
   uint32_t base = 0;
   for (uint32_t f0 = 0; f0 < n_frames; f0 += kSelThreads) {
     const uint32_t f = f0 + tid;
-    bool in = false;
-    if (f < n_frames) {
-      const float wf = w[f];
-      uint32_t above = 0;
-      for (uint32_t g = 0; g < n_frames && above < k; ++g) {
-        const float wg = w[g];
-        above += (wg > wf) || (wg == wf && g < f);
-      }
-      in = above < k;
-    }
+    const bool in = f < n_frames && flag[f];
     const uint32_t bal = __ballot_sync(0xffffffffu, in);
     const uint32_t before = __popc(bal & ((1u << lane) - 1u));
     if (lane == 0) wsum[warp] = __popc(bal);
@@ -318,9 +458,15 @@ __global__ void __launch_bounds__(kSelThreads) qer_select(const float* __restric
   if (tid == 0) *k_out = base;
 }
 
+uint32_t qer_stage_bytes(uint32_t n_pad) { return 2 * kQerM * 128 + ((n_pad * 128 + 1023) & ~1023u); }
+
+uint32_t qer_stages(uint32_t n_pad) {
+  const size_t n = kQerStageBudget / qer_stage_bytes(n_pad);
+  return static_cast<uint32_t>(n < kQerMaxStages ? n : kQerMaxStages);
+}
+
 size_t qer_smem_bytes(uint32_t n_pad) {
-  const uint32_t stage = kQerM * 128 + ((n_pad * 128 + 1023) & ~1023u);
-  return static_cast<size_t>(kQerStages) * stage + 1024;  // + slack for the 1024-byte alignment
+  return static_cast<size_t>(qer_stages(n_pad)) * qer_stage_bytes(n_pad) + 1024;  // + slack for 1024-B alignment
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
@@ -357,13 +503,22 @@ using namespace cofie;
 struct cofie_qer {
   cofie_qer_params p{};
   int device = 0;
-  uint32_t n_pad = 0, D = 0, tmem_cols = 0;
+  uint32_t n_pad = 0, D = 0, acc_cols = 0, n_buf = 1, n_stages = 0;
+  int grid = 0;          // persistent CTAs
+  size_t smem = 0;       // dynamic shared memory per CTA
   __nv_bfloat16_raw* d_qg = nullptr;
   float* d_colmax = nullptr;
   float* d_w = nullptr;
+  uint8_t* d_flag = nullptr;
   uint32_t* d_k = nullptr;
   uint32_t* d_err = nullptr;
   std::string err;
+  // launch counter and optional event timing of the scoring kernel
+  bool time_on = false;
+  uint64_t launches = 0;
+  double flops = 0.0, key_bytes = 0.0;
+  std::vector<cudaEvent_t> ev;
+  size_t ev_used = 0;
   int fail(int code, const std::string& m) {
     err = m;
     return code;
@@ -387,9 +542,10 @@ void qer_free(cofie_qer* h) {
   cudaGetDevice(&prev);
   cudaSetDevice(h->device);
   cudaDeviceSynchronize();
-  void* bufs[] = {h->d_qg, h->d_colmax, h->d_w, h->d_k, h->d_err};
+  void* bufs[] = {h->d_qg, h->d_colmax, h->d_w, h->d_k, h->d_err, h->d_flag};
   for (void* b : bufs)
     if (b) cudaFree(b);
+  for (cudaEvent_t e : h->ev) cudaEventDestroy(e);
   if (prev >= 0) cudaSetDevice(prev);
   delete h;
 }
@@ -427,18 +583,37 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   h->device = dev;
   h->D = static_cast<uint32_t>(D);
   h->n_pad = (p->n_text + 15) / 16 * 16;
-  h->tmem_cols = 32;
-  while (h->tmem_cols < h->n_pad) h->tmem_cols <<= 1;
+  h->acc_cols = 32;
+  while (h->acc_cols < h->n_pad) h->acc_cols <<= 1;
+  // Each tile needs two accumulators of acc_cols TMEM columns; double
+  // buffering (overlapping a tile's epilogue with the next tile's MMAs)
+  // doubles that when it still fits the SM's 512 columns.
+  h->n_buf = (4 * h->acc_cols <= 512) ? 2 : 1;
+  h->n_stages = qer_stages(h->n_pad);
+  // The CTAs resident on one SM must never ask for more than its 512 TMEM
+  // columns, or an allocation would wait for a CTA that only frees its
+  // columns at exit; shared memory is requested large enough to keep the
+  // residency within that limit.
+  const int max_ctas_by_tmem = static_cast<int>(512 / (2 * h->acc_cols * h->n_buf));
+  h->smem = qer_smem_bytes(h->n_pad);
+  const size_t per_sm = 228 * 1024;
+  while (max_ctas_by_tmem >= 1 && per_sm / (h->smem + 1024) > static_cast<size_t>(max_ctas_by_tmem))
+    h->smem += 1024;
   const uint64_t nv = static_cast<uint64_t>(p->max_frames) * p->tokens_per_frame;
   cudaError_t e = cudaMalloc(&h->d_qg, static_cast<size_t>(h->n_pad) * D * 2);
   if (e == cudaSuccess) e = cudaMalloc(&h->d_colmax, nv * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_w, static_cast<size_t>(p->max_frames) * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_k, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMalloc(&h->d_flag, p->max_frames);
   if (e == cudaSuccess) e = cudaMalloc(&h->d_err, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(qer_score, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(qer_smem_bytes(h->n_pad)));
+    e = cudaFuncSetAttribute(qer_score, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(h->smem));
+  int per_sm_ctas = 0, n_sms = 0;
+  if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_ctas, qer_score, kQerThreads, h->smem);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess && (per_sm_ctas < 1 || per_sm_ctas > max_ctas_by_tmem)) e = cudaErrorInvalidConfiguration;
+  h->grid = n_sms * (per_sm_ctas > 0 ? per_sm_ctas : 1);
   if (prev >= 0) cudaSetDevice(prev);
   if (e != cudaSuccess) {
     g_qer_error = std::string("QER set-up failed: ") + cudaGetErrorString(e);
@@ -476,16 +651,45 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   CUtensorMap map_k, map_q;
   if (!make_map(&map_k, k, nv, h->D, kQerM) || !make_map(&map_q, h->d_qg, h->n_pad, h->D, h->n_pad))
     return h->fail(COFIE_ECUDA, "tensor map encoding failed");
-  qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, h->n_pad, p.n_heads, p.n_kv_heads, p.head_dim, h->d_qg);
-  const uint32_t tiles = static_cast<uint32_t>((nv + kQerM - 1) / kQerM);
-  qer_score<<<tiles, kQerThreads, qer_smem_bytes(h->n_pad), st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text,
-                                                                   h->n_pad, h->tmem_cols, h->D / kQerKChunk,
-                                                                   h->d_colmax, h->d_err, 2000000000ull);
+  if (p.head_dim % 8 == 0 && reinterpret_cast<uintptr_t>(q) % 16 == 0) {
+    const uint64_t n8 = static_cast<uint64_t>(h->n_pad) * h->D / 8;
+    const uint32_t blocks = static_cast<uint32_t>(std::min<uint64_t>((n8 + 255) / 256, 1024));
+    qer_prepare_q8<<<blocks, 256, 0, st>>>(reinterpret_cast<const uint4*>(q), p.n_text, h->n_pad, p.n_heads,
+                                           p.n_kv_heads, p.head_dim, reinterpret_cast<uint4*>(h->d_qg));
+  } else {
+    qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, h->n_pad, p.n_heads, p.n_kv_heads, p.head_dim, h->d_qg);
+  }
+  const uint32_t tiles = static_cast<uint32_t>((nv + kQerTile - 1) / kQerTile);
+  const uint32_t grid = tiles < static_cast<uint32_t>(h->grid) ? tiles : static_cast<uint32_t>(h->grid);
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (h->time_on && h->ev_used + 2 <= (1u << 16)) {
+    while (h->ev.size() < h->ev_used + 2) {
+      cudaEvent_t x;
+      if (cudaEventCreate(&x) != cudaSuccess) break;
+      h->ev.push_back(x);
+    }
+    if (h->ev.size() >= h->ev_used + 2) {
+      e0 = h->ev[h->ev_used];
+      e1 = h->ev[h->ev_used + 1];
+      h->ev_used += 2;
+      cudaEventRecord(e0, st);
+    }
+  }
+  qer_score<<<grid, kQerThreads, h->smem, st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
+                                                h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles,
+                                                h->d_colmax, h->d_err, 2000000000ull);
+  if (e1) cudaEventRecord(e1, st);
+  h->launches += 1;
+  h->flops += 2.0 * h->n_pad * static_cast<double>(nv) * h->D;
+  h->key_bytes += 2.0 * static_cast<double>(nv) * h->D;
   const uint32_t kk = static_cast<uint32_t>(std::max(1.0, std::nearbyint(static_cast<double>(p.rho) * n_frames)));
   const float scale = static_cast<float>(1.0 / (static_cast<double>(p.n_heads) * std::sqrt(static_cast<double>(p.head_dim))));
   float* w = w_out ? w_out : h->d_w;
   uint32_t* kdev = is_device(k_out, h->device) ? k_out : h->d_k;
-  qer_select<<<1, kSelThreads, 0, st>>>(h->d_colmax, n_frames, p.tokens_per_frame, scale, kk, w, sel_out, kdev);
+  qer_mean<<<(n_frames + 7) / 8, 256, 0, st>>>(h->d_colmax, n_frames, p.tokens_per_frame, scale, w);
+  const size_t rank_smem = n_frames <= kSelSmemFrames ? n_frames * sizeof(float) : 0;
+  qer_rank<<<(n_frames + kRankThreads - 1) / kRankThreads, kRankThreads, rank_smem, st>>>(w, n_frames, kk, h->d_flag);
+  qer_compact<<<1, kSelThreads, 0, st>>>(h->d_flag, n_frames, sel_out, kdev);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess && kdev != k_out) {
     e = cudaMemcpyAsync(k_out, kdev, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
@@ -507,6 +711,34 @@ int cofie_qer_status(cofie_qer_t* h, void* cuda_stream) {
   if (prev >= 0) cudaSetDevice(prev);
   if (e != cudaSuccess) return h->fail(COFIE_ECUDA, cudaGetErrorString(e));
   if (word) return h->fail(COFIE_ETIMEOUT, "a device-side wait of the QER kernels ran out");
+  return COFIE_OK;
+}
+
+int cofie_qer_profile_reset(cofie_qer_t* h, int time_kernels) {
+  if (!h) return COFIE_EINVAL;
+  h->time_on = time_kernels != 0;
+  h->launches = 0;
+  h->flops = h->key_bytes = 0.0;
+  h->ev_used = 0;
+  return COFIE_OK;
+}
+
+int cofie_qer_profile_read(cofie_qer_t* h, uint64_t* launches, uint64_t* timed, double* score_ms, double* flops,
+                           double* key_bytes) {
+  if (!h || !launches || !timed || !score_ms || !flops || !key_bytes) return COFIE_EINVAL;
+  double ms = 0.0;
+  for (size_t i = 0; i + 1 < h->ev_used; i += 2) {
+    float t = 0.f;
+    cudaError_t e = cudaEventSynchronize(h->ev[i + 1]);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, h->ev[i], h->ev[i + 1]);
+    if (e != cudaSuccess) return h->fail(COFIE_ECUDA, cudaGetErrorString(e));
+    ms += t;
+  }
+  *launches = h->launches;
+  *timed = h->ev_used / 2;
+  *score_ms = ms;
+  *flops = h->flops;
+  *key_bytes = h->key_bytes;
   return COFIE_OK;
 }
 

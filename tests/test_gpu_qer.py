@@ -66,6 +66,8 @@ def check(spec, rho, frames=None):
                seed=4), 0.3),
     (S.QerSpec(n_text=256, n_heads=32, n_kv_heads=8, head_dim=128, n_frames=16, tokens_per_frame=256, n_evidence=4,
                seed=5), 0.25),
+    (S.QerSpec(n_text=20, n_heads=32, n_kv_heads=16, head_dim=68, n_frames=4, tokens_per_frame=33, n_evidence=1,
+               seed=9), 0.5),
 ])
 def test_qer_small_and_ragged(spec, rho):
     check(spec, rho)
