@@ -45,7 +45,7 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer"],
+    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards"],
                     default="hd1080",
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
@@ -641,6 +641,81 @@ def bench_qer(args):
         "n_evidence": int(len(ev))}), flush=True)
 
 
+def bench_shards(args):
+    """One 1080p stream split into 4 shards: each prepared from its frames and
+    an L_max-frame halo (independently; on several GPUs they would run in
+    parallel), chained through the gap maps, and committed. Reports the cost
+    against one whole-stream push, and the checkpoint size and latency."""
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.hd1080().with_(frames=min(3600, args.frames))
+    T = spec.frames
+    host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.cuda()
+    del host
+    S = 4
+    bounds = [T * i // S for i in range(S + 1)]
+    handles = [NGFF(spec.width, spec.height, max_frames_per_push=T) for _ in range(S)]
+    single = NGFF(spec.width, spec.height, max_frames_per_push=T)
+    keep_single = torch.empty(T, dtype=torch.uint8, device="cuda")
+
+    def run_single():
+        single.reset()
+        _, k = single.push(dev, keep=keep_single)
+
+    def run_sharded():
+        maps, prep_ev = [], []
+        for i in range(S):
+            a, b = bounds[i], bounds[i + 1]
+            halo = min(a, 30)
+            maps.append(handles[i].shard_prepare(dev[a - halo:b], n_halo=halo, t0=a))
+        g, keeps = 1, []
+        for i in range(S):
+            _, k = handles[i].shard_commit(g, bounds[i + 1] - bounds[i])
+            keeps.append(k)
+            g = int(maps[i][g - 1])
+        return torch.cat(keeps)
+
+    for _ in range(3):
+        run_single()
+        ks = run_sharded()
+    torch.cuda.synchronize()
+    assert torch.equal(ks, keep_single), "sharded decisions differ from the single pass"
+    reps = 10
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        run_single()
+    torch.cuda.synchronize()
+    t_single = (time.perf_counter() - t0) / reps
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        run_sharded()
+    torch.cuda.synchronize()
+    t_sharded = (time.perf_counter() - t0) / reps
+    # checkpoint / resume of one stream
+    state = single.state_save()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(100):
+        single.state_save(out=state)
+    t_save = (time.perf_counter() - t0) / 100
+    t0 = time.perf_counter()
+    for _ in range(100):
+        single.state_load(state)
+    t_load = (time.perf_counter() - t0) / 100
+    print(json.dumps({
+        "workload": f"shards: the {T}-frame 1080p stream in {S} shards, prepared and committed on one GPU",
+        "single_push_ms": t_single * 1e3, "sharded_ms": t_sharded * 1e3,
+        "sharded_over_single": t_sharded / t_single,
+        "halo_frames_extra": sum(min(bounds[i], 30) for i in range(S)),
+        "decisions_equal": True,
+        "state_bytes": int(state.numel()), "state_save_us": t_save * 1e6, "state_load_us": t_load * 1e6,
+        "timing": "host wall time with a device synchronise around each batch of repetitions"}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -655,6 +730,8 @@ def main():
         bench_gather(args)
     elif args.workload == "qer":
         bench_qer(args)
+    elif args.workload == "shards":
+        bench_shards(args)
     else:
         bench_gb300(args)
 

@@ -187,6 +187,53 @@ int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint
 int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames, const uint32_t* idx, uint32_t m,
                       uint8_t* out, void* cuda_stream);
 
+/*
+ * Checkpoint and resume of one stream. The saved state is everything a later
+ * push depends on (Sec. 3.2: r(t) enters only through the gap t - r(t), and
+ * distances reach back at most L_max frames): a 64-byte header (format tag
+ * "NGFS", version 1, width, height, bins, l_max, frames seen t, current gap
+ * g) followed by the ring of the last l_max histograms (l_max * bins uint32,
+ * slot i holds the frame t' with t' mod l_max == i).
+ *   cofie_ngff_state_bytes   the size of that buffer.
+ *   cofie_ngff_state_save    writes stream `stream`'s state to buf (device or
+ *                            host memory; host memory synchronises cuda_stream).
+ *   cofie_ngff_state_load    restores a saved state into stream `stream` of a
+ *                            handle with the same width, height, bins and l_max
+ *                            (COFIE_EINVAL otherwise); pushes that follow behave
+ *                            exactly as if the saved stream had continued.
+ */
+size_t cofie_ngff_state_bytes(const cofie_ngff_t* h);
+int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream);
+int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, void* cuda_stream);
+
+/*
+ * Sharding one stream across GPUs or machines. The decision of frame t
+ * depends on the past only through the gap g = t - r(t), which lies in
+ * [1, L_max], and through the histograms of the L_max frames before t
+ * (Sec. 3.2, Eqs. 3-5). So contiguous shards of one stream can be prepared
+ * independently, in any order or in parallel, and decided afterwards:
+ *   1. cofie_ngff_shard_prepare(h, stream, frames, n_halo, n, t0, map_out):
+ *      `frames` holds the halo (the n_halo = min(t0, L_max) frames just before
+ *      the shard) followed by the shard's n frames (device memory); t0 is the
+ *      stream index of the shard's first frame. Computes the shard's
+ *      histograms, distances and keep bits and writes its gap map: map_out[g-1]
+ *      (L_max uint16, device or host memory) is the gap after the shard's last
+ *      frame when the shard is entered with gap g. For t0 == 0 all entries are
+ *      equal (frame 0 is a first frame).
+ *   2. The caller chains the maps in stream order: the entry gap of the next
+ *      shard is map[entry - 1] of the previous one (any entry for t0 == 0).
+ *   3. cofie_ngff_shard_commit(h, stream, entry_gap, scores_out, keep_out):
+ *      emits the shard's scores and keep codes (n each, device or host memory)
+ *      and leaves the stream as after pushing frames [0, t0 + n).
+ * Steps 1 and 3 of one shard use the same handle and stream, with no other
+ * call on that handle between them; n_halo + n <= max_frames_per_push.
+ * Errors: COFIE_EINVAL, COFIE_ECUDA.
+ */
+int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n_halo, uint32_t n,
+                             uint64_t t0, uint16_t* map_out, void* cuda_stream);
+int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap, float* scores_out, uint8_t* keep_out,
+                            void* cuda_stream);
+
 /* Restarts stream `stream` at t = 0 (its next frame is a first frame). */
 int cofie_ngff_reset(cofie_ngff_t* h, uint32_t stream, void* cuda_stream);
 

@@ -155,6 +155,34 @@ class NGFF:
                                                 self._stream(cuda_stream)))
         return out
 
+    def state_save(self, stream: int = 0, out: torch.Tensor | None = None, cuda_stream=None) -> torch.Tensor:
+        """The stream's saved state (uint8; host memory unless ``out`` is given)."""
+        n = self._lib.cofie_ngff_state_bytes(self._h)
+        if out is None:
+            out = torch.empty(n, dtype=torch.uint8)
+        self._check(self._lib.cofie_ngff_state_save(self._h, stream, _ptr(out), self._stream(cuda_stream)))
+        return out
+
+    def state_load(self, state: torch.Tensor, stream: int = 0, cuda_stream=None):
+        self._check(self._lib.cofie_ngff_state_load(self._h, stream, _ptr(state), self._stream(cuda_stream)))
+
+    def shard_prepare(self, frames_with_halo: torch.Tensor, n_halo: int, t0: int, stream: int = 0, cuda_stream=None):
+        """Prepares one shard of a stream (halo frames then the shard's frames,
+        cuda uint8); returns its gap map as a host int tensor of l_max entries."""
+        n = self._frames(frames_with_halo) - n_halo
+        m = torch.zeros(self.l_max, dtype=torch.int16)
+        self._check(self._lib.cofie_ngff_shard_prepare(self._h, stream, _ptr(frames_with_halo), n_halo, n, t0,
+                                                       _ptr(m), self._stream(cuda_stream)))
+        return m.to(torch.int32)
+
+    def shard_commit(self, entry_gap: int, n: int, stream: int = 0, cuda_stream=None):
+        """Decides the prepared shard entered with ``entry_gap``; returns (scores, keep) on the device."""
+        scores = torch.empty(n, dtype=torch.float32, device=self.device)
+        keep = torch.empty(n, dtype=torch.uint8, device=self.device)
+        self._check(self._lib.cofie_ngff_shard_commit(self._h, stream, entry_gap, _ptr(scores), _ptr(keep),
+                                                      self._stream(cuda_stream)))
+        return scores, keep
+
     def reset(self, stream: int = 0, cuda_stream=None):
         self._check(self._lib.cofie_ngff_reset(self._h, stream, self._stream(cuda_stream)))
 

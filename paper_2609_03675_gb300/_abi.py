@@ -27,6 +27,11 @@ EXPORTS = (
     "cofie_ngff_candidates",
     "cofie_ngff_gather",
     "cofie_ngff_reset",
+    "cofie_ngff_state_bytes",
+    "cofie_ngff_state_save",
+    "cofie_ngff_state_load",
+    "cofie_ngff_shard_prepare",
+    "cofie_ngff_shard_commit",
     "cofie_ngff_status",
     "cofie_ngff_frames_seen",
     "cofie_ngff_debug_bins",
@@ -134,6 +139,16 @@ def load():
     lib.cofie_ngff_candidates.restype = ctypes.c_int
     lib.cofie_ngff_gather.argtypes = [H, vp, u32, vp, u32, vp, vp]
     lib.cofie_ngff_gather.restype = ctypes.c_int
+    lib.cofie_ngff_state_bytes.argtypes = [H]
+    lib.cofie_ngff_state_bytes.restype = ctypes.c_size_t
+    lib.cofie_ngff_state_save.argtypes = [H, u32, vp, vp]
+    lib.cofie_ngff_state_save.restype = ctypes.c_int
+    lib.cofie_ngff_state_load.argtypes = [H, u32, vp, vp]
+    lib.cofie_ngff_state_load.restype = ctypes.c_int
+    lib.cofie_ngff_shard_prepare.argtypes = [H, u32, vp, u32, u32, u64, vp, vp]
+    lib.cofie_ngff_shard_prepare.restype = ctypes.c_int
+    lib.cofie_ngff_shard_commit.argtypes = [H, u32, u32, vp, vp, vp]
+    lib.cofie_ngff_shard_commit.restype = ctypes.c_int
     lib.cofie_ngff_reset.argtypes = [H, u32, vp]
     lib.cofie_ngff_reset.restype = ctypes.c_int
     lib.cofie_ngff_status.argtypes = [H, vp]

@@ -8,6 +8,7 @@
 // overlapping the copy of piece i+1 with the kernels of piece i. Outputs in
 // host memory are written to device scratch and copied back on the caller's
 // stream.
+#include <cstddef>
 #include <cstdio>
 #include <cstring>
 #include <new>
@@ -66,6 +67,12 @@ struct cofie_ngff {
   uint32_t* d_err = nullptr;
   uint32_t* d_count = nullptr;  // candidate count when the caller's m_out is host memory
   uint64_t dirty_rows = 0;      // histogram rows [0, dirty_rows) may be nonzero
+  uint16_t* d_map = nullptr;    // a shard's gap map
+  struct {                      // the shard prepared and not yet committed
+    bool ready = false;
+    uint32_t stream = 0, n_halo = 0, n = 0;
+    uint64_t t0 = 0;
+  } shard;
   uint8_t* d_stage[2] = {nullptr, nullptr};
   uint64_t stage_bytes = 0;
   uint32_t stage_frames = 0;
@@ -338,7 +345,7 @@ void free_handle(cofie_ngff* h) {
   DeviceGuard guard(h->device);
   cudaDeviceSynchronize();
   void* bufs[] = {h->d_hist, h->d_l1, h->d_mask, h->d_ring, h->d_state, h->d_scores,
-                  h->d_keep, h->d_err,  h->d_stage[0], h->d_stage[1], h->d_count};
+                  h->d_keep, h->d_err,  h->d_stage[0], h->d_stage[1], h->d_count, h->d_map};
   for (void* b : bufs)
     if (b) cudaFree(b);
   for (cudaEvent_t ev : h->ev_pool) cudaEventDestroy(ev);
@@ -458,6 +465,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   if (e == cudaSuccess) e = dalloc(&h->d_keep, F);
   if (e == cudaSuccess) e = dalloc(&h->d_err, 1);
   if (e == cudaSuccess) e = dalloc(&h->d_count, 1);
+  if (e == cudaSuccess) e = dalloc(&h->d_map, COFIE_NGFF_MAX_LMAX);
   if (e != cudaSuccess) {
     cudaGetLastError();
     free_handle(h);
@@ -542,6 +550,215 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
   if (rc != COFIE_OK) return rc;
   for (uint32_t i = 0; i < nd; ++i) h->seen[desc[i].stream] += desc[i].n;
   h->err.clear();
+  return COFIE_OK;
+}
+
+namespace {
+
+constexpr uint32_t kStateMagic = 0x5346474Eu;  // "NGFS" little-endian
+constexpr uint32_t kStateVersion = 1;
+constexpr size_t kStateHeader = 64;
+
+struct StateHeader {  // the first 64 bytes of a saved state
+  uint32_t magic, version, width, height, bins, l_max;
+  uint32_t pad0, pad1;
+  StreamState st;  // frames seen, current gap (16 bytes)
+  uint32_t reserved[4];
+};
+static_assert(sizeof(StateHeader) == kStateHeader, "state header layout");
+
+}  // namespace
+
+size_t cofie_ngff_state_bytes(const cofie_ngff_t* h) {
+  return h ? kStateHeader + static_cast<size_t>(h->p.l_max) * h->p.bins * sizeof(uint32_t) : 0;
+}
+
+int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+  if (!buf) return h->fail(COFIE_EINVAL, "buf is NULL");
+  DeviceGuard guard(h->device);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const MemKind kb = classify(buf);
+  StateHeader hdr{};
+  hdr.magic = kStateMagic;
+  hdr.version = kStateVersion;
+  hdr.width = h->p.width;
+  hdr.height = h->p.height;
+  hdr.bins = h->p.bins;
+  hdr.l_max = h->p.l_max;
+  uint8_t* b = static_cast<uint8_t*>(buf);
+  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->p.bins * sizeof(uint32_t);
+  const uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->p.bins;
+  cudaError_t e;
+  if (kb == kDevice) {
+    // the header's fixed part travels through the handle's pinned-free path: a
+    // synchronous copy of 32 host bytes, then the device-resident parts
+    e = cudaMemcpyAsync(b, &hdr, offsetof(StateHeader, st), cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  } else {
+    memcpy(b, &hdr, kStateHeader);
+    e = cudaSuccess;
+  }
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(b + offsetof(StateHeader, st), h->d_state + stream, sizeof(StreamState), cudaMemcpyDefault, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(b + kStateHeader, ring, ring_bytes, cudaMemcpyDefault, st);
+  if (e == cudaSuccess && kb != kDevice) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "state save");
+  return COFIE_OK;
+}
+
+int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+  if (!buf) return h->fail(COFIE_EINVAL, "buf is NULL");
+  DeviceGuard guard(h->device);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  StateHeader hdr{};
+  cudaError_t e = cudaMemcpyAsync(&hdr, buf, kStateHeader, cudaMemcpyDefault, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "state load");
+  if (hdr.magic != kStateMagic || hdr.version != kStateVersion)
+    return h->fail(COFIE_EINVAL, "not a saved stream state (format tag or version)");
+  if (hdr.width != h->p.width || hdr.height != h->p.height || hdr.bins != h->p.bins || hdr.l_max != h->p.l_max)
+    return h->fail(COFIE_EINVAL, "saved state has another width, height, bins or l_max");
+  if (hdr.st.t > 0 && (hdr.st.g < 1 || hdr.st.g > h->p.l_max))
+    return h->fail(COFIE_EINVAL, "saved state has a gap outside [1, l_max]");
+  const uint8_t* b = static_cast<const uint8_t*>(buf);
+  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->p.bins * sizeof(uint32_t);
+  uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->p.bins;
+  e = cudaMemcpyAsync(ring, b + kStateHeader, ring_bytes, cudaMemcpyDefault, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->d_state + stream, b + offsetof(StateHeader, st), sizeof(StreamState), cudaMemcpyDefault, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // buf may be released when this returns
+  if (e != cudaSuccess) return h->cuda_fail(e, "state load");
+  h->seen[stream] = hdr.st.t;
+  return COFIE_OK;
+}
+
+int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n_halo, uint32_t n,
+                             uint64_t t0, uint16_t* map_out, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+  if (!frames || !map_out || n == 0) return h->fail(COFIE_EINVAL, "frames and map_out are required, n >= 1");
+  const uint64_t want_halo = t0 < h->p.l_max ? t0 : h->p.l_max;
+  if (n_halo != want_halo) return h->fail(COFIE_EINVAL, "n_halo must be min(t0, l_max)");
+  if (static_cast<uint64_t>(n_halo) + n > h->p.max_frames_per_push)
+    return h->fail(COFIE_EINVAL, "n_halo + n exceeds max_frames_per_push");
+  int fdev = -1;
+  if (classify(frames, &fdev) != kDevice || fdev != h->device)
+    return h->fail(COFIE_EINVAL, "shard frames must be device memory on the handle's device");
+  DeviceGuard guard(h->device);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  h->shard.ready = false;
+  // K1 over halo + shard frames; the stream's clock starts at t0 for K2
+  SegTable all;
+  memset(&all, 0, sizeof all);
+  all.count = 1;
+  all.rows = n_halo + n;
+  all.s[0].frames = frames;
+  all.s[0].n = n_halo + n;
+  all.s[0].stream = stream;
+  StreamState ss{t0, 1u, 0u};
+  cudaError_t e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "shard state");
+  // the histograms (K1 only): run_segments' selection must not run here, so
+  // the launch sequence is spelled out
+  if (h->dirty_rows) {
+    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->p.bins * 4, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+  }
+  h->dirty_rows = h->p.max_frames_per_push;
+  bool fast = h->size_fast && h->bin_path >= 0 && reinterpret_cast<uintptr_t>(frames) % 16 == 0;
+  HistArgs ha{};
+  ha.frame_bytes = h->frame_bytes;
+  ha.npix = h->npix;
+  ha.groups_per_frame = static_cast<uint32_t>(h->frame_bytes / 48);
+  ha.chunks_per_frame = (ha.groups_per_frame + hist_chunk_groups() - 1) / hist_chunk_groups();
+  ha.timeout_ns = kTimeoutNs;
+  if (fast) {
+    const uint64_t chunks = static_cast<uint64_t>(all.rows) * ha.chunks_per_frame;
+    e = launch_hist_fast(all, ha, h->lc, h->bin_path, h->d_hist, h->d_err,
+                         static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid), st);
+  } else {
+    e = launch_hist_generic(all, ha, h->lc, h->d_hist, st);
+  }
+  if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
+  h->n_hist += 1;
+  h->hist_bytes += static_cast<uint64_t>(all.rows) * (h->frame_bytes + 4ull * h->p.bins);
+  // K2 over the shard's rows, reading the halo rows before them
+  SegTable sh;
+  memset(&sh, 0, sizeof sh);
+  sh.count = 1;
+  sh.rows = n_halo + n;
+  sh.s[0].frames = frames + static_cast<uint64_t>(n_halo) * h->frame_bytes;
+  sh.s[0].n = n;
+  sh.s[0].row0 = n_halo;
+  sh.s[0].stream = stream;
+  sh.s[0].halo = n_halo;
+  SelectArgs sa{};
+  sa.bins = h->p.bins;
+  sa.l_max = h->p.l_max;
+  sa.mask_words = h->mask_words;
+  sa.tau = h->p.tau;
+  sa.two_n = h->two_n;
+  e = launch_window(sh, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
+  if (e == cudaSuccess) e = launch_gap_map(sh.s[0], sa, t0, h->d_mask, h->d_map, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(map_out, h->d_map, h->p.l_max * sizeof(uint16_t), cudaMemcpyDefault, st);
+  if (e == cudaSuccess && classify(map_out) != kDevice) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "shard preparation");
+  h->n_select += 2;
+  h->dirty_rows = n_halo + n;
+  h->shard.ready = true;
+  h->shard.stream = stream;
+  h->shard.n_halo = n_halo;
+  h->shard.n = n;
+  h->shard.t0 = t0;
+  return COFIE_OK;
+}
+
+int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap, float* scores_out, uint8_t* keep_out,
+                            void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (!h->shard.ready || h->shard.stream != stream)
+    return h->fail(COFIE_EINVAL, "no shard of this stream is prepared on this handle");
+  if (h->shard.t0 > 0 && (entry_gap < 1 || entry_gap > h->p.l_max))
+    return h->fail(COFIE_EINVAL, "entry_gap must be in [1, l_max]");
+  DeviceGuard guard(h->device);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const uint32_t n_halo = h->shard.n_halo, n = h->shard.n;
+  SelectArgs sa{};
+  sa.bins = h->p.bins;
+  sa.l_max = h->p.l_max;
+  sa.mask_words = h->mask_words;
+  sa.tau = h->p.tau;
+  sa.two_n = h->two_n;
+  // the stream's ring holds the halo frames (the last frames before t0) ...
+  cudaError_t e = launch_ring_store(h->d_hist, n_halo, h->shard.t0 - n_halo, stream, sa, h->d_ring, st);
+  // ... and its gap is the resolved entry gap
+  StreamState ss{h->shard.t0, h->shard.t0 > 0 ? entry_gap : 1u, 0u};
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "shard commit");
+  const MemKind ks = classify(scores_out), kk = classify(keep_out);
+  SegTable sh;
+  memset(&sh, 0, sizeof sh);
+  sh.count = 1;
+  sh.rows = n_halo + n;
+  sh.s[0].n = n;
+  sh.s[0].row0 = n_halo;
+  sh.s[0].stream = stream;
+  sh.s[0].halo = n_halo;
+  sh.s[0].scores = ks == kDevice ? scores_out : (ks == kNull ? nullptr : h->d_scores);
+  sh.s[0].keep = kk == kDevice ? keep_out : (kk == kNull ? nullptr : h->d_keep);
+  e = launch_scan(sh, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st);
+  if (e == cudaSuccess && (ks == kHostPinned || ks == kHostPageable))
+    e = cudaMemcpyAsync(scores_out, h->d_scores, n * sizeof(float), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess && (kk == kHostPinned || kk == kHostPageable))
+    e = cudaMemcpyAsync(keep_out, h->d_keep, n, cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "shard commit");
+  h->n_select += 1;
+  h->shard.ready = false;
+  h->seen[stream] = h->shard.t0 + n;
   return COFIE_OK;
 }
 

@@ -28,7 +28,7 @@ struct Segment {
   uint32_t n;
   uint32_t row0;
   uint32_t stream;
-  uint32_t pad;
+  uint32_t halo;          // histogram rows before row0 that hold the frames just before it
 };
 
 struct SegTable {
@@ -101,6 +101,10 @@ cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint3
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);
+cudaError_t launch_gap_map(const Segment& seg, const SelectArgs& a, unsigned long long t0, const uint32_t* mask,
+                           uint16_t* map_out, cudaStream_t st);
+cudaError_t launch_ring_store(const uint32_t* hist, uint32_t rows, unsigned long long t_first, uint32_t stream,
+                              const SelectArgs& a, uint32_t* ring, cudaStream_t st);
 cudaError_t launch_candidates(const uint8_t* keep, uint32_t T, uint32_t m_min, uint32_t* idx, uint32_t* m_out,
                               cudaStream_t st);
 cudaError_t launch_gather(const uint8_t* frames, uint32_t n_frames, uint64_t frame_bytes, const uint32_t* idx, uint32_t m,

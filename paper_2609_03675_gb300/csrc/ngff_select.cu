@@ -59,8 +59,8 @@ __device__ __forceinline__ void window_row(uint32_t row, uint32_t lane, const Se
     const bool valid = k <= L && k <= t;
     const uint32_t* src = ct;
     if (valid)
-      src = (k <= j) ? hist + static_cast<uint64_t>(row - k) * B
-                     : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
+      src = (k <= j + sg.halo) ? hist + static_cast<uint64_t>(row - k) * B
+                               : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
     uint32_t d = 0;
     if (kVec4) {
       const uint4* c4 = reinterpret_cast<const uint4*>(ct);
@@ -99,6 +99,7 @@ __global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, S
   uint32_t seg = 0;
   while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
   const Segment sg = segs.s[seg];
+  if (row < sg.row0) return;  // halo rows: history only, no decision
   window_row<kVec4>(row, lane, sg, a, hist, ring, state[sg.stream].t, l1, mask);
 }
 
@@ -245,6 +246,62 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
   scan_segment<kOneWord>(sseg, s_t0, s_g, a, l1, mask, hist, ring, state, ssm, entry);
 }
 
+// The gap map of one stream segment: map[g-1] = the gap after its last frame
+// when its first frame is entered with gap g (for a stream's first segment,
+// frame 0 is a first frame and every entry gives the same result). One CTA:
+// each warp composes the maps of a run of frames for all entry gaps (lane =
+// entry gap), then lanes chain the 32 run maps; tiles of kScanTile frames are
+// chained the same way.
+template <bool kOneWord>
+__global__ void __launch_bounds__(kScanThreads) gap_map_kernel(Segment sg, SelectArgs a, unsigned long long t0,
+                                                               const uint32_t* __restrict__ mask,
+                                                               uint16_t* __restrict__ map_out) {
+  extern __shared__ __align__(16) uint32_t ssm[];
+  __shared__ uint16_t smap[kMaxLmax];
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t W = a.mask_words, L = a.l_max;
+  uint32_t* smask = ssm;
+  uint16_t* sexit = reinterpret_cast<uint16_t*>(smask + kScanTile * W) + kScanTile;  // [kScanWarps][L]
+  for (uint32_t g = tid; g < L; g += kScanThreads) smap[g] = static_cast<uint16_t>(g + 1);  // identity
+  const uint32_t j_start = (t0 == 0) ? 1u : 0u;  // frame 0 of a stream is a first frame: gap 1 after it
+  if (t0 == 0 && sg.n > 0)
+    for (uint32_t g = tid; g < L; g += kScanThreads) smap[g] = 1;
+  __syncthreads();
+  for (uint32_t tile0 = j_start; tile0 < sg.n; tile0 += kScanTile) {
+    const uint32_t m = min(kScanTile, sg.n - tile0);
+    for (uint32_t i = tid; i < m * W; i += kScanThreads)
+      smask[i] = mask[static_cast<uint64_t>(sg.row0 + tile0) * W + i];
+    __syncthreads();
+    const uint32_t run = (m + kScanWarps - 1) / kScanWarps;
+    const uint32_t f0 = min(warp * run, m), f1 = min(f0 + run, m);
+    for (uint32_t gin = lane + 1; gin <= L; gin += 32) {
+      uint32_t g = gin;
+      for (uint32_t f = f0; f < f1; ++f) g = step_gap<kOneWord>(smask + f * W, g);
+      sexit[warp * L + gin - 1] = static_cast<uint16_t>(g);
+    }
+    __syncthreads();
+    // compose: the map so far, then the 32 runs of this tile in order
+    for (uint32_t e = tid; e < L; e += kScanThreads) {
+      uint32_t g = smap[e];
+      for (uint32_t w = 0; w < kScanWarps; ++w)
+        if (min(w * run, m) < min(w * run + run, m)) g = sexit[w * L + g - 1];
+      smap[e] = static_cast<uint16_t>(g);
+    }
+    __syncthreads();
+  }
+  for (uint32_t g = tid; g < L; g += kScanThreads) map_out[g] = smap[g];
+}
+
+// ring[(t_first + i) mod L] = hist row i, for rows [0, rows) of a stream.
+__global__ void ring_store_kernel(const uint32_t* __restrict__ hist, uint32_t rows, unsigned long long t_first,
+                                  uint32_t stream, SelectArgs a, uint32_t* __restrict__ ring) {
+  const uint32_t B = a.bins, L = a.l_max;
+  for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < rows * B; i += gridDim.x * blockDim.x) {
+    const uint32_t r = i / B, b = i % B;
+    ring[(static_cast<uint64_t>(stream) * L + (t_first + r) % L) * B + b] = hist[static_cast<uint64_t>(r) * B + b];
+  }
+}
+
 size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
   return static_cast<size_t>(kScanTile) * mask_words * 4 + kScanTile * 2 + static_cast<size_t>(kScanWarps) * l_max * 2;
 }
@@ -252,6 +309,27 @@ size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
 }  // namespace
 
 uint32_t select_small_max() { return kSmallMax; }
+
+cudaError_t launch_gap_map(const Segment& seg, const SelectArgs& a, unsigned long long t0, const uint32_t* mask,
+                           uint16_t* map_out, cudaStream_t st) {
+  const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
+  cudaError_t e;
+  if (a.mask_words == 1) {
+    e = cudaFuncSetAttribute(gap_map_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e == cudaSuccess) gap_map_kernel<true><<<1, kScanThreads, smem, st>>>(seg, a, t0, mask, map_out);
+  } else {
+    e = cudaFuncSetAttribute(gap_map_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e == cudaSuccess) gap_map_kernel<false><<<1, kScanThreads, smem, st>>>(seg, a, t0, mask, map_out);
+  }
+  return e == cudaSuccess ? cudaGetLastError() : e;
+}
+
+cudaError_t launch_ring_store(const uint32_t* hist, uint32_t rows, unsigned long long t_first, uint32_t stream,
+                              const SelectArgs& a, uint32_t* ring, cudaStream_t st) {
+  if (rows == 0) return cudaSuccess;
+  ring_store_kernel<<<(rows * a.bins + 255) / 256, 256, 0, st>>>(hist, rows, t_first, stream, a, ring);
+  return cudaGetLastError();
+}
 
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max) {
   const int smem = static_cast<int>(scan_smem_bytes(mask_words, l_max));
