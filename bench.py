@@ -45,7 +45,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards"],
+    ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards",
+                                           "signals"],
                     default="hd1080",
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
@@ -716,6 +717,90 @@ def bench_shards(args):
         "timing": "host wall time with a device synchronise around each batch of repetitions"}), flush=True)
 
 
+def bench_signals(args):
+    """The three NGFF signals on the 1080p stream (frames/s, first-stage
+    bandwidth against the measured copy peak) and on the 720p rare-event
+    stream (keep ratio and event recall across thresholds): the synthetic
+    counterpart of the paper's signal ablation."""
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    names = {0: "histogram", 1: "lowres", 2: "dhash"}
+    taus = {0: (0.30, 0.10, 0.05), 1: (0.05, 0.02, 0.01), 2: (0.20, 0.10, 0.05)}
+    peak, peak_kind = peaks()
+    spec = synth.hd1080()
+    T = min(spec.frames, 600)
+    spec = spec.with_(frames=T)
+    host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.cuda()
+    scores = torch.empty(T, dtype=torch.float32, device="cuda")
+    keep = torch.empty(T, dtype=torch.uint8, device="cuda")
+    out = {"workload": f"signals: 1080p stream of {T} frames (throughput), 720p rare-event stream of 3600 frames "
+                       "with 40 events (recall)", "peak_gbs": peak, "peak_kind": f"{peak_kind} copy bandwidth",
+           "signals": {}}
+    for sig, name in names.items():
+        f = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=sig)
+
+        def step():
+            f.reset()
+            f.push(dev, scores=scores, keep=keep)
+
+        for _ in range(max(3, args.warmup)):
+            step()
+        torch.cuda.synchronize()
+        f.profile_reset(time_kernels=True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(20):
+            step()
+        e1.record()
+        torch.cuda.synchronize()
+        f.status()
+        prof = f.profile_read()
+        ms = e0.elapsed_time(e1) / 20
+        k_ms = prof["hist_ms"] / max(prof["hist_timed"], 1)
+        k_bytes = prof["hist_bytes"] / max(prof["hist_launches"], 1)
+        out["signals"][name] = {"frames_per_s": T / (ms / 1e3), "ms_per_step": ms, "first_stage_ms": k_ms,
+                                "first_stage_gbs": k_bytes / (k_ms / 1e3) / 1e9,
+                                "first_stage_frac": k_bytes / (k_ms / 1e3) / 1e9 / peak,
+                                "select_ms": prof["select_ms"] / max(prof["select_timed"], 1),
+                                "keep_ratio_default_tau": float((keep != 0).float().mean().item())}
+        f.close()
+    del dev, host
+    rs = synth.rare_event()
+    rhost = torch.empty((rs.frames, rs.height, rs.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(rs, out=rhost.data_ptr())
+    rdev = rhost.cuda()
+    ev = synth.event_mask(rs).astype(bool)
+    runs, t = [], 0
+    while t < rs.frames:
+        if ev[t]:
+            u = t
+            while u < rs.frames and ev[u]:
+                u += 1
+            runs.append((t, u))
+            t = u
+        else:
+            t += 1
+    rk = torch.empty(rs.frames, dtype=torch.uint8, device="cuda")
+    rsc = torch.empty(rs.frames, dtype=torch.float32, device="cuda")
+    for sig, name in names.items():
+        rec = {}
+        for tau in taus[sig]:
+            f = NGFF(rs.width, rs.height, tau=tau, signal=sig)
+            f.push(rdev, scores=rsc, keep=rk)
+            torch.cuda.synchronize()
+            f.status()
+            kc = rk.cpu().numpy() != 0
+            rec[str(tau)] = {"keep_ratio": float(kc.mean()), "event_frame_recall": float(kc[ev].mean()),
+                             "event_recall": sum(1 for a, b in runs if kc[a:b].any()) / max(1, len(runs))}
+            f.close()
+        out["signals"][name]["rare_event"] = rec
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -732,6 +817,8 @@ def main():
         bench_qer(args)
     elif args.workload == "shards":
         bench_shards(args)
+    elif args.workload == "signals":
+        bench_signals(args)
     else:
         bench_gb300(args)
 

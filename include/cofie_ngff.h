@@ -47,7 +47,7 @@
 extern "C" {
 #endif
 
-#define COFIE_NGFF_ABI_VERSION 1
+#define COFIE_NGFF_ABI_VERSION 2
 
 /* Return codes. */
 #define COFIE_OK 0
@@ -62,6 +62,11 @@ extern "C" {
 #define COFIE_KEEP_NOVELTY 1 /* s >= tau_h (Eq. 5, first term) */
 #define COFIE_KEEP_GAP 2     /* t - r(t) >= L_max and not novelty (Eq. 5, second term) */
 #define COFIE_KEEP_FIRST 3   /* the stream's first frame (Sec. 3.2 safeguard) */
+
+/* Novelty signals (the distance d inside Eqs. 3-5). */
+#define COFIE_SIGNAL_HISTOGRAM 0 /* TV distance of B-bin grayscale histograms (Sec. 3.2, the paper's signal) */
+#define COFIE_SIGNAL_LOWRES 1    /* mean |difference| of 16 x 16-cell block-averaged grayscale frames */
+#define COFIE_SIGNAL_DHASH 2     /* Hamming distance / 64 of 9 x 8-cell difference hashes */
 
 /* Limits. */
 #define COFIE_NGFF_MAX_BINS 256
@@ -86,6 +91,17 @@ typedef struct cofie_ngff cofie_ngff_t;
  *   device            CUDA device ordinal, or -1 for the calling thread's current device.
  *   host_stage_bytes  size of each of the two device staging buffers used when
  *                     frames come from host memory; 0 picks 256 MiB (at least one frame).
+ *   signal            COFIE_SIGNAL_*: the distance in the retention rule. The
+ *                     alternatives are the lightweight signals of the paper's
+ *                     signal ablation (Table "hdiff-signal"), defined here as:
+ *                     low-res: cells (floor(y 16 / H), floor(x 16 / W)), S_c the
+ *                       cell's grayscale sum, d = sum_c |S_c - S'_c| / (255 W H)
+ *                       (W, H >= 16, W H <= 16,777,216);
+ *                     dHash: 8 rows x 9 columns of cells, bit (r, c) = cell mean
+ *                       (r, c) > cell mean (r, c+1), d = Hamming distance / 64
+ *                       (W >= 9, H >= 8).
+ *                     hist_out of cofie_ngff_push_ex then receives the signal's
+ *                     feature rows (cofie_ngff_feature_words uint32 per frame).
  */
 typedef struct {
   uint32_t width, height;
@@ -99,6 +115,8 @@ typedef struct {
   uint32_t max_frames_per_push;
   int32_t device;
   uint64_t host_stage_bytes;
+  uint32_t signal;
+  uint32_t reserved;
 } cofie_ngff_params;
 
 /* One stream's frames in a batched push (see cofie_ngff_push_batch). */
@@ -109,6 +127,9 @@ typedef struct {
   float* scores_out;      /* n floats, device memory, or NULL */
   uint8_t* keep_out;      /* n keep codes, device memory, or NULL */
 } cofie_ngff_push_desc;
+
+/* uint32 words per frame of the handle's signal features (bins for the histogram). */
+uint32_t cofie_ngff_feature_words(const cofie_ngff_t* h);
 
 /* Fills *p with the paper's defaults for a width x height stream. */
 void cofie_ngff_default_params(cofie_ngff_params* p, uint32_t width, uint32_t height);

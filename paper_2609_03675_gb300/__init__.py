@@ -39,7 +39,8 @@ class NGFF:
 
     def __init__(self, width: int, height: int, *, bins: int = 32, l_max: int = 30, m_min: int = 4,
                  tau: float = 0.30, luma_weights=(299, 587, 114), luma_den: int = 1000, max_streams: int = 1,
-                 max_frames_per_push: int = 4096, device: int | None = None, host_stage_bytes: int = 0):
+                 max_frames_per_push: int = 4096, device: int | None = None, host_stage_bytes: int = 0,
+                 signal: int = 0):
         lib = _abi.load()
         p = _abi.Params()
         lib.cofie_ngff_default_params(ctypes.byref(p), width, height)
@@ -51,6 +52,7 @@ class NGFF:
             device = torch.cuda.current_device()
         p.device = device
         p.host_stage_bytes = host_stage_bytes
+        p.signal = signal
         h = ctypes.c_void_p()
         rc = lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h))
         if rc != _abi.OK:
@@ -59,6 +61,8 @@ class NGFF:
         self.width, self.height, self.bins, self.l_max, self.m_min, self.tau = width, height, bins, l_max, m_min, tau
         self.device = torch.device("cuda", device)
         self.frame_bytes = 3 * width * height
+        self.signal = signal
+        self.feature_words = int(lib.cofie_ngff_feature_words(h))
 
     # ----------------------------------------------------------------- util --
     def _check(self, rc: int):
@@ -80,7 +84,7 @@ class NGFF:
         if keep is None:
             keep = torch.empty(n, dtype=torch.uint8, **kw)
         if want_hist and hist is None:
-            hist = torch.empty((n, self.bins), dtype=torch.int32, **kw)
+            hist = torch.empty((n, self.feature_words), dtype=torch.int32, **kw)
         return scores, keep, hist
 
     def _frames(self, frames):

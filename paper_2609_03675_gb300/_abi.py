@@ -15,10 +15,12 @@ LIB_PATH = os.path.join(HERE, "libcofie_ngff.so")
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE = 0, 1, 2, 3, 4, 5
 KEEP_DROP, KEEP_NOVELTY, KEEP_GAP, KEEP_FIRST = 0, 1, 2, 3
 MAX_BINS, MAX_LMAX, MAX_BATCH = 256, 256, 64
+SIGNAL_HISTOGRAM, SIGNAL_LOWRES, SIGNAL_DHASH = 0, 1, 2
 
 # Every symbol include/cofie_ngff.h declares.
 EXPORTS = (
     "cofie_ngff_default_params",
+    "cofie_ngff_feature_words",
     "cofie_ngff_create",
     "cofie_ngff_destroy",
     "cofie_ngff_push",
@@ -64,6 +66,8 @@ class Params(ctypes.Structure):
         ("max_frames_per_push", ctypes.c_uint32),
         ("device", ctypes.c_int32),
         ("host_stage_bytes", ctypes.c_uint64),
+        ("signal", ctypes.c_uint32),
+        ("reserved", ctypes.c_uint32),
     ]
 
 
@@ -125,6 +129,8 @@ def load():
     H = ctypes.c_void_p
     lib.cofie_ngff_default_params.argtypes = [P, u32, u32]
     lib.cofie_ngff_default_params.restype = None
+    lib.cofie_ngff_feature_words.argtypes = [H]
+    lib.cofie_ngff_feature_words.restype = u32
     lib.cofie_ngff_create.argtypes = [P, ctypes.POINTER(H)]
     lib.cofie_ngff_create.restype = ctypes.c_int
     lib.cofie_ngff_destroy.argtypes = [H]

@@ -8,6 +8,7 @@
 // overlapping the copy of piece i+1 with the kernels of piece i. Outputs in
 // host memory are written to device scratch and copied back on the caller's
 // stream.
+#include <algorithm>
 #include <cstddef>
 #include <cstdio>
 #include <cstring>
@@ -52,10 +53,15 @@ struct cofie_ngff {
   uint64_t frame_bytes = 0;
   uint32_t npix = 0;
   uint32_t mask_words = 0;
+  uint32_t fw = 0;       // uint32 feature words per frame: bins, 256 (low-res) or 2 (dHash)
+  FeatArgs fa{};         // the spatial signals' grid
   LumaConsts lc{};
   int bin_path = -1;  // kBinFast, kBinTwoStep, or -1 (generic kernel only)
   bool size_fast = false;
   int hist_grid = 0;
+  int cells_grid = 0;    // the TMA kernel's grid for the spatial signals (0: not usable)
+  uint32_t m_gpr = 0, m_h = 0, m_gw = 0;  // its multiply-high divisors (16-pixel groups per row, height, grid columns)
+  uint32_t* d_cells = nullptr;  // dHash only: [F][72] cell sums, kept zero between pushes
   float two_n = 0.f;
   uint32_t* d_hist = nullptr;
   uint32_t* d_l1 = nullptr;
@@ -121,6 +127,18 @@ MemKind classify(const void* ptr, int* dev_out = nullptr) {
   }
 }
 
+// m = ceil(2^32 / d) with e = m d - 2^32 gives umulhi(n, m) = floor(n / d)
+// for every n with n e < 2^32: n m / 2^32 = n / d + n e / (d 2^32), and the
+// fraction of n / d is at most (d - 1) / d. Returns 0 when d < 2 or n_max is
+// out of that range.
+uint32_t magic_for(uint32_t d, uint64_t n_max) {
+  if (d < 2) return 0;
+  const uint64_t m = ((1ull << 32) + d - 1) / d;
+  const uint64_t e = m * d - (1ull << 32);
+  if (m > 0xffffffffull || (e && n_max >= (1ull << 32) / e)) return 0;
+  return static_cast<uint32_t>(m);
+}
+
 bool verify_magic(uint32_t magic, uint32_t vmax, uint32_t den, uint32_t bins, bool divide_only) {
   for (uint32_t v = 0; v <= vmax; ++v) {
     const uint32_t y = v / den;
@@ -144,6 +162,14 @@ int validate_params(const cofie_ngff_params* p, std::string& why) {
     return why = "luma weights must sum to luma_den", COFIE_EINVAL;
   if (p->max_streams < 1) return why = "max_streams must be >= 1", COFIE_EINVAL;
   if (p->max_frames_per_push < 1) return why = "max_frames_per_push must be >= 1", COFIE_EINVAL;
+  if (p->signal > COFIE_SIGNAL_DHASH) return why = "signal must be one of COFIE_SIGNAL_*", COFIE_EINVAL;
+  if (p->signal == COFIE_SIGNAL_LOWRES && (p->width < 16 || p->height < 16 || npix > (1ull << 24)))
+    return why = "the low-res signal needs width, height >= 16 and width * height <= 2^24", COFIE_EINVAL;
+  if (p->signal == COFIE_SIGNAL_DHASH && (p->width < 9 || p->height < 8))
+    return why = "the dHash signal needs width >= 9 and height >= 8", COFIE_EINVAL;
+  if (p->signal == COFIE_SIGNAL_DHASH &&
+      255ull * ((p->height + 7) / 8) * ((p->width + 8) / 9) > 0xffffffffull)  // a cell's grayscale sum in 32 bits
+    return why = "the dHash signal's cells are too large for 32-bit sums", COFIE_EINVAL;
   return COFIE_OK;
 }
 
@@ -182,20 +208,11 @@ double sum_pairs(const std::vector<cudaEvent_t>& pool, size_t used, cudaError_t*
   return ms;
 }
 
-// Runs K1-K3 over the rows described by segs (device frames). Histogram rows
-// must be zero when K1 starts: the fused small-push kernel clears its rows
-// after use (unless keep_hist: the caller copies them out afterwards);
-// otherwise the rows are marked dirty and the next push clears them first.
-int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep_hist = false) {
-  if (segs.rows == 0) return COFIE_OK;
-  cudaError_t e = cudaSuccess;
-  if (h->dirty_rows) {
-    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->p.bins * 4, st);
-    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
-    h->dirty_rows = 0;
-  }
-  h->dirty_rows = h->p.max_frames_per_push;  // until the whole sequence is enqueued
-  bool fast = h->size_fast && h->bin_path >= 0;
+// The first stage over the rows of segs: grayscale histograms (K1), or the
+// spatial signal's per-frame features.
+cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
+  const bool cells = h->p.signal != COFIE_SIGNAL_HISTOGRAM;
+  bool fast = cells ? h->cells_grid > 0 : h->size_fast && h->bin_path >= 0;
   for (uint32_t i = 0; i < segs.count && fast; ++i)
     if (reinterpret_cast<uintptr_t>(segs.s[i].frames) % 16 != 0) fast = false;
   HistArgs ha{};
@@ -204,25 +221,64 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
   ha.groups_per_frame = static_cast<uint32_t>(h->frame_bytes / 48);
   ha.chunks_per_frame = (ha.groups_per_frame + hist_chunk_groups() - 1) / hist_chunk_groups();
   ha.timeout_ns = kTimeoutNs;
-  cudaEvent_t ev0 = nullptr, ev1 = nullptr;
-  if (h->time_kernels && take_pair(h->ev_pool, h->ev_used, &ev0, &ev1)) cudaEventRecord(ev0, st);
+  if (cells) {
+    if (!fast) return launch_features(segs, h->fa, h->lc, h->d_hist, h->fw, st);
+    ha.width = h->p.width;
+    ha.height = h->p.height;
+    ha.grid_h = h->fa.grid_h;
+    ha.grid_w = h->fa.grid_w;
+    ha.gpr = h->p.width / 16;
+    ha.m_gpr = h->m_gpr;
+    ha.m_h = h->m_h;
+    ha.m_gw = h->m_gw;
+    ha.wide = (h->p.width / h->fa.grid_w >= 16 && h->m_gw) ? 1u : 0u;
+    const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
+    const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->cells_grid) ? chunks : h->cells_grid);
+    const bool dhash = h->p.signal == COFIE_SIGNAL_DHASH;
+    cudaError_t e = launch_cells_fast(segs, ha, h->lc, dhash ? h->d_cells : h->d_hist, h->d_err, grid, st);
+    if (e == cudaSuccess && dhash) e = launch_dhash_finish(h->d_cells, segs.rows, h->fa, h->d_hist, st);
+    return e;
+  }
   if (fast) {
     const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
     const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid);
-    e = launch_hist_fast(segs, ha, h->lc, h->bin_path, h->d_hist, h->d_err, grid, st);
-  } else {
-    e = launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
+    return launch_hist_fast(segs, ha, h->lc, h->bin_path, h->d_hist, h->d_err, grid, st);
   }
-  if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
-  if (ev1) cudaEventRecord(ev1, st);
-  h->n_hist += 1;
-  h->hist_bytes += static_cast<uint64_t>(segs.rows) * (h->frame_bytes + 4ull * h->p.bins);
+  return launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
+}
+
+SelectArgs select_args(const cofie_ngff* h) {
   SelectArgs sa{};
-  sa.bins = h->p.bins;
+  sa.bins = h->fw;
   sa.l_max = h->p.l_max;
   sa.mask_words = h->mask_words;
   sa.tau = h->p.tau;
   sa.two_n = h->two_n;
+  sa.dist_kind = h->p.signal == COFIE_SIGNAL_DHASH ? 1u : 0u;
+  return sa;
+}
+
+// Runs K1-K3 over the rows described by segs (device frames). Histogram rows
+// must be zero when K1 starts: the fused small-push kernel clears its rows
+// after use (unless keep_hist: the caller copies them out afterwards);
+// otherwise the rows are marked dirty and the next push clears them first.
+int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep_hist = false) {
+  if (segs.rows == 0) return COFIE_OK;
+  cudaError_t e = cudaSuccess;
+  if (h->dirty_rows && h->p.signal != COFIE_SIGNAL_DHASH) {  // dHash rows are written whole
+    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->fw * 4, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+    h->dirty_rows = 0;
+  }
+  h->dirty_rows = h->p.max_frames_per_push;  // until the whole sequence is enqueued
+  cudaEvent_t ev0 = nullptr, ev1 = nullptr;
+  if (h->time_kernels && take_pair(h->ev_pool, h->ev_used, &ev0, &ev1)) cudaEventRecord(ev0, st);
+  e = launch_first_stage(h, segs, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
+  if (ev1) cudaEventRecord(ev1, st);
+  h->n_hist += 1;
+  h->hist_bytes += static_cast<uint64_t>(segs.rows) * (h->frame_bytes + 4ull * h->fw);
+  SelectArgs sa = select_args(h);
   uint32_t longest = 0;
   for (uint32_t i = 0; i < segs.count; ++i) longest = segs.s[i].n > longest ? segs.s[i].n : longest;
   // small pushes clear their rows inside the fused kernel (saving a launch);
@@ -269,7 +325,7 @@ int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n
   if (e == cudaSuccess && (kk == kHostPinned || kk == kHostPageable))
     e = cudaMemcpyAsync(keep, h->d_keep, n, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess && kh != kNull)
-    e = cudaMemcpyAsync(hist_out, h->d_hist, static_cast<size_t>(n) * h->p.bins * 4, cudaMemcpyDefault, st);
+    e = cudaMemcpyAsync(hist_out, h->d_hist, static_cast<size_t>(n) * h->fw * 4, cudaMemcpyDefault, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "output copy");
   return COFIE_OK;
 }
@@ -303,7 +359,7 @@ int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n,
   const MemKind kf = classify(frames, &fdev);
   const MemKind ks = classify(scores), kk = classify(keep), kh = classify(hist_out);
   if (kf == kDevice && fdev != h->device) return h->fail(COFIE_EINVAL, "frames live on another device");
-  const uint32_t B = h->p.bins;
+  const uint32_t B = h->fw;
   if (kf == kDevice) {
     const uint32_t step = h->p.max_frames_per_push;
     for (uint32_t off = 0; off < n; off += step) {
@@ -344,8 +400,8 @@ void free_handle(cofie_ngff* h) {
   if (!h) return;
   DeviceGuard guard(h->device);
   cudaDeviceSynchronize();
-  void* bufs[] = {h->d_hist, h->d_l1, h->d_mask, h->d_ring, h->d_state, h->d_scores,
-                  h->d_keep, h->d_err,  h->d_stage[0], h->d_stage[1], h->d_count, h->d_map};
+  void* bufs[] = {h->d_hist, h->d_l1, h->d_mask, h->d_ring, h->d_state, h->d_scores, h->d_keep,
+                  h->d_err,  h->d_stage[0], h->d_stage[1], h->d_count, h->d_map, h->d_cells};
   for (void* b : bufs)
     if (b) cudaFree(b);
   for (cudaEvent_t ev : h->ev_pool) cudaEventDestroy(ev);
@@ -361,6 +417,8 @@ void free_handle(cofie_ngff* h) {
 }  // namespace
 
 extern "C" {
+
+uint32_t cofie_ngff_feature_words(const cofie_ngff_t* h) { return h ? h->fw : 0; }
 
 void cofie_ngff_default_params(cofie_ngff_params* p, uint32_t width, uint32_t height) {
   if (!p) return;
@@ -420,7 +478,28 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   h->npix = p->width * p->height;
   h->frame_bytes = 3ull * h->npix;
   h->mask_words = (p->l_max + 31) / 32;
-  h->two_n = static_cast<float>(2ull * h->npix);
+  if (p->signal == COFIE_SIGNAL_LOWRES) {
+    h->fw = 256;
+    h->two_n = static_cast<float>(255ull * h->npix);
+  } else if (p->signal == COFIE_SIGNAL_DHASH) {
+    h->fw = 2;
+    h->two_n = 64.0f;
+  } else {
+    h->fw = p->bins;
+    h->two_n = static_cast<float>(2ull * h->npix);
+  }
+  if (p->signal != COFIE_SIGNAL_HISTOGRAM) {
+    FeatArgs& fa = h->fa;
+    fa.frame_bytes = 3ull * h->npix;
+    fa.width = p->width;
+    fa.height = p->height;
+    fa.npix = h->npix;
+    fa.grid_h = p->signal == COFIE_SIGNAL_LOWRES ? 16 : 8;
+    fa.grid_w = p->signal == COFIE_SIGNAL_LOWRES ? 16 : 9;
+    fa.kind = p->signal;
+    for (uint32_t y = 0; y < p->height; ++y) fa.row_h[y * fa.grid_h / p->height] += 1;
+    for (uint32_t x = 0; x < p->width; ++x) fa.col_w[x * fa.grid_w / p->width] += 1;
+  }
   h->size_fast = (h->npix % 16) == 0;
   h->seen.assign(p->max_streams, 0);
 
@@ -446,26 +525,33 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
       h->bin_path = kBinFast;
     }
   }
-  if (h->bin_path < 0 && den >= 2) {
+  bool magic_y_ok = false;
+  if (den >= 2) {
     const uint64_t M = ((1ull << 32) + den - 1) / den;
     if (M <= 0xffffffffull && verify_magic(static_cast<uint32_t>(M), vmax, den, p->bins, true)) {
       lc.magic_y = static_cast<uint32_t>(M);
-      h->bin_path = kBinTwoStep;
+      magic_y_ok = true;
     }
   }
+  if (h->bin_path < 0 && magic_y_ok) h->bin_path = kBinTwoStep;
+  h->fa.use_magic = magic_y_ok ? 1u : 0u;
 
   const uint64_t F = p->max_frames_per_push, S = p->max_streams;
   cudaError_t e = cudaSuccess;
-  if (e == cudaSuccess) e = dalloc(&h->d_hist, F * p->bins);
+  if (e == cudaSuccess) e = dalloc(&h->d_hist, F * h->fw);
   if (e == cudaSuccess) e = dalloc(&h->d_l1, F * p->l_max);
   if (e == cudaSuccess) e = dalloc(&h->d_mask, F * h->mask_words);
-  if (e == cudaSuccess) e = dalloc(&h->d_ring, S * p->l_max * p->bins);
+  if (e == cudaSuccess) e = dalloc(&h->d_ring, S * p->l_max * h->fw);
   if (e == cudaSuccess) e = dalloc(&h->d_state, S);
   if (e == cudaSuccess) e = dalloc(&h->d_scores, F);
   if (e == cudaSuccess) e = dalloc(&h->d_keep, F);
   if (e == cudaSuccess) e = dalloc(&h->d_err, 1);
   if (e == cudaSuccess) e = dalloc(&h->d_count, 1);
   if (e == cudaSuccess) e = dalloc(&h->d_map, COFIE_NGFF_MAX_LMAX);
+  if (e == cudaSuccess && p->signal == COFIE_SIGNAL_DHASH) {
+    e = dalloc(&h->d_cells, F * 72);
+    if (e == cudaSuccess) e = cudaMemset(h->d_cells, 0, F * 72 * sizeof(uint32_t));
+  }
   if (e != cudaSuccess) {
     cudaGetLastError();
     free_handle(h);
@@ -473,7 +559,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     return COFIE_ENOMEM;
   }
   if (e == cudaSuccess) e = cudaMemset(h->d_state, 0, S * sizeof(StreamState));
-  if (e == cudaSuccess) e = cudaMemset(h->d_hist, 0, F * p->bins * sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMemset(h->d_hist, 0, F * h->fw * sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
   for (int i = 0; i < 2 && e == cudaSuccess; ++i) {
@@ -485,6 +571,20 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     const int per_sm = hist_blocks_per_sm(h->bin_path, p->bins);
     if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
     h->hist_grid = h->num_sms * (per_sm > 0 ? per_sm : 1);
+  }
+  if (p->signal != COFIE_SIGNAL_HISTOGRAM) {
+    const uint32_t gpr = p->width / 16, gw = h->fa.grid_w, gh = h->fa.grid_h;
+    const uint64_t groups = h->npix / 16;
+    const uint64_t n_gpr = std::max<uint64_t>(groups, static_cast<uint64_t>(gpr) * gw);
+    h->m_gpr = magic_for(gpr, n_gpr);
+    h->m_h = magic_for(p->height, static_cast<uint64_t>(p->height) * gh);
+    h->m_gw = magic_for(gw, static_cast<uint64_t>(p->width) * gw + gw);
+  }
+  if (e == cudaSuccess && p->signal != COFIE_SIGNAL_HISTOGRAM && p->width % 16 == 0 && h->fa.use_magic &&
+      h->m_gpr && h->m_h && static_cast<uint64_t>(p->width) * h->fa.grid_w < (1ull << 32)) {
+    const int per_sm = cells_blocks_per_sm();
+    if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
+    h->cells_grid = h->num_sms * (per_sm > 0 ? per_sm : 1);
   }
   if (e != cudaSuccess) {
     g_global_error = std::string("CUDA setup failed: ") + cudaGetErrorString(e);
@@ -570,7 +670,7 @@ static_assert(sizeof(StateHeader) == kStateHeader, "state header layout");
 }  // namespace
 
 size_t cofie_ngff_state_bytes(const cofie_ngff_t* h) {
-  return h ? kStateHeader + static_cast<size_t>(h->p.l_max) * h->p.bins * sizeof(uint32_t) : 0;
+  return h ? kStateHeader + static_cast<size_t>(h->p.l_max) * h->fw * sizeof(uint32_t) : 0;
 }
 
 int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream) {
@@ -587,9 +687,10 @@ int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cud
   hdr.height = h->p.height;
   hdr.bins = h->p.bins;
   hdr.l_max = h->p.l_max;
+  hdr.pad0 = h->p.signal;
   uint8_t* b = static_cast<uint8_t*>(buf);
-  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->p.bins * sizeof(uint32_t);
-  const uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->p.bins;
+  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->fw * sizeof(uint32_t);
+  const uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->fw;
   cudaError_t e;
   if (kb == kDevice) {
     // the header's fixed part travels through the handle's pinned-free path: a
@@ -620,13 +721,14 @@ int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, voi
   if (e != cudaSuccess) return h->cuda_fail(e, "state load");
   if (hdr.magic != kStateMagic || hdr.version != kStateVersion)
     return h->fail(COFIE_EINVAL, "not a saved stream state (format tag or version)");
-  if (hdr.width != h->p.width || hdr.height != h->p.height || hdr.bins != h->p.bins || hdr.l_max != h->p.l_max)
-    return h->fail(COFIE_EINVAL, "saved state has another width, height, bins or l_max");
+  if (hdr.width != h->p.width || hdr.height != h->p.height || hdr.bins != h->p.bins || hdr.l_max != h->p.l_max ||
+      hdr.pad0 != h->p.signal)
+    return h->fail(COFIE_EINVAL, "saved state has another width, height, bins, l_max or signal");
   if (hdr.st.t > 0 && (hdr.st.g < 1 || hdr.st.g > h->p.l_max))
     return h->fail(COFIE_EINVAL, "saved state has a gap outside [1, l_max]");
   const uint8_t* b = static_cast<const uint8_t*>(buf);
-  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->p.bins * sizeof(uint32_t);
-  uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->p.bins;
+  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->fw * sizeof(uint32_t);
+  uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->fw;
   e = cudaMemcpyAsync(ring, b + kStateHeader, ring_bytes, cudaMemcpyDefault, st);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(h->d_state + stream, b + offsetof(StateHeader, st), sizeof(StreamState), cudaMemcpyDefault, st);
@@ -662,30 +764,16 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   StreamState ss{t0, 1u, 0u};
   cudaError_t e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "shard state");
-  // the histograms (K1 only): run_segments' selection must not run here, so
-  // the launch sequence is spelled out
-  if (h->dirty_rows) {
-    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->p.bins * 4, st);
+  // the first stage only (histograms or features): the selection runs later
+  if (h->dirty_rows && h->p.signal != COFIE_SIGNAL_DHASH) {
+    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->fw * 4, st);
     if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
   }
   h->dirty_rows = h->p.max_frames_per_push;
-  bool fast = h->size_fast && h->bin_path >= 0 && reinterpret_cast<uintptr_t>(frames) % 16 == 0;
-  HistArgs ha{};
-  ha.frame_bytes = h->frame_bytes;
-  ha.npix = h->npix;
-  ha.groups_per_frame = static_cast<uint32_t>(h->frame_bytes / 48);
-  ha.chunks_per_frame = (ha.groups_per_frame + hist_chunk_groups() - 1) / hist_chunk_groups();
-  ha.timeout_ns = kTimeoutNs;
-  if (fast) {
-    const uint64_t chunks = static_cast<uint64_t>(all.rows) * ha.chunks_per_frame;
-    e = launch_hist_fast(all, ha, h->lc, h->bin_path, h->d_hist, h->d_err,
-                         static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid), st);
-  } else {
-    e = launch_hist_generic(all, ha, h->lc, h->d_hist, st);
-  }
+  e = launch_first_stage(h, all, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
   h->n_hist += 1;
-  h->hist_bytes += static_cast<uint64_t>(all.rows) * (h->frame_bytes + 4ull * h->p.bins);
+  h->hist_bytes += static_cast<uint64_t>(all.rows) * (h->frame_bytes + 4ull * h->fw);
   // K2 over the shard's rows, reading the halo rows before them
   SegTable sh;
   memset(&sh, 0, sizeof sh);
@@ -696,12 +784,7 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   sh.s[0].row0 = n_halo;
   sh.s[0].stream = stream;
   sh.s[0].halo = n_halo;
-  SelectArgs sa{};
-  sa.bins = h->p.bins;
-  sa.l_max = h->p.l_max;
-  sa.mask_words = h->mask_words;
-  sa.tau = h->p.tau;
-  sa.two_n = h->two_n;
+  SelectArgs sa = select_args(h);
   e = launch_window(sh, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
   if (e == cudaSuccess) e = launch_gap_map(sh.s[0], sa, t0, h->d_mask, h->d_map, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(map_out, h->d_map, h->p.l_max * sizeof(uint16_t), cudaMemcpyDefault, st);
@@ -727,12 +810,7 @@ int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap
   DeviceGuard guard(h->device);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   const uint32_t n_halo = h->shard.n_halo, n = h->shard.n;
-  SelectArgs sa{};
-  sa.bins = h->p.bins;
-  sa.l_max = h->p.l_max;
-  sa.mask_words = h->mask_words;
-  sa.tau = h->p.tau;
-  sa.two_n = h->two_n;
+  SelectArgs sa = select_args(h);
   // the stream's ring holds the halo frames (the last frames before t0) ...
   cudaError_t e = launch_ring_store(h->d_hist, n_halo, h->shard.t0 - n_halo, stream, sa, h->d_ring, st);
   // ... and its gap is the resolved entry gap

@@ -52,7 +52,9 @@ struct LumaConsts {
   uint32_t den;
 };
 
-enum BinPath : int { kBinFast = 0, kBinTwoStep = 1 };
+// kCells: the fast kernel's consumers sum grayscale per cell of a grid
+// (the spatial signals) instead of counting bins.
+enum BinPath : int { kBinFast = 0, kBinTwoStep = 1, kCells = 2 };
 
 struct StreamState {
   unsigned long long t;  // frames seen
@@ -72,6 +74,12 @@ struct HistArgs {
   uint32_t groups_per_frame; // frame_bytes / 48 (fast kernel)
   uint32_t chunks_per_frame; // ceil(groups_per_frame / chunk groups)
   uint64_t timeout_ns;
+  // kCells only (width a multiple of 16): the grid (output row stride grid_h * grid_w),
+  // groups per image row, and multiply-high constants for / gpr and / height
+  uint32_t width, height, grid_h, grid_w;
+  uint32_t gpr, m_gpr, m_h;
+  uint32_t wide;  // every cell column is at least 16 pixels wide
+  uint32_t m_gw;  // multiply-high constant for / grid_w (wide path)
 };
 
 struct SelectArgs {
@@ -79,8 +87,19 @@ struct SelectArgs {
   uint32_t l_max;
   uint32_t mask_words;
   float tau;
-  float two_n;        // fp32(2 W H)
+  float two_n;        // fp32 of the distance's denominator: 2 W H (histogram), 255 W H (low-res), 64 (dHash)
   uint32_t zero_hist;  // the scan zeroes the push's histogram rows after use
+  uint32_t dist_kind;  // 0: sum of |differences| (histogram, low-res); 1: Hamming (dHash)
+};
+
+// The spatial signals: per-frame grayscale sums on a grid of cells.
+struct FeatArgs {
+  uint64_t frame_bytes;
+  uint32_t width, height, npix;
+  uint32_t grid_h, grid_w;    // cell rows, cell columns
+  uint32_t kind;              // 1: low-res (writes the cell sums), 2: dHash (writes 64 bits)
+  uint32_t use_magic;         // Y = umulhi(v, magic_y) (host-verified), else v / den
+  uint32_t row_h[16], col_w[16];  // pixels per cell row / cell column
 };
 
 // Launchers (stream-ordered; return the launch error).
@@ -98,6 +117,12 @@ cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_
 uint32_t select_small_max();
 cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
                                 StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st);
+cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const LumaConsts& lc, uint32_t* feat, uint32_t fw,
+                            cudaStream_t st);
+int cells_blocks_per_sm();
+cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* cells,
+                              uint32_t* err, int grid, cudaStream_t st);
+cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st);
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);

@@ -19,6 +19,10 @@
 //   - when the chunk sequence moves to the next frame, the consumers reduce
 //     the 32 lane columns per bin and add them to hist[row][bin] with one
 //     global atomic per bin.
+// The same kernel, instantiated for kCells, serves the spatial signals: the
+// consumers add each 16-pixel group's grayscale to its cell of the grid (one
+// shared atomic per cell the group touches), and the fold adds the CTA's cell
+// sums to the frame's row.
 // Every mbarrier wait is bounded (globaltimer); a wait that runs out sets a
 // bit in the error word, stops issuing work and returns without leaving bulk
 // copies in flight.
@@ -49,6 +53,23 @@ namespace {
 constexpr int kConsumerWarps = COFIE_K1_CONSUMER_WARPS;
 constexpr int kConsumers = kConsumerWarps * 32;
 constexpr int kThreads = kConsumers + 32;  // + one producer warp
+// The spatial signals' shape (consumer warps, ring stages), from a sweep on
+// GB300 over the 1080p stream: 4 warps and a 2-stage ring (4 CTAs per SM)
+// stream fastest.
+#ifndef COFIE_CELL_WARPS
+#define COFIE_CELL_WARPS 4
+#endif
+#ifndef COFIE_CELL_STAGES
+#define COFIE_CELL_STAGES 2
+#endif
+constexpr int kCellWarps = COFIE_CELL_WARPS;
+template <int kBin>
+struct Shape {
+  static constexpr int warps = kBin == kCells ? kCellWarps : kConsumerWarps;
+  static constexpr int consumers = warps * 32;
+  static constexpr int threads = consumers + 32;
+  static constexpr int stages = kBin == kCells ? COFIE_CELL_STAGES : COFIE_K1_STAGES;
+};
 constexpr int kStages = COFIE_K1_STAGES;
 constexpr int kGroupBytes = 48;            // 16 RGB pixels
 constexpr int kChunkGroups = COFIE_K1_CHUNK_GROUPS;
@@ -127,7 +148,10 @@ __device__ __forceinline__ void red_add_shared(uint32_t addr) {
   asm volatile("red.shared.add.u32 [%0], 1;" ::"r"(addr) : "memory");
 }
 
-__device__ __forceinline__ void consumer_bar() { asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory"); }
+template <int kN>
+__device__ __forceinline__ void consumer_bar() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kN) : "memory");
+}
 
 // Luma sums v = wR R + wG G + wB B + half of the four pixels packed in three
 // little-endian words (bytes R0 G0 B0 R1 | G1 B1 R2 G2 | B2 R3 G3 B3).
@@ -154,6 +178,70 @@ __device__ __forceinline__ void count4(uint32_t w0, uint32_t w1, uint32_t w2, co
   red_add_shared(cnt_lane + (bin_of<kBin>(v1, L) << 7));
   red_add_shared(cnt_lane + (bin_of<kBin>(v2, L) << 7));
   red_add_shared(cnt_lane + (bin_of<kBin>(v3, L) << 7));
+}
+
+// One chunk of 16-pixel groups for the spatial signals: group j of the chunk
+// is group g0 + j of its frame (row-major, width a multiple of 16, so a group
+// never spans two image rows). Each run of a group's pixels that lies in one
+// cell is added to that cell with one shared atomic (lanes of a warp that hit
+// the same cell serialise; that costs less than reducing across the warp).
+template <int kN>
+__device__ __forceinline__ void cells_chunk(const uint8_t* buf, uint32_t groups, uint32_t g0, const HistArgs& a,
+                                            const LumaConsts& L, uint32_t* cells, uint32_t tid) {
+  const uint32_t W = a.width, gh = a.grid_h, gw = a.grid_w;
+  for (uint32_t j = tid; j < groups; j += kN) {
+    const uint4* p = reinterpret_cast<const uint4*>(buf + j * kGroupBytes);
+    const uint4 x = p[0], y = p[1], z = p[2];
+    uint32_t v[16];
+    luma4(x.x, x.y, x.z, L, v[0], v[1], v[2], v[3]);
+    luma4(x.w, y.x, y.y, L, v[4], v[5], v[6], v[7]);
+    luma4(y.z, y.w, z.x, L, v[8], v[9], v[10], v[11]);
+    luma4(z.y, z.z, z.w, L, v[12], v[13], v[14], v[15]);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __umulhi(v[i], L.magic_y);  // Y = floor(v / den), host-verified
+    // divisions by multiply-high, each host-verified over its whole range:
+    // image row r = gi / gpr, cell column floor(xg gw / gpr) of the first
+    // pixel (x0 = 16 xg, W = 16 gpr), cell row floor(r gh / H)
+    const uint32_t gi = g0 + j, r = __umulhi(gi, a.m_gpr), xg = gi - r * a.gpr, x0 = xg << 4;
+    const uint32_t crow = __umulhi(r * gh, a.m_h) * gw;
+    uint32_t cx = __umulhi(xg * gw, a.m_gpr);
+    uint32_t edge = (cx + 1) * W;  // pixel x lies past cell column cx iff x gw >= edge
+    if (a.wide) {
+      // cell columns of 16 pixels or more: a group spans one or two cells.
+      // Prefix sums P of the group's grayscale; the first s pixels lie in
+      // cell cx, s = (first x of the next cell column) - x0, capped at 16;
+      // P[s - 1] is picked by a 4-level select tree on the bits of s - 1.
+      uint32_t P[16];
+      P[0] = v[0];
+#pragma unroll
+      for (int i = 1; i < 16; ++i) P[i] = P[i - 1] + v[i];
+      const uint32_t nx = __umulhi(edge + gw - 1, a.m_gw);  // ceil(edge / gw), host-verified
+      const uint32_t i = min(nx - x0, 16u) - 1;
+      uint32_t q[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) q[k] = (i & 1) ? P[2 * k + 1] : P[2 * k];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) q[k] = (i & 2) ? q[2 * k + 1] : q[2 * k];
+#pragma unroll
+      for (int k = 0; k < 2; ++k) q[k] = (i & 4) ? q[2 * k + 1] : q[2 * k];
+      const uint32_t lo = (i & 8) ? q[1] : q[0];
+      atomicAdd(&cells[crow + cx], lo);
+      if (i < 15) atomicAdd(&cells[crow + cx + 1], P[15] - lo);
+    } else {
+      uint32_t acc = 0;
+#pragma unroll
+      for (uint32_t i = 0; i < 16; ++i) {
+        if ((x0 + i) * gw >= edge) {
+          atomicAdd(&cells[crow + cx], acc);
+          acc = 0;
+          ++cx;
+          edge += W;
+        }
+        acc += v[i];
+      }
+      atomicAdd(&cells[crow + cx], acc);
+    }
+  }
 }
 
 // Walks the chunk sequence of a push: chunk c is chunk k of frame row.
@@ -184,13 +272,17 @@ struct ChunkCursor {
 };
 
 template <int kBin>
-__global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, HistArgs a, LumaConsts L,
-                                                             uint32_t* __restrict__ hist, uint32_t* __restrict__ err) {
+__global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTable segs, HistArgs a, LumaConsts L,
+                                                                         uint32_t* __restrict__ hist,
+                                                                         uint32_t* __restrict__ err) {
+  constexpr int kCW = Shape<kBin>::warps, kNC = Shape<kBin>::consumers, kNT = Shape<kBin>::threads;
+  constexpr int kS = Shape<kBin>::stages;
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ SegLite sseg[kMaxSegs];
   uint8_t* ring = smem;
-  uint32_t* cnt = reinterpret_cast<uint32_t*>(smem + kStages * kChunkBytes);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(cnt + L.bins * 32);
+  uint32_t* cnt = reinterpret_cast<uint32_t*>(smem + kS * kChunkBytes);
+  const uint32_t n_cnt = kBin == kCells ? a.grid_h * a.grid_w : L.bins * 32;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(cnt + (kBin == kCells ? kMaxBins : L.bins * 32));
 
   const uint64_t total = static_cast<uint64_t>(segs.rows) * a.chunks_per_frame;
   const uint64_t c0 = total * blockIdx.x / gridDim.x;
@@ -198,17 +290,17 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
   if (c0 >= c1) return;  // uniform across the CTA
 
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
-  for (uint32_t i = tid; i < segs.count; i += kThreads) {
+  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kS);
+  for (uint32_t i = tid; i < segs.count; i += kNT) {
     sseg[i].frames = segs.s[i].frames;
     sseg[i].n = segs.s[i].n;
     sseg[i].row0 = segs.s[i].row0;
   }
-  for (uint32_t i = tid; i < L.bins * 32; i += kThreads) cnt[i] = 0;
+  for (uint32_t i = tid; i < n_cnt; i += kNT) cnt[i] = 0;
   if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kS; ++s) {
       mbar_init(full0 + 8 * s, 1);
-      mbar_init(empty0 + 8 * s, kConsumerWarps);
+      mbar_init(empty0 + 8 * s, kCW);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -216,7 +308,7 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
 
   const uint32_t nseg = segs.count, cpf = a.chunks_per_frame, gpf = a.groups_per_frame;
 
-  if (warp == kConsumerWarps) {
+  if (warp == kCW) {
     // ---------------------------------------------------------- producer --
     if (lane != 0) return;
     const uint64_t pol = l2_read_policy();
@@ -225,7 +317,7 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
     cur.init(c0, cpf, sseg, nseg);
     uint32_t issued = 0;
     for (uint64_t c = c0; c < c1; ++c) {
-      const uint32_t slot = issued % kStages, use = issued / kStages;
+      const uint32_t slot = issued % kS, use = issued / kS;
       if (use > 0 && !mbar_wait_bounded(empty0 + 8 * slot, (use - 1) & 1, a.timeout_ns)) {
         atomicOr(err, kErrProducerTimeout);
         break;
@@ -237,9 +329,9 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
       ++issued;
     }
     // No copy may still be writing shared memory when the CTA exits.
-    const uint32_t first = issued > kStages ? issued - kStages : 0;
+    const uint32_t first = issued > kS ? issued - kS : 0;
     for (uint32_t j = first; j < issued; ++j)
-      if (!mbar_wait_bounded(full0 + 8 * (j % kStages), (j / kStages) & 1, a.timeout_ns))
+      if (!mbar_wait_bounded(full0 + 8 * (j % kS), (j / kS) & 1, a.timeout_ns))
         atomicOr(err, kErrDrainTimeout);
     return;
   }
@@ -252,16 +344,18 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
   bool ok = true;
   uint32_t i = 0;
   for (uint64_t c = c0; c < c1; ++c, ++i) {
-    const uint32_t slot = i % kStages, use = i / kStages;
+    const uint32_t slot = i % kS, use = i / kS;
     if (ok && !mbar_wait_bounded(full0 + 8 * slot, use & 1, a.timeout_ns)) {
       atomicOr(err, kErrConsumerTimeout);
       ok = false;  // keep walking the sequence so every CTA barrier is still reached
     }
-    if (ok) {
+    if constexpr (kBin == kCells) {
+      if (ok) cells_chunk<kNC>(ring + slot * kChunkBytes, cur.groups(gpf), cur.k * kChunkGroups, a, L, cnt, tid);
+    } else if (ok) {
       const uint32_t groups = cur.groups(gpf);
       const uint8_t* buf = ring + slot * kChunkBytes;
 #pragma unroll 2
-      for (uint32_t g = tid; g < groups; g += kConsumers) {
+      for (uint32_t g = tid; g < groups; g += kNC) {
         const uint4* p = reinterpret_cast<const uint4*>(buf + g * kGroupBytes);
         const uint4 x = p[0], y = p[1], z = p[2];
         count4<kBin>(x.x, x.y, x.z, L, cnt_lane);
@@ -269,25 +363,36 @@ __global__ void __launch_bounds__(kThreads) hist_fast_kernel(SegTable segs, Hist
         count4<kBin>(y.z, y.w, z.x, L, cnt_lane);
         count4<kBin>(z.y, z.z, z.w, L, cnt_lane);
       }
+    }
+    if (ok) {
       __syncwarp();
       if (lane == 0) mbar_arrive(empty0 + 8 * slot);
     }
     cur.advance(cpf, sseg, nseg);
     if (c + 1 == c1 || cur.row != row) {
-      // frame done for this CTA: fold the 32 lane columns of every bin
-      consumer_bar();
-      for (uint32_t b = tid; b < L.bins; b += kConsumers) {
-        uint32_t sum = 0;
-        uint32_t* rowp = cnt + b * 32;
-#pragma unroll 8
-        for (uint32_t l = 0; l < 32; ++l) {
-          const uint32_t idx = (l + b) & 31;  // rotate: conflict-free across the warp
-          sum += rowp[idx];
-          rowp[idx] = 0;
+      // frame done for this CTA: fold the 32 lane columns of every bin (or
+      // hand over the cell sums)
+      consumer_bar<kNC>();
+      if (kBin == kCells) {
+        for (uint32_t b = tid; b < n_cnt; b += kNC) {
+          const uint32_t sum = cnt[b];
+          cnt[b] = 0;
+          if (sum && ok) atomicAdd(hist + static_cast<uint64_t>(row) * n_cnt + b, sum);
         }
-        if (sum && ok) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, sum);
+      } else {
+        for (uint32_t b = tid; b < L.bins; b += kNC) {
+          uint32_t sum = 0;
+          uint32_t* rowp = cnt + b * 32;
+#pragma unroll 8
+          for (uint32_t l = 0; l < 32; ++l) {
+            const uint32_t idx = (l + b) & 31;  // rotate: conflict-free across the warp
+            sum += rowp[idx];
+            rowp[idx] = 0;
+          }
+          if (sum && ok) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, sum);
+        }
       }
-      consumer_bar();
+      consumer_bar<kNC>();
       row = cur.row;
     }
   }
@@ -320,6 +425,98 @@ __global__ void __launch_bounds__(kGenericThreads) hist_generic_kernel(SegTable 
     if (cnt[b]) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, cnt[b]);
 }
 
+// The spatial signals (low-res difference, dHash) where the TMA kernel does
+// not apply (width not a multiple of 16, unaligned frames, or no verified
+// multiply-high for the grayscale division): one CTA per frame sums the
+// grayscale of each cell of a grid_h x grid_w grid in shared memory. Fast path
+// (width a multiple of 16, aligned frames): 16-pixel groups, the same dp2a
+// luma as the histogram kernel, runs of pixels of one cell added in registers
+// and flushed with one shared atomic per run. Then low-res writes the cell
+// sums, dHash the 64 bits [mean(r, c) > mean(r, c + 1)] compared exactly by
+// cross-multiplying sums and pixel counts.
+constexpr int kFeatThreads = 512;
+
+__global__ void __launch_bounds__(kFeatThreads) features_kernel(SegTable segs, FeatArgs fa, LumaConsts L,
+                                                                uint32_t* __restrict__ feat, uint32_t fw) {
+  __shared__ uint32_t cell[256];
+  const uint32_t row = blockIdx.x, tid = threadIdx.x;
+  uint32_t seg = 0;
+  while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
+  const uint8_t* frame = segs.s[seg].frames + static_cast<uint64_t>(row - segs.s[seg].row0) * fa.frame_bytes;
+  const uint32_t gh = fa.grid_h, gw = fa.grid_w, W = fa.width, H = fa.height;
+  for (uint32_t i = tid; i < gh * gw; i += kFeatThreads) cell[i] = 0;
+  __syncthreads();
+  const bool fast = (W % 16 == 0) && (reinterpret_cast<uintptr_t>(frame) % 16 == 0) && (fa.frame_bytes % 16 == 0);
+  if (fast) {
+    const uint32_t gpr = W / 16, groups = fa.npix / 16;
+    for (uint32_t g = tid; g < groups; g += kFeatThreads) {
+      const uint32_t y = g / gpr, x0 = (g - y * gpr) * 16;
+      const uint32_t cy = y * gh / H;
+      const uint4* p4 = reinterpret_cast<const uint4*>(frame + static_cast<uint64_t>(g) * 48);
+      const uint4 a = p4[0], b = p4[1], c = p4[2];
+      uint32_t v[16];
+      luma4(a.x, a.y, a.z, L, v[0], v[1], v[2], v[3]);
+      luma4(a.w, b.x, b.y, L, v[4], v[5], v[6], v[7]);
+      luma4(b.z, b.w, c.x, L, v[8], v[9], v[10], v[11]);
+      luma4(c.y, c.z, c.w, L, v[12], v[13], v[14], v[15]);
+      uint32_t cx = x0 * gw / W;
+      uint32_t next = ((cx + 1) * W + gw - 1) / gw;  // first x of the next cell column
+      uint32_t acc = 0;
+#pragma unroll
+      for (uint32_t i = 0; i < 16; ++i) {
+        const uint32_t yv = fa.use_magic ? __umulhi(v[i], L.magic_y) : v[i] / L.den;
+        if (x0 + i >= next) {
+          atomicAdd(&cell[cy * gw + cx], acc);
+          acc = 0;
+          ++cx;
+          next = ((cx + 1) * W + gw - 1) / gw;
+        }
+        acc += yv;
+      }
+      atomicAdd(&cell[cy * gw + cx], acc);
+    }
+  } else {
+    for (uint32_t p = tid; p < fa.npix; p += kFeatThreads) {
+      const uint8_t* px = frame + 3ull * p;
+      const uint32_t yv = (L.w[0] * px[0] + L.w[1] * px[1] + L.w[2] * px[2] + L.half) / L.den;
+      const uint32_t y = p / W, x = p - y * W;
+      atomicAdd(&cell[(y * gh / H) * gw + x * gw / W], yv);
+    }
+  }
+  __syncthreads();
+  uint32_t* out = feat + static_cast<uint64_t>(row) * fw;
+  if (fa.kind == 1) {
+    for (uint32_t i = tid; i < gh * gw; i += kFeatThreads) out[i] = cell[i];
+  } else if (tid < 64) {  // warps 0 and 1: bit (r, c) of the 8 x 8 hash
+    const uint32_t r = tid / 8, c = tid % 8;
+    const uint64_t sa = cell[r * gw + c], sb = cell[r * gw + c + 1];
+    const uint64_t na = static_cast<uint64_t>(fa.row_h[r]) * fa.col_w[c];
+    const uint64_t nb = static_cast<uint64_t>(fa.row_h[r]) * fa.col_w[c + 1];
+    const uint32_t word = __ballot_sync(0xffffffffu, sa * nb > sb * na);
+    if ((tid & 31) == 0) out[tid >> 5] = word;
+  }
+}
+
+// dHash from the 8 x 9 cell sums the fast kernel accumulated (row-major, 72
+// per frame): bit (r, c) = [S(r, c) n(r, c + 1) > S(r, c + 1) n(r, c)], the
+// comparison of the two cell means without division. The cell row is zeroed
+// for the next push once read.
+__global__ void __launch_bounds__(96) dhash_finish_kernel(uint32_t* __restrict__ cells, FeatArgs fa,
+                                                          uint32_t* __restrict__ bits) {
+  const uint32_t row = blockIdx.x, tid = threadIdx.x;
+  uint32_t* c = cells + static_cast<uint64_t>(row) * 72;
+  if (tid < 64) {
+    const uint32_t r = tid / 8, k = tid % 8;
+    const uint64_t sa = c[r * 9 + k], sb = c[r * 9 + k + 1];
+    const uint64_t na = static_cast<uint64_t>(fa.row_h[r]) * fa.col_w[k];
+    const uint64_t nb = static_cast<uint64_t>(fa.row_h[r]) * fa.col_w[k + 1];
+    const uint32_t word = __ballot_sync(0xffffffffu, sa * nb > sb * na);
+    if ((tid & 31) == 0) bits[static_cast<uint64_t>(row) * 2 + (tid >> 5)] = word;
+  }
+  __syncthreads();
+  if (tid < 72) c[tid] = 0;
+}
+
 // Diagnostic: the fast kernel's per-pixel luma and bin functions applied to
 // 4-pixel groups (12 bytes each), one bin index per pixel.
 template <int kBin>
@@ -347,6 +544,11 @@ size_t hist_smem_bytes(uint32_t bins) {
   return static_cast<size_t>(kStages) * kChunkBytes + static_cast<size_t>(bins) * 32 * 4 + 2 * kStages * 8;
 }
 
+static size_t cells_smem_bytes() {
+  constexpr int kS = Shape<kCells>::stages;
+  return static_cast<size_t>(kS) * kChunkBytes + static_cast<size_t>(kMaxBins) * 4 + 2 * kS * 8;
+}
+
 static int configure(int bin_path, uint32_t bins) {
   const size_t smem = hist_smem_bytes(bins);
   cudaError_t e = (bin_path == kBinFast)
@@ -369,6 +571,29 @@ int hist_blocks_per_sm(int bin_path, uint32_t bins) {
 
 uint32_t hist_chunk_groups() { return kChunkGroups; }
 
+int cells_blocks_per_sm() {
+  const size_t smem = cells_smem_bytes();
+  if (cudaFuncSetAttribute(hist_fast_kernel<kCells>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(smem)) != cudaSuccess)
+    return -1;
+  int n = 0;
+  return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, hist_fast_kernel<kCells>, Shape<kCells>::threads, smem) ==
+                 cudaSuccess
+             ? n
+             : -1;
+}
+
+cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* cells,
+                              uint32_t* err, int grid, cudaStream_t st) {
+  hist_fast_kernel<kCells><<<grid, Shape<kCells>::threads, cells_smem_bytes(), st>>>(segs, a, lc, cells, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st) {
+  dhash_finish_kernel<<<rows, 96, 0, st>>>(cells, fa, bits);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
                              uint32_t* hist, uint32_t* err, int grid, cudaStream_t st) {
   const size_t smem = hist_smem_bytes(lc.bins);
@@ -383,6 +608,12 @@ cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const L
                                 cudaStream_t st) {
   dim3 grid((a.npix + kGenericPixels - 1) / kGenericPixels, segs.rows);
   hist_generic_kernel<<<grid, kGenericThreads, 0, st>>>(segs, a, lc, hist);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const LumaConsts& lc, uint32_t* feat, uint32_t fw,
+                            cudaStream_t st) {
+  features_kernel<<<segs.rows, kFeatThreads, 0, st>>>(segs, fa, lc, feat, fw);
   return cudaGetLastError();
 }
 

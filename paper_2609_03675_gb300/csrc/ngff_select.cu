@@ -70,6 +70,8 @@ __device__ __forceinline__ void window_row(uint32_t row, uint32_t lane, const Se
         const uint4 x = c4[q], y = s4[q];
         d += absdiff(x.x, y.x) + absdiff(x.y, y.y) + absdiff(x.z, y.z) + absdiff(x.w, y.w);
       }
+    } else if (a.dist_kind == 1) {  // Hamming distance of bit vectors (dHash)
+      for (uint32_t b = 0; b < B; ++b) d += __popc(ct[b] ^ src[b]);
     } else {
 #pragma unroll 4
       for (uint32_t b = 0; b < B; ++b) d += absdiff(ct[b], src[b]);
@@ -353,7 +355,7 @@ cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max) {
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
                           const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
   const uint32_t grid = (segs.rows + kWinWarps - 1) / kWinWarps;
-  if (a.bins % 4 == 0)
+  if (a.bins % 4 == 0 && a.dist_kind == 0)
     window_kernel<true><<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
   else
     window_kernel<false><<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
@@ -373,7 +375,7 @@ cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_
 cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
                                 StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
   const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
-  const bool vec = a.bins % 4 == 0, one = a.mask_words == 1;
+  const bool vec = a.bins % 4 == 0 && a.dist_kind == 0, one = a.mask_words == 1;
   if (vec && one)
     select_small_kernel<true, true><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
   else if (vec)

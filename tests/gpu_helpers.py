@@ -24,7 +24,8 @@ def run_stream(f, frames_dev: torch.Tensor, chunks, stream: int = 0):
     torch.cuda.synchronize()
     f.status()
     cat = (lambda xs, d: torch.cat(xs).cpu().numpy() if xs else np.zeros((0,), d))
-    return (cat(hs, np.int32).view(np.uint32).reshape(-1, f.bins), cat(ss, np.float32), cat(ks, np.uint8))
+    return (cat(hs, np.int32).view(np.uint32).reshape(-1, f.feature_words), cat(ss, np.float32),
+            cat(ks, np.uint8))
 
 
 def assert_parity(got, want, tau: float, label: str = ""):

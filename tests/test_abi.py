@@ -36,8 +36,8 @@ def test_exports_every_declared_symbol(lib):
 
 def test_param_struct_layout_matches_header(lib):
     from paper_2609_03675_gb300 import _abi
-    # width..luma_den: 10 x 4 bytes, max_streams, max_frames_per_push, device, pad, u64
-    assert ctypes.sizeof(_abi.Params) == 64
+    # width..luma_den: 10 x 4 bytes, max_streams, max_frames_per_push, device, pad, u64, signal, reserved
+    assert ctypes.sizeof(_abi.Params) == 72
     assert ctypes.sizeof(_abi.PushDesc) == 32
 
 
@@ -76,3 +76,18 @@ def test_null_handle_calls_are_rejected(lib):
     assert lib.cofie_ngff_status(None, None) == _abi.EINVAL
     assert lib.cofie_ngff_last_error(None) == b""
     lib.cofie_ngff_destroy(None)
+
+
+@pytest.mark.parametrize("width,height,signal,msg", [
+    (64, 48, 3, "signal"), (15, 48, 1, "low-res"), (64, 15, 1, "low-res"), (4097, 4097, 1, "low-res"),
+    (8, 48, 2, "dHash"), (64, 7, 2, "dHash"), (46341, 46340, 2, "too large"),
+])
+def test_create_rejects_bad_signal_shapes(lib, width, height, signal, msg):
+    from paper_2609_03675_gb300 import _abi
+    p = _abi.Params()
+    lib.cofie_ngff_default_params(ctypes.byref(p), width, height)
+    p.signal = signal
+    h = ctypes.c_void_p()
+    assert lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h)) == _abi.EINVAL
+    assert msg in lib.cofie_ngff_global_error().decode()
+    assert not h.value
