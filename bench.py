@@ -51,6 +51,8 @@ def parse():
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
     ap.add_argument("--qer-frames", type=int, default=128, help="candidate frames of the qer workload")
+    ap.add_argument("--signal", choices=["histogram", "lowres", "dhash"], default="histogram",
+                    help="NGFF's novelty signal for the hd1080 workload (histogram is the paper's)")
     ap.add_argument("--frames", type=int, default=3600,
                     help="use the first FRAMES frames of the stream (small cases for profiling; default all 3600)")
     return ap.parse_args()
@@ -155,14 +157,19 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def oracle_sample(frames_u8_ptr, spec, target_s: float):
-    """The oracle as it stands (single-threaded C) on the first k frames of the
-    stream; k sized to about target_s seconds of CPU work."""
+SIGNALS = {"histogram": 0, "lowres": 1, "dhash": 2}
+
+
+def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0):
+    """The oracle as it stands (single-threaded C for the histogram, numpy for
+    the spatial signals) on the first k frames of the stream; k sized to about
+    target_s seconds of CPU work."""
     import ctypes
 
     import numpy as np
 
     import oracle as O
+    from oracle import signals_oracle as SO
     o = O.load()
     p = O.Params(spec.width, spec.height)
     fb = spec.frame_bytes
@@ -170,7 +177,10 @@ def oracle_sample(frames_u8_ptr, spec, target_s: float):
     def run(k):
         arr = np.ctypeslib.as_array((ctypes.c_uint8 * (k * fb)).from_address(frames_u8_ptr))
         t = time.perf_counter()
-        o.run(arr.reshape(k, spec.height, spec.width, 3), p)
+        if signal:
+            SO.run(arr.reshape(k, spec.height, spec.width, 3), p, signal)
+        else:
+            o.run(arr.reshape(k, spec.height, spec.width, 3), p)
         return time.perf_counter() - t
 
     t2 = run(2)
@@ -200,7 +210,8 @@ def bench_gb300(args):
     dev = host.to("cuda", non_blocking=True)
     scores = torch.empty(T, dtype=torch.float32, device="cuda")
     keep = torch.empty(T, dtype=torch.uint8, device="cuda")
-    f = NGFF(spec.width, spec.height, max_frames_per_push=T)
+    signal = SIGNALS[args.signal]
+    f = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=signal)
     stream = torch.cuda.current_stream()
 
     def step():
@@ -243,7 +254,7 @@ def bench_gb300(args):
     k1_ms = prof["hist_ms"] / max(prof["hist_timed"], 1)
     k1_bytes = prof["hist_bytes"] / max(prof["hist_launches"], 1)
     achieved = k1_bytes / (k1_ms / 1e3) / 1e9
-    traffic = k1_traffic_per_launch()
+    traffic = k1_traffic_per_launch() if signal == 0 else None
 
     # end to end through the same C entry point with host buffers: H2D of the
     # step's frames and D2H of its scores and keep codes inside the timed region
@@ -251,7 +262,7 @@ def bench_gb300(args):
     if not args.no_e2e:
         hs = torch.empty(T, dtype=torch.float32, pin_memory=True)
         hk = torch.empty(T, dtype=torch.uint8, pin_memory=True)
-        fe = NGFF(spec.width, spec.height, max_frames_per_push=T)
+        fe = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=signal)
 
         def estep():
             fe.reset()
@@ -295,9 +306,11 @@ def bench_gb300(args):
 
     cpu = None
     if rank == 0 and world == 1 and args.cpu_seconds > 0:
-        k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds)
+        k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds, signal)
+        what = "single-threaded C oracle (histograms + selection)" if signal == 0 else \
+            f"numpy signals oracle ({args.signal} features + selection)"
         cpu = {"value": k / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"first {k} frames of the 1080p stream, single-threaded C oracle (histograms + selection)"}
+               "sample": f"first {k} frames of the 1080p stream, {what}"}
 
     if rank == 0:
         line = {
@@ -305,15 +318,17 @@ def bench_gb300(args):
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u8", "data": "synthetic",
             "config": {"workload": f"1080p stream: {T} uint8 RGB frames of 1920x1080 (HWC), one whole-stream push "
-                                   "per step, B=32, L_max=30, tau_h=0.30",
-                       "frames_per_step": T, "width": spec.width, "height": spec.height, "bins": 32, "l_max": 30,
+                                   "per step, B=32, L_max=30, tau_h=0.30"
+                                   + ("" if signal == 0 else f", signal {args.signal} in place of the histogram"),
+                       "signal": args.signal, "frames_per_step": T, "width": spec.width, "height": spec.height, "bins": 32, "l_max": 30,
                        "tau": 0.30, "l2": f"inputs larger than L2 ({T * spec.frame_bytes / 1e9:.1f} GB per step), no flush",
                        "parallelism": f"{world} independent stream(s), one per GPU"},
             "pixel_gbs": pixel_gbs,
             "frac_of_nominal_8tbs": pixel_gbs / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "peak_kind": f"{peak_kind} copy bandwidth", "traffic": traffic,
-                         "kernel": "ngff histogram (K1)", "launch_ms": k1_ms, "bytes_per_launch": k1_bytes,
+                         "kernel": "ngff histogram (K1)" if signal == 0 else f"ngff {args.signal} cell sums (K1 cells)",
+                         "launch_ms": k1_ms, "bytes_per_launch": k1_bytes,
                          "select_ms_per_step": prof["select_ms"] / max(prof["select_timed"], 1)},
             "e2e": e2e,
             "cpu_baseline": cpu,
