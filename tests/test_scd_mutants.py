@@ -1,0 +1,76 @@
+"""Plants one-spot mistakes in a copy of the scene-change oracle (on the CPU)
+and checks that the pins of test_scd_oracle catch each of them."""
+import inspect
+import types
+
+import pytest
+
+from oracle import scd_oracle as SC
+from tests import test_scd_oracle as PINS
+
+MUTANTS = {
+    "cut does not end the run": ("            flags[t] = True\n            acc = 0\n",
+                                 "            flags[t] = True\n"),
+    "low difference does not end the run": ("        else:\n            acc = 0\n", "        else:\n            pass\n"),
+    "fires on every frame past T_b": ("and not at_least(before, two_n, t_cut)", ""),
+    "strict comparison": (">= np.float32(threshold)", "> np.float32(threshold)"),
+    "scene change before novelty": (
+        "        if at_least(max(na, nr), two_n, p.tau):\n            keep[t] = O.KEEP_NOVELTY\n"
+        "        elif scene[t]:\n            keep[t] = KEEP_SCENE\n",
+        "        if scene[t]:\n            keep[t] = KEEP_SCENE\n"
+        "        elif at_least(max(na, nr), two_n, p.tau):\n            keep[t] = O.KEEP_NOVELTY\n"),
+    "gap before scene change": (
+        "        elif scene[t]:\n            keep[t] = KEEP_SCENE\n        elif t - r >= p.l_max:\n"
+        "            keep[t] = O.KEEP_GAP\n",
+        "        elif t - r >= p.l_max:\n            keep[t] = O.KEEP_GAP\n        elif scene[t]:\n"
+        "            keep[t] = KEEP_SCENE\n"),
+    "scene keeps do not move r": ("        if keep[t]:\n            r = t\n",
+                                  "        if keep[t] and keep[t] != KEEP_SCENE:\n            r = t\n"),
+    "gradual threshold used for the cut": ("    if at_least(a, two_n, t_cut):\n        return HIGH",
+                                           "    if at_least(a, two_n, t_grad):\n        return HIGH"),
+}
+
+
+def _mutant(src_from, src_to):
+    src = inspect.getsource(SC)
+    assert src_from in src, "mutation site not found"
+    mod = types.ModuleType("scd_mutant")
+    mod.__dict__["__name__"] = "scd_mutant"
+    exec(compile(src.replace(src_from, src_to, 1), "scd_mutant", "exec"), mod.__dict__)
+    return mod
+
+
+def _pins():
+    return [(n, f) for n, f in inspect.getmembers(PINS, inspect.isfunction) if n.startswith("test_")]
+
+
+def _call(fn):
+    marks = getattr(fn, "pytestmark", [])
+    params = [m for m in marks if m.name == "parametrize"]
+    if not params:
+        fn()
+        return
+    names = [s.strip() for s in params[0].args[0].split(",")]
+    for vals in params[0].args[1]:
+        vals = vals if isinstance(vals, tuple) else (vals,)
+        fn(**dict(zip(names, vals)))
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_each_mutant_is_caught(name, monkeypatch):
+    mod = _mutant(*MUTANTS[name])
+    monkeypatch.setattr(PINS, "SC", mod)
+    caught = []
+    for pin, fn in _pins():
+        try:
+            _call(fn)
+        except AssertionError:
+            caught.append(pin)
+    assert caught, f"mutant '{name}' passes every pin"
+
+
+def test_unmutated_copy_passes_every_pin(monkeypatch):
+    mod = _mutant("KEEP_SCENE = 4", "KEEP_SCENE = 4")
+    monkeypatch.setattr(PINS, "SC", mod)
+    for _, fn in _pins():
+        _call(fn)
