@@ -51,7 +51,7 @@ def parse():
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
     ap.add_argument("--qer-frames", type=int, default=128, help="candidate frames of the qer workload")
-    ap.add_argument("--signal", choices=["histogram", "lowres", "dhash"], default="histogram",
+    ap.add_argument("--signal", choices=["histogram", "lowres", "dhash", "scd"], default="histogram",
                     help="NGFF's novelty signal for the hd1080 workload (histogram is the paper's)")
     ap.add_argument("--frames", type=int, default=3600,
                     help="use the first FRAMES frames of the stream (small cases for profiling; default all 3600)")
@@ -157,7 +157,7 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-SIGNALS = {"histogram": 0, "lowres": 1, "dhash": 2}
+SIGNALS = {"histogram": 0, "lowres": 1, "dhash": 2, "scd": 3}
 
 
 def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0):
@@ -169,6 +169,7 @@ def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0):
     import numpy as np
 
     import oracle as O
+    from oracle import scd_oracle as SC
     from oracle import signals_oracle as SO
     o = O.load()
     p = O.Params(spec.width, spec.height)
@@ -177,7 +178,9 @@ def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0):
     def run(k):
         arr = np.ctypeslib.as_array((ctypes.c_uint8 * (k * fb)).from_address(frames_u8_ptr))
         t = time.perf_counter()
-        if signal:
+        if signal == 3:
+            SC.run(arr.reshape(k, spec.height, spec.width, 3), p, 0.30, 0.10)
+        elif signal:
             SO.run(arr.reshape(k, spec.height, spec.width, 3), p, signal)
         else:
             o.run(arr.reshape(k, spec.height, spec.width, 3), p)
@@ -307,8 +310,9 @@ def bench_gb300(args):
     cpu = None
     if rank == 0 and world == 1 and args.cpu_seconds > 0:
         k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds, signal)
-        what = "single-threaded C oracle (histograms + selection)" if signal == 0 else \
-            f"numpy signals oracle ({args.signal} features + selection)"
+        what = {0: "single-threaded C oracle (histograms + selection)",
+                3: "C oracle histograms + the scene-change oracle's rule (Python)"}.get(
+            signal, f"numpy signals oracle ({args.signal} features + selection)")
         cpu = {"value": k / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
                "sample": f"first {k} frames of the 1080p stream, {what}"}
 
@@ -733,7 +737,7 @@ def bench_shards(args):
 
 
 def bench_signals(args):
-    """The three NGFF signals on the 1080p stream (frames/s, first-stage
+    """The NGFF signals on the 1080p stream (frames/s, first-stage
     bandwidth against the measured copy peak) and on the 720p rare-event
     stream (keep ratio and event recall across thresholds): the synthetic
     counterpart of the paper's signal ablation."""
@@ -741,8 +745,8 @@ def bench_signals(args):
 
     import synth
     from paper_2609_03675_gb300 import NGFF
-    names = {0: "histogram", 1: "lowres", 2: "dhash"}
-    taus = {0: (0.30, 0.10, 0.05), 1: (0.05, 0.02, 0.01), 2: (0.20, 0.10, 0.05)}
+    names = {0: "histogram", 1: "lowres", 2: "dhash", 3: "scd"}
+    taus = {0: (0.30, 0.10, 0.05), 1: (0.05, 0.02, 0.01), 2: (0.20, 0.10, 0.05), 3: (0.30, 0.10, 0.05)}
     peak, peak_kind = peaks()
     spec = synth.hd1080()
     T = min(spec.frames, 600)

@@ -47,7 +47,7 @@
 extern "C" {
 #endif
 
-#define COFIE_NGFF_ABI_VERSION 2
+#define COFIE_NGFF_ABI_VERSION 3
 
 /* Return codes. */
 #define COFIE_OK 0
@@ -62,11 +62,13 @@ extern "C" {
 #define COFIE_KEEP_NOVELTY 1 /* s >= tau_h (Eq. 5, first term) */
 #define COFIE_KEEP_GAP 2     /* t - r(t) >= L_max and not novelty (Eq. 5, second term) */
 #define COFIE_KEEP_FIRST 3   /* the stream's first frame (Sec. 3.2 safeguard) */
+#define COFIE_KEEP_SCENE 4   /* a scene change (signal COFIE_SIGNAL_SCD only), not novelty */
 
 /* Novelty signals (the distance d inside Eqs. 3-5). */
 #define COFIE_SIGNAL_HISTOGRAM 0 /* TV distance of B-bin grayscale histograms (Sec. 3.2, the paper's signal) */
 #define COFIE_SIGNAL_LOWRES 1    /* mean |difference| of 16 x 16-cell block-averaged grayscale frames */
 #define COFIE_SIGNAL_DHASH 2     /* Hamming distance / 64 of 9 x 8-cell difference hashes */
+#define COFIE_SIGNAL_SCD 3       /* the histogram rule plus twin-comparison scene changes */
 
 /* Limits. */
 #define COFIE_NGFF_MAX_BINS 256
@@ -100,8 +102,22 @@ typedef struct cofie_ngff cofie_ngff_t;
  *                     dHash: 8 rows x 9 columns of cells, bit (r, c) = cell mean
  *                       (r, c) > cell mean (r, c+1), d = Hamming distance / 64
  *                       (W >= 9, H >= 8).
+ *                     scene change detection + H-diff: the histogram rule
+ *                       unchanged, and a frame is also kept (code
+ *                       COFIE_KEEP_SCENE, moving r(t)) at a scene change found
+ *                       by twin comparison of the adjacent histogram
+ *                       differences SD_t = d(c_t, c_{t-1}): a cut when
+ *                       SD_t >= scd_cut; frames with scd_gradual <= SD_t <
+ *                       scd_cut form a run whose summed SD is a gradual
+ *                       transition at the frame where the sum first reaches
+ *                       scd_cut; a cut or SD_t < scd_gradual ends the run.
+ *                       Comparisons are fp32(L1 numerator) / fp32(2 W H).
+ *                       Streams of this signal cannot be sharded.
  *                     hist_out of cofie_ngff_push_ex then receives the signal's
  *                     feature rows (cofie_ngff_feature_words uint32 per frame).
+ *   scd_cut, scd_gradual
+ *                     the twin-comparison thresholds T_b, T_s of the scene
+ *                     change signal (non-NaN); defaults 0.30f and 0.10f.
  */
 typedef struct {
   uint32_t width, height;
@@ -116,6 +132,8 @@ typedef struct {
   int32_t device;
   uint64_t host_stage_bytes;
   uint32_t signal;
+  float scd_cut;
+  float scd_gradual;
   uint32_t reserved;
 } cofie_ngff_params;
 
@@ -212,15 +230,16 @@ int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames,
  * Checkpoint and resume of one stream. The saved state is everything a later
  * push depends on (Sec. 3.2: r(t) enters only through the gap t - r(t), and
  * distances reach back at most L_max frames): a 64-byte header (format tag
- * "NGFS", version 1, width, height, bins, l_max, frames seen t, current gap
- * g) followed by the ring of the last l_max histograms (l_max * bins uint32,
+ * "NGFS", version 2, width, height, bins, l_max, signal, frames seen t,
+ * current gap g, the scene-change signal's open run sum) followed by the ring
+ * of the last l_max feature rows (l_max * cofie_ngff_feature_words uint32,
  * slot i holds the frame t' with t' mod l_max == i).
  *   cofie_ngff_state_bytes   the size of that buffer.
  *   cofie_ngff_state_save    writes stream `stream`'s state to buf (device or
  *                            host memory; host memory synchronises cuda_stream).
  *   cofie_ngff_state_load    restores a saved state into stream `stream` of a
- *                            handle with the same width, height, bins and l_max
- *                            (COFIE_EINVAL otherwise); pushes that follow behave
+ *                            handle with the same width, height, bins, l_max and
+ *                            signal (COFIE_EINVAL otherwise); pushes that follow behave
  *                            exactly as if the saved stream had continued.
  */
 size_t cofie_ngff_state_bytes(const cofie_ngff_t* h);

@@ -40,7 +40,7 @@ class NGFF:
     def __init__(self, width: int, height: int, *, bins: int = 32, l_max: int = 30, m_min: int = 4,
                  tau: float = 0.30, luma_weights=(299, 587, 114), luma_den: int = 1000, max_streams: int = 1,
                  max_frames_per_push: int = 4096, device: int | None = None, host_stage_bytes: int = 0,
-                 signal: int = 0):
+                 signal: int = 0, scd_cut: float | None = None, scd_gradual: float | None = None):
         lib = _abi.load()
         p = _abi.Params()
         lib.cofie_ngff_default_params(ctypes.byref(p), width, height)
@@ -53,6 +53,10 @@ class NGFF:
         p.device = device
         p.host_stage_bytes = host_stage_bytes
         p.signal = signal
+        if scd_cut is not None:
+            p.scd_cut = scd_cut
+        if scd_gradual is not None:
+            p.scd_gradual = scd_gradual
         h = ctypes.c_void_p()
         rc = lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h))
         if rc != _abi.OK:

@@ -13,9 +13,9 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libcofie_ngff.so")
 
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EDEVICE = 0, 1, 2, 3, 4, 5
-KEEP_DROP, KEEP_NOVELTY, KEEP_GAP, KEEP_FIRST = 0, 1, 2, 3
+KEEP_DROP, KEEP_NOVELTY, KEEP_GAP, KEEP_FIRST, KEEP_SCENE = 0, 1, 2, 3, 4
 MAX_BINS, MAX_LMAX, MAX_BATCH = 256, 256, 64
-SIGNAL_HISTOGRAM, SIGNAL_LOWRES, SIGNAL_DHASH = 0, 1, 2
+SIGNAL_HISTOGRAM, SIGNAL_LOWRES, SIGNAL_DHASH, SIGNAL_SCD = 0, 1, 2, 3
 
 # Every symbol include/cofie_ngff.h declares.
 EXPORTS = (
@@ -67,6 +67,8 @@ class Params(ctypes.Structure):
         ("device", ctypes.c_int32),
         ("host_stage_bytes", ctypes.c_uint64),
         ("signal", ctypes.c_uint32),
+        ("scd_cut", ctypes.c_float),
+        ("scd_gradual", ctypes.c_float),
         ("reserved", ctypes.c_uint32),
     ]
 

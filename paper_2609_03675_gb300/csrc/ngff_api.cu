@@ -162,7 +162,9 @@ int validate_params(const cofie_ngff_params* p, std::string& why) {
     return why = "luma weights must sum to luma_den", COFIE_EINVAL;
   if (p->max_streams < 1) return why = "max_streams must be >= 1", COFIE_EINVAL;
   if (p->max_frames_per_push < 1) return why = "max_frames_per_push must be >= 1", COFIE_EINVAL;
-  if (p->signal > COFIE_SIGNAL_DHASH) return why = "signal must be one of COFIE_SIGNAL_*", COFIE_EINVAL;
+  if (p->signal > COFIE_SIGNAL_SCD) return why = "signal must be one of COFIE_SIGNAL_*", COFIE_EINVAL;
+  if (p->signal == COFIE_SIGNAL_SCD && (p->scd_cut != p->scd_cut || p->scd_gradual != p->scd_gradual))
+    return why = "scd_cut or scd_gradual is NaN", COFIE_EINVAL;
   if (p->signal == COFIE_SIGNAL_LOWRES && (p->width < 16 || p->height < 16 || npix > (1ull << 24)))
     return why = "the low-res signal needs width, height >= 16 and width * height <= 2^24", COFIE_EINVAL;
   if (p->signal == COFIE_SIGNAL_DHASH && (p->width < 9 || p->height < 8))
@@ -211,7 +213,7 @@ double sum_pairs(const std::vector<cudaEvent_t>& pool, size_t used, cudaError_t*
 // The first stage over the rows of segs: grayscale histograms (K1), or the
 // spatial signal's per-frame features.
 cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
-  const bool cells = h->p.signal != COFIE_SIGNAL_HISTOGRAM;
+  const bool cells = h->p.signal == COFIE_SIGNAL_LOWRES || h->p.signal == COFIE_SIGNAL_DHASH;
   bool fast = cells ? h->cells_grid > 0 : h->size_fast && h->bin_path >= 0;
   for (uint32_t i = 0; i < segs.count && fast; ++i)
     if (reinterpret_cast<uintptr_t>(segs.s[i].frames) % 16 != 0) fast = false;
@@ -255,6 +257,9 @@ SelectArgs select_args(const cofie_ngff* h) {
   sa.tau = h->p.tau;
   sa.two_n = h->two_n;
   sa.dist_kind = h->p.signal == COFIE_SIGNAL_DHASH ? 1u : 0u;
+  sa.scd = h->p.signal == COFIE_SIGNAL_SCD ? 1u : 0u;
+  sa.scd_cut = h->p.scd_cut;
+  sa.scd_grad = h->p.scd_gradual;
   return sa;
 }
 
@@ -437,6 +442,10 @@ void cofie_ngff_default_params(cofie_ngff_params* p, uint32_t width, uint32_t he
   p->max_frames_per_push = 4096;
   p->device = -1;
   p->host_stage_bytes = 0;
+  p->signal = COFIE_SIGNAL_HISTOGRAM;
+  p->scd_cut = 0.30f;     // twin-comparison thresholds of the scene-change signal
+  p->scd_gradual = 0.10f;
+  p->reserved = 0;
 }
 
 int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
@@ -488,7 +497,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     h->fw = p->bins;
     h->two_n = static_cast<float>(2ull * h->npix);
   }
-  if (p->signal != COFIE_SIGNAL_HISTOGRAM) {
+  if (p->signal == COFIE_SIGNAL_LOWRES || p->signal == COFIE_SIGNAL_DHASH) {
     FeatArgs& fa = h->fa;
     fa.frame_bytes = 3ull * h->npix;
     fa.width = p->width;
@@ -572,7 +581,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
     h->hist_grid = h->num_sms * (per_sm > 0 ? per_sm : 1);
   }
-  if (p->signal != COFIE_SIGNAL_HISTOGRAM) {
+  if (p->signal == COFIE_SIGNAL_LOWRES || p->signal == COFIE_SIGNAL_DHASH) {
     const uint32_t gpr = p->width / 16, gw = h->fa.grid_w, gh = h->fa.grid_h;
     const uint64_t groups = h->npix / 16;
     const uint64_t n_gpr = std::max<uint64_t>(groups, static_cast<uint64_t>(gpr) * gw);
@@ -580,7 +589,8 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     h->m_h = magic_for(p->height, static_cast<uint64_t>(p->height) * gh);
     h->m_gw = magic_for(gw, static_cast<uint64_t>(p->width) * gw + gw);
   }
-  if (e == cudaSuccess && p->signal != COFIE_SIGNAL_HISTOGRAM && p->width % 16 == 0 && h->fa.use_magic &&
+  if (e == cudaSuccess && (p->signal == COFIE_SIGNAL_LOWRES || p->signal == COFIE_SIGNAL_DHASH) &&
+      p->width % 16 == 0 && h->fa.use_magic &&
       h->m_gpr && h->m_h && static_cast<uint64_t>(p->width) * h->fa.grid_w < (1ull << 32)) {
     const int per_sm = cells_blocks_per_sm();
     if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
@@ -656,14 +666,14 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
 namespace {
 
 constexpr uint32_t kStateMagic = 0x5346474Eu;  // "NGFS" little-endian
-constexpr uint32_t kStateVersion = 1;
+constexpr uint32_t kStateVersion = 2;
 constexpr size_t kStateHeader = 64;
 
 struct StateHeader {  // the first 64 bytes of a saved state
   uint32_t magic, version, width, height, bins, l_max;
   uint32_t pad0, pad1;
-  StreamState st;  // frames seen, current gap (16 bytes)
-  uint32_t reserved[4];
+  StreamState st;  // frames seen, current gap, open scene-change run (24 bytes)
+  uint32_t reserved[2];
 };
 static_assert(sizeof(StateHeader) == kStateHeader, "state header layout");
 
@@ -743,6 +753,8 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   if (!h) return COFIE_EINVAL;
   if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
   if (!frames || !map_out || n == 0) return h->fail(COFIE_EINVAL, "frames and map_out are required, n >= 1");
+  if (h->p.signal == COFIE_SIGNAL_SCD)  // a scene-change run can reach back past any halo
+    return h->fail(COFIE_EINVAL, "streams of the scene-change signal cannot be sharded");
   const uint64_t want_halo = t0 < h->p.l_max ? t0 : h->p.l_max;
   if (n_halo != want_halo) return h->fail(COFIE_EINVAL, "n_halo must be min(t0, l_max)");
   if (static_cast<uint64_t>(n_halo) + n > h->p.max_frames_per_push)
@@ -761,7 +773,7 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   all.s[0].frames = frames;
   all.s[0].n = n_halo + n;
   all.s[0].stream = stream;
-  StreamState ss{t0, 1u, 0u};
+  StreamState ss{t0, 1u, 0u, 0ull};
   cudaError_t e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "shard state");
   // the first stage only (histograms or features): the selection runs later
@@ -814,7 +826,7 @@ int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap
   // the stream's ring holds the halo frames (the last frames before t0) ...
   cudaError_t e = launch_ring_store(h->d_hist, n_halo, h->shard.t0 - n_halo, stream, sa, h->d_ring, st);
   // ... and its gap is the resolved entry gap
-  StreamState ss{h->shard.t0, h->shard.t0 > 0 ? entry_gap : 1u, 0u};
+  StreamState ss{h->shard.t0, h->shard.t0 > 0 ? entry_gap : 1u, 0u, 0ull};
   if (e == cudaSuccess) e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "shard commit");
   const MemKind ks = classify(scores_out), kk = classify(keep_out);

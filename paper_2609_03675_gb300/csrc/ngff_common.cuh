@@ -57,9 +57,10 @@ struct LumaConsts {
 enum BinPath : int { kBinFast = 0, kBinTwoStep = 1, kCells = 2 };
 
 struct StreamState {
-  unsigned long long t;  // frames seen
-  uint32_t g;            // t - r(t) of the next frame (valid when t > 0)
+  unsigned long long t;    // frames seen
+  uint32_t g;              // t - r(t) of the next frame (valid when t > 0)
   uint32_t pad;
+  unsigned long long acc;  // scene-change signal: L1 numerator summed over the open gradual run (0: none)
 };
 
 // Bits of the device error word.
@@ -90,6 +91,8 @@ struct SelectArgs {
   float two_n;        // fp32 of the distance's denominator: 2 W H (histogram), 255 W H (low-res), 64 (dHash)
   uint32_t zero_hist;  // the scan zeroes the push's histogram rows after use
   uint32_t dist_kind;  // 0: sum of |differences| (histogram, low-res); 1: Hamming (dHash)
+  uint32_t scd;        // twin-comparison scene changes are added to the rule
+  float scd_cut, scd_grad;
 };
 
 // The spatial signals: per-frame grayscale sums on a grid of cells.

@@ -111,11 +111,105 @@ __device__ __forceinline__ uint32_t step_gap(const uint32_t* m, uint32_t g) {
   return ((word >> ((g - 1) & 31)) & 1u) ? 1u : g + 1u;
 }
 
+// (reset, sum) pairs of the twin comparison's run accumulator over a span of
+// frames: "reset" marks that the run ended inside the span, "sum" is the L1
+// numerator summed since the last end. Spans combine left to right:
+static_assert(kScanTile == 4 * kScanThreads, "scd_tile: four frames per thread");
+
+struct RunSum {
+  uint32_t reset;
+  unsigned long long sum;
+};
+__device__ __forceinline__ RunSum run_cat(RunSum a, RunSum b) {
+  return RunSum{a.reset | b.reset, b.reset ? b.sum : a.sum + b.sum};
+}
+__device__ __forceinline__ RunSum run_shfl_up(RunSum v, uint32_t off) {
+  return RunSum{__shfl_up_sync(0xffffffffu, v.reset, off), __shfl_up_sync(0xffffffffu, v.sum, off)};
+}
+
+// Scene changes (signal SCD) of the m <= 4 kScanThreads frames of one tile:
+// twin comparison of the adjacent differences SD_t = L1[t][lag 1] / 2N. A cut
+// (SD >= T_b) and a low difference (SD < T_s) end the run; a middle
+// difference adds to it; a gradual transition is found where the run's sum
+// first reaches T_b. The run sums are a block-wide segmented prefix sum
+// (thread: 4 consecutive frames; warps and the block by shuffles and shared
+// memory) entered with the sum carry_in open before the tile. A scene-change
+// frame gets every keep bit of its mask row and its bit in sflag. Returns the
+// sum open after the tile (the same in every thread).
+__device__ __forceinline__ unsigned long long scd_tile(const uint32_t* __restrict__ l1, uint64_t row_first,
+                                                       uint32_t m, const SelectArgs& a, uint32_t* smask,
+                                                       uint32_t* sflag, unsigned long long carry_in) {
+  __shared__ uint32_t wreset[kScanWarps + 1];
+  __shared__ unsigned long long wsum[kScanWarps + 1];
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t W = a.mask_words, L = a.l_max;
+  uint32_t adj[4], cls[4];  // cls: 2 cut, 1 middle, 0 low (or past the tile)
+  RunSum loc[4];
+  RunSum acc{0u, 0ull};
+#pragma unroll
+  for (uint32_t k = 0; k < 4; ++k) {
+    const uint32_t f = 4 * tid + k;
+    adj[k] = f < m ? l1[(row_first + f) * L] : 0u;
+    const float sd = __fdiv_rn(static_cast<float>(adj[k]), a.two_n);
+    cls[k] = f >= m ? 0u : (sd >= a.scd_cut ? 2u : (sd >= a.scd_grad ? 1u : 0u));
+    const RunSum e = f >= m ? RunSum{0u, 0ull}                                    // past the tile: identity
+                            : (cls[k] == 1u ? RunSum{0u, adj[k]} : RunSum{1u, 0ull});  // joins / ends the run
+    acc = run_cat(acc, e);
+    loc[k] = acc;
+  }
+  RunSum incl = acc;  // inclusive over this warp's threads
+#pragma unroll
+  for (uint32_t off = 1; off < 32; off <<= 1) {
+    const RunSum o = run_shfl_up(incl, off);
+    if (lane >= off) incl = run_cat(o, incl);
+  }
+  if (lane == 31) {
+    wreset[warp] = incl.reset;
+    wsum[warp] = incl.sum;
+  }
+  __syncthreads();
+  if (warp == 0) {  // exclusive scan of the warp totals; slot kScanWarps = the whole tile
+    RunSum w{wreset[lane], wsum[lane]};
+#pragma unroll
+    for (uint32_t off = 1; off < 32; off <<= 1) {
+      const RunSum o = run_shfl_up(w, off);
+      if (lane >= off) w = run_cat(o, w);
+    }
+    const RunSum before = run_shfl_up(w, 1);
+    __syncwarp();
+    wreset[lane] = lane ? before.reset : 0u;
+    wsum[lane] = lane ? before.sum : 0ull;
+    if (lane == 31) {
+      wreset[kScanWarps] = w.reset;
+      wsum[kScanWarps] = w.sum;
+    }
+  }
+  __syncthreads();
+  RunSum ex = run_shfl_up(incl, 1);
+  if (lane == 0) ex = RunSum{0u, 0ull};
+  ex = run_cat(RunSum{wreset[warp], wsum[warp]}, ex);  // everything before this thread's frames
+  const auto reaches = [&](unsigned long long x) { return __fdiv_rn(__ull2float_rn(x), a.two_n) >= a.scd_cut; };
+#pragma unroll
+  for (uint32_t k = 0; k < 4; ++k) {
+    const uint32_t f = 4 * tid + k;
+    if (f >= m) break;
+    const RunSum pre = run_cat(ex, loc[k]);
+    const unsigned long long run = pre.reset ? pre.sum : carry_in + pre.sum;  // the run's sum at f
+    const bool scene = cls[k] == 2u || (cls[k] == 1u && reaches(run) && !reaches(run - adj[k]));
+    if (scene) {
+      for (uint32_t w = 0; w < W; ++w) smask[f * W + w] = 0xffffffffu;
+      atomicOr(&sflag[f >> 5], 1u << (f & 31));
+    }
+  }
+  return wreset[kScanWarps] ? wsum[kScanWarps] : carry_in + wsum[kScanWarps];
+}
+
 // K3's work for one stream segment, done by a whole 1024-thread CTA. sseg,
-// t0 and g0 are the segment and its stream's state on entry (shared memory).
+// t0, g0 and acc0 are the segment and its stream's state on entry (shared
+// memory).
 template <bool kOneWord>
 __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long long t0, uint32_t g0,
-                                             const SelectArgs& a, const uint32_t* __restrict__ l1,
+                                             unsigned long long acc0, const SelectArgs& a, const uint32_t* __restrict__ l1,
                                              const uint32_t* __restrict__ mask, uint32_t* __restrict__ hist,
                                              uint32_t* __restrict__ ring, StreamState* __restrict__ state,
                                              uint32_t* ssm, uint32_t* entry) {
@@ -128,13 +222,21 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
   if (n == 0) return;
   const uint32_t j_start = (t0 == 0) ? 1u : 0u;  // the stream's first frame is decided below
   uint32_t g_entry = (t0 == 0) ? 1u : g0;
+  unsigned long long acc = (t0 == 0) ? 0ull : acc0;  // the scene-change run open before the segment
+  __shared__ uint32_t sflag[kScanTile / 32];
   if (g_entry < 1u || g_entry > L) g_entry = L;  // the state only ever holds [1, L]
 
   for (uint32_t tile0 = j_start; tile0 < n; tile0 += kScanTile) {
     const uint32_t m = min(kScanTile, n - tile0);
     for (uint32_t i = tid; i < m * W; i += kScanThreads)
       smask[i] = mask[static_cast<uint64_t>(row0 + tile0) * W + i];
+    if (a.scd)
+      for (uint32_t i = tid; i < kScanTile / 32; i += kScanThreads) sflag[i] = 0;
     __syncthreads();
+    if (a.scd) {
+      acc = scd_tile(l1, static_cast<uint64_t>(row0 + tile0), m, a, smask, sflag, acc);
+      __syncthreads();
+    }
     const uint32_t run = (m + kScanWarps - 1) / kScanWarps;
     const uint32_t f0 = min(warp * run, m), f1 = min(f0 + run, m);
     // compose this warp's run of gap maps for every entry gap
@@ -171,7 +273,8 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
       const uint32_t lm = max(l1[r], l1[r + g - 1]);
       const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
       const bool nov = s >= a.tau;
-      const uint8_t code = nov ? 1 : (g >= L ? 2 : 0);
+      const bool scene = a.scd && ((sflag[f >> 5] >> (f & 31)) & 1u);
+      const uint8_t code = nov ? 1 : (scene ? 4 : (g >= L ? 2 : 0));
       if (sseg.scores) sseg.scores[jj] = s;
       if (sseg.keep) sseg.keep[jj] = code;
     }
@@ -186,6 +289,7 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
     }
     state[stream].t = t0 + n;
     state[stream].g = g_entry;
+    state[stream].acc = acc;
   }
   // ring: histograms of the last min(n, L) frames of the push
   const uint32_t keep_n = min(n, L);
@@ -210,15 +314,16 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
   extern __shared__ __align__(16) uint32_t ssm[];
   __shared__ Segment sseg;
   __shared__ uint32_t entry[kScanWarps + 1];
-  __shared__ unsigned long long s_t0;
+  __shared__ unsigned long long s_t0, s_acc;
   __shared__ uint32_t s_g;
   if (threadIdx.x == 0) {
     sseg = segs.s[blockIdx.x];
     s_t0 = state[sseg.stream].t;
     s_g = state[sseg.stream].g;
+    s_acc = state[sseg.stream].acc;
   }
   __syncthreads();
-  scan_segment<kOneWord>(sseg, s_t0, s_g, a, l1, mask, hist, ring, state, ssm, entry);
+  scan_segment<kOneWord>(sseg, s_t0, s_g, s_acc, a, l1, mask, hist, ring, state, ssm, entry);
 }
 
 // Small pushes: one CTA per stream segment computes the segment's windowed
@@ -233,19 +338,20 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
   extern __shared__ __align__(16) uint32_t ssm[];
   __shared__ Segment sseg;
   __shared__ uint32_t entry[kScanWarps + 1];
-  __shared__ unsigned long long s_t0;
+  __shared__ unsigned long long s_t0, s_acc;
   __shared__ uint32_t s_g;
   if (threadIdx.x == 0) {
     sseg = segs.s[blockIdx.x];
     s_t0 = state[sseg.stream].t;
     s_g = state[sseg.stream].g;
+    s_acc = state[sseg.stream].acc;
   }
   __syncthreads();
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (uint32_t j = warp; j < sseg.n; j += kScanWarps)
     window_row<kVec4>(sseg.row0 + j, lane, sseg, a, hist, ring, s_t0, l1, mask);
   __syncthreads();  // this CTA's distance and mask rows are visible to all its threads
-  scan_segment<kOneWord>(sseg, s_t0, s_g, a, l1, mask, hist, ring, state, ssm, entry);
+  scan_segment<kOneWord>(sseg, s_t0, s_g, s_acc, a, l1, mask, hist, ring, state, ssm, entry);
 }
 
 // The gap map of one stream segment: map[g-1] = the gap after its last frame

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(lib):
 def test_param_struct_layout_matches_header(lib):
     from paper_2609_03675_gb300 import _abi
     # width..luma_den: 10 x 4 bytes, max_streams, max_frames_per_push, device, pad, u64, signal, reserved
-    assert ctypes.sizeof(_abi.Params) == 72
+    assert ctypes.sizeof(_abi.Params) == 80
     assert ctypes.sizeof(_abi.PushDesc) == 32
 
 
@@ -79,7 +79,7 @@ def test_null_handle_calls_are_rejected(lib):
 
 
 @pytest.mark.parametrize("width,height,signal,msg", [
-    (64, 48, 3, "signal"), (15, 48, 1, "low-res"), (64, 15, 1, "low-res"), (4097, 4097, 1, "low-res"),
+    (64, 48, 4, "signal"), (15, 48, 1, "low-res"), (64, 15, 1, "low-res"), (4097, 4097, 1, "low-res"),
     (8, 48, 2, "dHash"), (64, 7, 2, "dHash"), (46341, 46340, 2, "too large"),
 ])
 def test_create_rejects_bad_signal_shapes(lib, width, height, signal, msg):
@@ -91,3 +91,16 @@ def test_create_rejects_bad_signal_shapes(lib, width, height, signal, msg):
     assert lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h)) == _abi.EINVAL
     assert msg in lib.cofie_ngff_global_error().decode()
     assert not h.value
+
+
+@pytest.mark.parametrize("field", ["scd_cut", "scd_gradual"])
+def test_create_rejects_nan_scene_thresholds(lib, field):
+    from paper_2609_03675_gb300 import _abi
+    p = _abi.Params()
+    lib.cofie_ngff_default_params(ctypes.byref(p), 64, 48)
+    assert (p.scd_cut, p.scd_gradual) == (pytest.approx(0.30), pytest.approx(0.10))
+    p.signal = _abi.SIGNAL_SCD
+    setattr(p, field, float("nan"))
+    h = ctypes.c_void_p()
+    assert lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h)) == _abi.EINVAL
+    assert "NaN" in lib.cofie_ngff_global_error().decode()
