@@ -293,6 +293,29 @@ int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream);
 int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_out);
 
 /*
+ * Test hooks for the failure paths (no counterpart in the paper). Neither
+ * faults, traps or hangs a GPU.
+ *   cofie_ngff_debug_fail_alloc  after >= 0: that many further device
+ *                                allocations of the library succeed and the
+ *                                next one fails (cofie_ngff_create then returns
+ *                                COFIE_ENOMEM and frees what it had taken; a
+ *                                push from host memory whose staging buffer
+ *                                fails returns COFIE_ENOMEM); the hook then
+ *                                switches itself off. after < 0 switches it off.
+ *                                Process-wide, not thread-safe against creates.
+ *   cofie_ngff_debug_wait        enqueues a one-thread kernel that waits, with
+ *                                the streaming kernel's bounded mbarrier wait,
+ *                                for a phase nothing completes; after
+ *                                timeout_ns (<= 1 s, else COFIE_EINVAL) it sets
+ *                                the same error bit a stalled consumer sets and
+ *                                returns, so cofie_ngff_status then reports
+ *                                COFIE_ETIMEOUT and clears it; the context and
+ *                                the handle stay usable.
+ */
+void cofie_ngff_debug_fail_alloc(int32_t after);
+int cofie_ngff_debug_wait(cofie_ngff_t* h, uint64_t timeout_ns, void* cuda_stream);
+
+/*
  * Diagnostic: applies the fast histogram kernel's own per-pixel grayscale and
  * bin functions to n_pixels RGB triples (device memory, 3 * n_pixels bytes,
  * n_pixels a multiple of 4) and writes one bin index per pixel to bins_out

@@ -211,6 +211,11 @@ class NGFF:
         self._check(self._lib.cofie_ngff_debug_bins(self._h, _ptr(pixels), n, _ptr(out), self._stream(cuda_stream)))
         return out
 
+    def debug_wait(self, timeout_ns: int, cuda_stream=None):
+        """Enqueues the bounded-wait probe (a wait nothing completes); status()
+        then raises NGFFError with code ETIMEOUT."""
+        self._check(self._lib.cofie_ngff_debug_wait(self._h, int(timeout_ns), self._stream(cuda_stream)))
+
     def profile_reset(self, time_kernels: bool = False):
         """Zeroes the launch counters; with time_kernels every histogram-kernel
         launch is bracketed by CUDA events on its stream."""

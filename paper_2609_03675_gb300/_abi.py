@@ -37,6 +37,8 @@ EXPORTS = (
     "cofie_ngff_status",
     "cofie_ngff_frames_seen",
     "cofie_ngff_debug_bins",
+    "cofie_ngff_debug_fail_alloc",
+    "cofie_ngff_debug_wait",
     "cofie_ngff_profile_reset",
     "cofie_ngff_profile_read",
     "cofie_ngff_select_static",
@@ -165,6 +167,10 @@ def load():
     lib.cofie_ngff_frames_seen.restype = ctypes.c_int
     lib.cofie_ngff_debug_bins.argtypes = [H, vp, u64, vp, vp]
     lib.cofie_ngff_debug_bins.restype = ctypes.c_int
+    lib.cofie_ngff_debug_fail_alloc.argtypes = [ctypes.c_int32]
+    lib.cofie_ngff_debug_fail_alloc.restype = None
+    lib.cofie_ngff_debug_wait.argtypes = [H, u64, vp]
+    lib.cofie_ngff_debug_wait.restype = ctypes.c_int
     lib.cofie_ngff_profile_reset.argtypes = [H, ctypes.c_int]
     lib.cofie_ngff_profile_reset.restype = ctypes.c_int
     lib.cofie_ngff_profile_read.argtypes = [H, ctypes.POINTER(Profile)]

@@ -21,6 +21,10 @@
 
 using namespace cofie;
 
+namespace cofie {
+std::atomic<int> g_fail_alloc{-1};
+}
+
 namespace {
 
 thread_local std::string g_global_error;
@@ -177,6 +181,7 @@ int validate_params(const cofie_ngff_params* p, std::string& why) {
 
 template <typename T>
 cudaError_t dalloc(T** p, size_t count) {
+  if (injected_alloc_failure()) return cudaErrorMemoryAllocation;
   return cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) + 16);
 }
 
@@ -338,7 +343,8 @@ int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n
 int ensure_staging(cofie_ngff* h) {
   if (h->d_stage[0]) return COFIE_OK;
   for (int i = 0; i < 2; ++i) {
-    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&h->d_stage[i]), h->stage_bytes);
+    cudaError_t e = injected_alloc_failure() ? cudaErrorMemoryAllocation
+                                             : cudaMalloc(reinterpret_cast<void**>(&h->d_stage[i]), h->stage_bytes);
     if (e != cudaSuccess) {
       cudaGetLastError();
       for (int j = 0; j < 2; ++j) {
@@ -353,6 +359,7 @@ int ensure_staging(cofie_ngff* h) {
 
 int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n, float* scores, uint8_t* keep,
               uint32_t* hist_out, void* cuda_stream) {
+  NvtxRange nvtx("ngff.push");
   if (!h) return COFIE_EINVAL;
   if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
   if (n == 0) return COFIE_OK;
@@ -623,6 +630,7 @@ int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, 
 }
 
 int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream) {
+  NvtxRange nvtx("ngff.push_batch");
   if (!h) return COFIE_EINVAL;
   if (nd == 0) return COFIE_OK;
   if (!desc) return h->fail(COFIE_EINVAL, "desc is NULL");
@@ -684,6 +692,7 @@ size_t cofie_ngff_state_bytes(const cofie_ngff_t* h) {
 }
 
 int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream) {
+  NvtxRange nvtx("ngff.state_save");
   if (!h) return COFIE_EINVAL;
   if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
   if (!buf) return h->fail(COFIE_EINVAL, "buf is NULL");
@@ -720,6 +729,7 @@ int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cud
 }
 
 int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, void* cuda_stream) {
+  NvtxRange nvtx("ngff.state_load");
   if (!h) return COFIE_EINVAL;
   if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
   if (!buf) return h->fail(COFIE_EINVAL, "buf is NULL");
@@ -750,6 +760,7 @@ int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, voi
 
 int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n_halo, uint32_t n,
                              uint64_t t0, uint16_t* map_out, void* cuda_stream) {
+  NvtxRange nvtx("ngff.shard_prepare");
   if (!h) return COFIE_EINVAL;
   if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
   if (!frames || !map_out || n == 0) return h->fail(COFIE_EINVAL, "frames and map_out are required, n >= 1");
@@ -814,6 +825,7 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
 
 int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap, float* scores_out, uint8_t* keep_out,
                             void* cuda_stream) {
+  NvtxRange nvtx("ngff.shard_commit");
   if (!h) return COFIE_EINVAL;
   if (!h->shard.ready || h->shard.stream != stream)
     return h->fail(COFIE_EINVAL, "no shard of this stream is prepared on this handle");
@@ -889,6 +901,16 @@ int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_o
   return COFIE_OK;
 }
 
+void cofie_ngff_debug_fail_alloc(int32_t after) { g_fail_alloc.store(after < 0 ? -1 : after); }
+
+int cofie_ngff_debug_wait(cofie_ngff_t* h, uint64_t timeout_ns, void* cuda_stream) {
+  if (!h) return COFIE_EINVAL;
+  if (timeout_ns > 1000000000ull) return h->fail(COFIE_EINVAL, "timeout_ns must be at most 1 s");
+  DeviceGuard guard(h->device);
+  const cudaError_t e = launch_wait_probe(timeout_ns, h->d_err, static_cast<cudaStream_t>(cuda_stream));
+  return e == cudaSuccess ? COFIE_OK : h->cuda_fail(e, "wait probe launch");
+}
+
 int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pixels, uint8_t* bins_out,
                           void* cuda_stream) {
   if (!h) return COFIE_EINVAL;
@@ -906,6 +928,7 @@ int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pix
 
 int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out, uint32_t* m_out,
                           void* cuda_stream) {
+  NvtxRange nvtx("ngff.candidates");
   if (!h) return COFIE_EINVAL;
   if (!m_out) return h->fail(COFIE_EINVAL, "m_out is NULL");
   DeviceGuard guard(h->device);
@@ -936,6 +959,7 @@ int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint
 
 int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames, const uint32_t* idx, uint32_t m,
                       uint8_t* out, void* cuda_stream) {
+  NvtxRange nvtx("ngff.gather");
   if (!h) return COFIE_EINVAL;
   if (m == 0) return COFIE_OK;
   int d0 = -1, d1 = -1, d2 = -1;

@@ -11,8 +11,10 @@
 //   state    StreamState [streams]    frames seen and current gap
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 namespace cofie {
 
@@ -105,6 +107,25 @@ struct FeatArgs {
   uint32_t row_h[16], col_w[16];  // pixels per cell row / cell column
 };
 
+// An NVTX range over one C-ABI call (a no-op unless a profiler is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
+// Host-side fault injection for tests: when >= 0, that many further device
+// allocations of the library succeed and the next one fails (then the hook
+// switches itself off). Set through cofie_ngff_debug_fail_alloc.
+extern std::atomic<int> g_fail_alloc;
+inline bool injected_alloc_failure() {
+  int left = g_fail_alloc.load();
+  while (left >= 0 && !g_fail_alloc.compare_exchange_weak(left, left - 1)) {
+  }
+  return left == 0;
+}
+
 // Launchers (stream-ordered; return the launch error).
 int hist_blocks_per_sm(int bin_path, uint32_t bins);
 uint32_t hist_chunk_groups();
@@ -126,6 +147,7 @@ int cells_blocks_per_sm();
 cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* cells,
                               uint32_t* err, int grid, cudaStream_t st);
 cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st);
+cudaError_t launch_wait_probe(uint64_t timeout_ns, uint32_t* err, cudaStream_t st);
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);

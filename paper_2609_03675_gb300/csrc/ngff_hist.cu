@@ -517,6 +517,18 @@ __global__ void __launch_bounds__(96) dhash_finish_kernel(uint32_t* __restrict__
   if (tid < 72) c[tid] = 0;
 }
 
+// Failure-path probe: one thread waits, with the pipeline's bounded wait, for
+// an mbarrier phase that nothing completes; when the bound runs out it sets
+// the consumer-timeout bit, exactly as a stalled K1 consumer would, and the
+// kernel returns normally.
+__global__ void wait_probe_kernel(uint64_t timeout_ns, uint32_t* __restrict__ err) {
+  __shared__ __align__(8) uint64_t bar;
+  const uint32_t b = smem_u32(&bar);
+  mbar_init(b, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  if (!mbar_wait_bounded(b, 0, timeout_ns)) atomicOr(err, kErrConsumerTimeout);
+}
+
 // Diagnostic: the fast kernel's per-pixel luma and bin functions applied to
 // 4-pixel groups (12 bytes each), one bin index per pixel.
 template <int kBin>
@@ -614,6 +626,11 @@ cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const L
 cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const LumaConsts& lc, uint32_t* feat, uint32_t fw,
                             cudaStream_t st) {
   features_kernel<<<segs.rows, kFeatThreads, 0, st>>>(segs, fa, lc, feat, fw);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_probe(uint64_t timeout_ns, uint32_t* err, cudaStream_t st) {
+  wait_probe_kernel<<<1, 1, 0, st>>>(timeout_ns, err);
   return cudaGetLastError();
 }
 
