@@ -26,7 +26,8 @@
  *      the most recent retained frame before t; s = max(s_adj, s_ref) (Eq. 4).
  *   5. Retention (Eq. 5 and the safeguards before it): the first frame is
  *      always retained; frame t > 0 is retained when s >= tau_h or
- *      t - r(t) >= L_max. The keep decision is taken in fp32, the precision
+ *      t - r(t) >= L_max (L_max = 0, a value the paper does not use, is read
+ *      as no forced retention). The keep decision is taken in fp32, the precision
  *      the GPU library decides in: d32 = fp32(sum_b |c_i[b] - c_j[b]|) /
  *      fp32(2N), one correctly rounded fp32 division.
  *   6. Finalisation (safeguards of Sec. 3.2): add the last frame T-1; if
@@ -49,7 +50,7 @@
 typedef struct {
   uint32_t width, height;
   uint32_t bins;       /* B */
-  uint32_t l_max;      /* L_max, >= 1 */
+  uint32_t l_max;      /* L_max; 0 turns the forced-retention term of Eq. 5 off */
   uint32_t m_min;      /* M_min */
   float tau;           /* tau_h */
   uint32_t luma_w[3];  /* wR, wG, wB */
@@ -61,7 +62,6 @@ enum { KEEP_DROP = 0, KEEP_NOVELTY = 1, KEEP_GAP = 2, KEEP_FIRST = 3 };
 static int params_ok(const ngff_oracle_params* p) {
   if (!p || p->width == 0 || p->height == 0) return 0;
   if (p->bins < 1 || p->bins > 256) return 0;
-  if (p->l_max < 1) return 0;
   if (p->luma_den == 0 || p->luma_w[0] + p->luma_w[1] + p->luma_w[2] != p->luma_den) return 0;
   if (p->tau != p->tau) return 0; /* NaN */
   return 1;
@@ -139,7 +139,7 @@ int ngff_oracle_select(const uint32_t* hist, uint32_t T, const ngff_oracle_param
       float d_ref = ngff_oracle_tv32(ht, hist + (size_t)r * B, B, N);
       float s32 = d_adj > d_ref ? d_adj : d_ref;
       int novelty = s32 >= p->tau;                                         /* Eq. 5 */
-      int gap = (t - r) >= p->l_max;                                       /* Eq. 5 */
+      int gap = p->l_max > 0 && (t - r) >= p->l_max;                       /* Eq. 5 */
       keep = novelty ? KEEP_NOVELTY : (gap ? KEEP_GAP : KEEP_DROP);
     }
     if (keep != KEEP_DROP) r = t;

@@ -87,7 +87,7 @@ def select(hist: np.ndarray, p: O.Params, t_cut: float, t_grad: float):
             keep[t] = O.KEEP_NOVELTY
         elif scene[t]:
             keep[t] = KEEP_SCENE
-        elif t - r >= p.l_max:
+        elif p.l_max > 0 and t - r >= p.l_max:
             keep[t] = O.KEEP_GAP
         if keep[t]:
             r = t

@@ -80,7 +80,7 @@ def select(feats: np.ndarray, p: O.Params, kind: int):
         score[t] = max(na, nr) / den
         s32 = np.float32(max(na, nr)) / np.float32(den)
         nov = s32 >= np.float32(p.tau)
-        gap = (t - r) >= p.l_max
+        gap = p.l_max > 0 and (t - r) >= p.l_max
         keep[t] = O.KEEP_NOVELTY if nov else (O.KEEP_GAP if gap else O.KEEP_DROP)
         if keep[t]:
             r = t

@@ -209,10 +209,17 @@ def pin_rule_thresholds(o):
             assert np.array_equal(kept, np.arange(0, T, L)), "tau > 1 keeps exactly 0, L, 2L, ..."
             assert (keep[kept[1:]] == O.KEEP_GAP).all()
             assert ((score >= 0) & (score <= 1)).all()
+        # L_max = 0 turns the forced retention off: with tau > 1 only the first frame is kept
+        _, keep = o.select(hist, O.Params(10, 10, bins=B, l_max=0, tau=1.5))
+        assert np.array_equal(np.flatnonzero(keep), [0])
+        _, keep = o.select(hist, O.Params(10, 10, bins=B, l_max=0, tau=0.0))
+        assert (keep[1:] == O.KEEP_NOVELTY).all()
     # a constant stream scores zero everywhere
     hist = np.tile(np.array([[100, 0, 0, 0]], dtype=np.uint32), (40, 1))
     score, keep = o.select(hist, O.Params(10, 10, bins=4, l_max=7, tau=0.1))
     assert (score == 0).all() and np.array_equal(np.flatnonzero(keep), np.arange(0, 40, 7))
+    _, keep = o.select(hist, O.Params(10, 10, bins=4, l_max=0, tau=0.1))
+    assert np.array_equal(np.flatnonzero(keep), [0]), "no forced retention: a constant stream keeps its first frame"
 
 
 def pin_rule_terms(o):
@@ -276,7 +283,7 @@ def _bruteforce_mask(hist, N, tau, L):
             r = max(u for u in range(t) if mask[u])
             d_adj = np.float32(np.abs(hist[t] - hist[t - 1]).sum()) / two_n
             d_ref = np.float32(np.abs(hist[t] - hist[r]).sum()) / two_n
-            rule = (max(d_adj, d_ref) >= tau32) or (t - r >= L)
+            rule = (max(d_adj, d_ref) >= tau32) or (L > 0 and t - r >= L)
             ok = mask[t] == int(rule)
         if ok:
             sols.append(mask)
@@ -301,7 +308,7 @@ def pin_bruteforce_4x8x8(o):
                 frames.append(g.integers(0, 256, size=(8, 8, 3), dtype=np.uint8))
         frames = np.stack(frames)
         tau = float(g.choice([0.05, 0.1, 0.2, 0.3, 0.5]))
-        L = int(g.integers(1, 5))
+        L = int(g.integers(0, 5))  # 0: no forced retention
         p = O.Params(8, 8, bins=B, l_max=L, tau=tau)
         hist_np = np.stack([np_hist(f, B) for f in frames])
         h, _, keep = o.run(frames, p)

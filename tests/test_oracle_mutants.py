@@ -35,8 +35,10 @@ MUTANTS = {
     "min_not_max": ("float s32 = d_adj > d_ref ? d_adj : d_ref;", "float s32 = d_adj < d_ref ? d_adj : d_ref;"),
     "score_min_not_max": ("score = s_adj > s_ref ? s_adj : s_ref;", "score = s_adj < s_ref ? s_adj : s_ref;"),
     "strict_tau": ("int novelty = s32 >= p->tau;", "int novelty = s32 > p->tau;"),
-    "strict_gap": ("int gap = (t - r) >= p->l_max;", "int gap = (t - r) > p->l_max;"),
-    "gap_off_by_one": ("int gap = (t - r) >= p->l_max;", "int gap = (t - r) >= p->l_max + 1;"),
+    "strict_gap": ("int gap = p->l_max > 0 && (t - r) >= p->l_max;", "int gap = p->l_max > 0 && (t - r) > p->l_max;"),
+    "gap_off_by_one": ("int gap = p->l_max > 0 && (t - r) >= p->l_max;",
+                       "int gap = p->l_max > 0 && (t - r) >= p->l_max + 1;"),
+    "gap_rule_with_zero_l_max": ("int gap = p->l_max > 0 && (t - r) >= p->l_max;", "int gap = (t - r) >= p->l_max;"),
     "r_not_moved_by_gap": ("if (keep != KEEP_DROP) r = t;", "if (keep == KEEP_NOVELTY || keep == KEEP_FIRST) r = t;"),
     "first_not_kept": ("keep = KEEP_FIRST; /* the first", "keep = KEEP_DROP; /* the first"),
     "gap_code_wins": ("keep = novelty ? KEEP_NOVELTY : (gap ? KEEP_GAP : KEEP_DROP);",

@@ -20,9 +20,9 @@ MUTANTS = {
         "        if scene[t]:\n            keep[t] = KEEP_SCENE\n"
         "        elif at_least(max(na, nr), two_n, p.tau):\n            keep[t] = O.KEEP_NOVELTY\n"),
     "gap before scene change": (
-        "        elif scene[t]:\n            keep[t] = KEEP_SCENE\n        elif t - r >= p.l_max:\n"
+        "        elif scene[t]:\n            keep[t] = KEEP_SCENE\n        elif p.l_max > 0 and t - r >= p.l_max:\n"
         "            keep[t] = O.KEEP_GAP\n",
-        "        elif t - r >= p.l_max:\n            keep[t] = O.KEEP_GAP\n        elif scene[t]:\n"
+        "        elif p.l_max > 0 and t - r >= p.l_max:\n            keep[t] = O.KEEP_GAP\n        elif scene[t]:\n"
         "            keep[t] = KEEP_SCENE\n"),
     "scene keeps do not move r": ("        if keep[t]:\n            r = t\n",
                                   "        if keep[t] and keep[t] != KEEP_SCENE:\n            r = t\n"),

@@ -66,6 +66,8 @@ def test_rule_special_cases(kind):
         assert keep[0] == O.KEEP_FIRST and (keep[1:] == O.KEEP_NOVELTY).all()
         _, _, keep = SO.run(frames, O.Params(W, H, l_max=L, tau=1.5), kind)
         assert list(np.flatnonzero(keep)) == list(range(0, T, L))
+    _, _, keep = SO.run(frames, O.Params(W, H, l_max=0, tau=1.5), kind)
+    assert list(np.flatnonzero(keep)) == [0], "L_max = 0: no forced retention"
     f, s, k = SO.run(frames, O.Params(W, H, tau=0.2), kind)
     for cut in (1, 9, 25):
         f2, s2, k2 = SO.run(frames[:cut], O.Params(W, H, tau=0.2), kind)
