@@ -51,6 +51,8 @@ def parse():
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
     ap.add_argument("--qer-frames", type=int, default=128, help="candidate frames of the qer workload")
+    ap.add_argument("--l-max", type=int, default=30,
+                    help="L_max of the hd1080 workload (0: no forced retention, the rule walked in frame order)")
     ap.add_argument("--signal", choices=["histogram", "lowres", "dhash", "scd"], default="histogram",
                     help="NGFF's novelty signal for the hd1080 workload (histogram is the paper's)")
     ap.add_argument("--frames", type=int, default=3600,
@@ -160,7 +162,7 @@ class ClockSampler:
 SIGNALS = {"histogram": 0, "lowres": 1, "dhash": 2, "scd": 3}
 
 
-def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0):
+def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0, l_max: int = 30):
     """The oracle as it stands (single-threaded C for the histogram, numpy for
     the spatial signals) on the first k frames of the stream; k sized to about
     target_s seconds of CPU work."""
@@ -172,7 +174,7 @@ def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0):
     from oracle import scd_oracle as SC
     from oracle import signals_oracle as SO
     o = O.load()
-    p = O.Params(spec.width, spec.height)
+    p = O.Params(spec.width, spec.height, l_max=l_max)
     fb = spec.frame_bytes
 
     def run(k):
@@ -214,7 +216,7 @@ def bench_gb300(args):
     scores = torch.empty(T, dtype=torch.float32, device="cuda")
     keep = torch.empty(T, dtype=torch.uint8, device="cuda")
     signal = SIGNALS[args.signal]
-    f = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=signal)
+    f = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=signal, l_max=args.l_max)
     stream = torch.cuda.current_stream()
 
     def step():
@@ -265,7 +267,7 @@ def bench_gb300(args):
     if not args.no_e2e:
         hs = torch.empty(T, dtype=torch.float32, pin_memory=True)
         hk = torch.empty(T, dtype=torch.uint8, pin_memory=True)
-        fe = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=signal)
+        fe = NGFF(spec.width, spec.height, max_frames_per_push=T, signal=signal, l_max=args.l_max)
 
         def estep():
             fe.reset()
@@ -309,7 +311,7 @@ def bench_gb300(args):
 
     cpu = None
     if rank == 0 and world == 1 and args.cpu_seconds > 0:
-        k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds, signal)
+        k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds, signal, args.l_max)
         what = {0: "single-threaded C oracle (histograms + selection)",
                 3: "C oracle histograms + the scene-change oracle's rule (Python)"}.get(
             signal, f"numpy signals oracle ({args.signal} features + selection)")
@@ -322,9 +324,10 @@ def bench_gb300(args):
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u8", "data": "synthetic",
             "config": {"workload": f"1080p stream: {T} uint8 RGB frames of 1920x1080 (HWC), one whole-stream push "
-                                   "per step, B=32, L_max=30, tau_h=0.30"
+                                   f"per step, B=32, L_max={args.l_max}, tau_h=0.30"
                                    + ("" if signal == 0 else f", signal {args.signal} in place of the histogram"),
-                       "signal": args.signal, "frames_per_step": T, "width": spec.width, "height": spec.height, "bins": 32, "l_max": 30,
+                       "signal": args.signal, "frames_per_step": T, "width": spec.width, "height": spec.height,
+                       "bins": 32, "l_max": args.l_max,
                        "tau": 0.30, "l2": f"inputs larger than L2 ({T * spec.frame_bytes / 1e9:.1f} GB per step), no flush",
                        "parallelism": f"{world} independent stream(s), one per GPU"},
             "pixel_gbs": pixel_gbs,

@@ -81,7 +81,11 @@ typedef struct cofie_ngff cofie_ngff_t;
  * Parameters of a handle. Fill with cofie_ngff_default_params() and override.
  *   width, height     frame size in pixels, >= 1 each.
  *   bins              B, 1..256; default 32 (App. A).
- *   l_max             L_max in sampled-frame indices, 1..256; default 30 (App. B.2).
+ *   l_max             L_max in sampled-frame indices, 0..256; default 30 (App. B.2).
+ *                     0 turns the forced retention (Eq. 5's second term) off:
+ *                     frames are then kept only as first, novelty or scene
+ *                     change, the rule is walked in frame order by one warp
+ *                     per stream, and the stream cannot be sharded.
  *   m_min             M_min, used by cofie_ngff_candidates only; default 4 (App. B.2).
  *   tau               tau_h, any non-NaN float; default 0.30f (App. B.2).
  *   luma_w, luma_den  grayscale weights (wR, wG, wB) / den; each weight <= 65535,

@@ -18,7 +18,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(REPO, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcofie_ngff.so")
-SOURCES = ["ngff_api.cu", "ngff_hist.cu", "ngff_select.cu", "ngff_finalize.cu", "ngff_static.cu", "qer.cu"]
+SOURCES = ["ngff_api.cu", "ngff_hist.cu", "ngff_select.cu", "ngff_lazy.cu", "ngff_finalize.cu", "ngff_static.cu",
+           "qer.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -159,7 +159,7 @@ int validate_params(const cofie_ngff_params* p, std::string& why) {
   const uint64_t npix = static_cast<uint64_t>(p->width) * p->height;
   if (npix > 0x7fffffffull) return why = "width * height must be < 2^31", COFIE_EINVAL;
   if (p->bins < 1 || p->bins > COFIE_NGFF_MAX_BINS) return why = "bins must be in [1, 256]", COFIE_EINVAL;
-  if (p->l_max < 1 || p->l_max > COFIE_NGFF_MAX_LMAX) return why = "l_max must be in [1, 256]", COFIE_EINVAL;
+  if (p->l_max > COFIE_NGFF_MAX_LMAX) return why = "l_max must be in [0, 256]", COFIE_EINVAL;
   if (p->tau != p->tau) return why = "tau is NaN", COFIE_EINVAL;
   if (p->luma_den == 0 || p->luma_den > 65535) return why = "luma_den must be in [1, 65535]", COFIE_EINVAL;
   if (static_cast<uint64_t>(p->luma_w[0]) + p->luma_w[1] + p->luma_w[2] != p->luma_den)
@@ -254,6 +254,10 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
   return launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
 }
 
+// Ring rows per stream: the last L_max feature rows, or for L_max = 0 the
+// previous frame's row and the reference frame's row.
+uint32_t ring_rows(const cofie_ngff* h) { return h->p.l_max ? h->p.l_max : 2u; }
+
 SelectArgs select_args(const cofie_ngff* h) {
   SelectArgs sa{};
   sa.bins = h->fw;
@@ -294,10 +298,14 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
   // small pushes clear their rows inside the fused kernel (saving a launch);
   // large ones leave that to one device-wide memset before the next push
   const bool fused = longest <= select_small_max();
-  sa.zero_hist = (fused && !keep_hist) ? 1u : 0u;
+  sa.zero_hist = (fused && !keep_hist && h->p.l_max > 0) ? 1u : 0u;
   cudaEvent_t es0 = nullptr, es1 = nullptr;
   if (h->time_kernels && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
-  if (fused) {  // distances and scan in one launch
+  if (h->p.l_max == 0) {  // no forced retention: the rule walked in frame order
+    e = launch_lazy_select(segs, sa, h->d_hist, h->d_ring, h->d_state, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "lazy selection kernel launch");
+    h->n_select += 1;
+  } else if (fused) {  // distances and scan in one launch
     e = launch_select_small(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
     if (e != cudaSuccess) return h->cuda_fail(e, "selection kernel launch");
     h->n_select += 1;
@@ -557,7 +565,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   if (e == cudaSuccess) e = dalloc(&h->d_hist, F * h->fw);
   if (e == cudaSuccess) e = dalloc(&h->d_l1, F * p->l_max);
   if (e == cudaSuccess) e = dalloc(&h->d_mask, F * h->mask_words);
-  if (e == cudaSuccess) e = dalloc(&h->d_ring, S * p->l_max * h->fw);
+  if (e == cudaSuccess) e = dalloc(&h->d_ring, S * ring_rows(h) * h->fw);
   if (e == cudaSuccess) e = dalloc(&h->d_state, S);
   if (e == cudaSuccess) e = dalloc(&h->d_scores, F);
   if (e == cudaSuccess) e = dalloc(&h->d_keep, F);
@@ -582,7 +590,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     e = cudaEventCreateWithFlags(&h->ev_copied[i], cudaEventDisableTiming);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_free[i], cudaEventDisableTiming);
   }
-  if (e == cudaSuccess) e = scan_prepare(h->mask_words, p->l_max);
+  if (e == cudaSuccess && p->l_max > 0) e = scan_prepare(h->mask_words, p->l_max);
   if (e == cudaSuccess && h->bin_path >= 0) {
     const int per_sm = hist_blocks_per_sm(h->bin_path, p->bins);
     if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
@@ -688,7 +696,7 @@ static_assert(sizeof(StateHeader) == kStateHeader, "state header layout");
 }  // namespace
 
 size_t cofie_ngff_state_bytes(const cofie_ngff_t* h) {
-  return h ? kStateHeader + static_cast<size_t>(h->p.l_max) * h->fw * sizeof(uint32_t) : 0;
+  return h ? kStateHeader + static_cast<size_t>(ring_rows(h)) * h->fw * sizeof(uint32_t) : 0;
 }
 
 int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream) {
@@ -708,8 +716,8 @@ int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cud
   hdr.l_max = h->p.l_max;
   hdr.pad0 = h->p.signal;
   uint8_t* b = static_cast<uint8_t*>(buf);
-  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->fw * sizeof(uint32_t);
-  const uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->fw;
+  const size_t ring_bytes = static_cast<size_t>(ring_rows(h)) * h->fw * sizeof(uint32_t);
+  const uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * ring_rows(h) * h->fw;
   cudaError_t e;
   if (kb == kDevice) {
     // the header's fixed part travels through the handle's pinned-free path: a
@@ -744,11 +752,11 @@ int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, voi
   if (hdr.width != h->p.width || hdr.height != h->p.height || hdr.bins != h->p.bins || hdr.l_max != h->p.l_max ||
       hdr.pad0 != h->p.signal)
     return h->fail(COFIE_EINVAL, "saved state has another width, height, bins, l_max or signal");
-  if (hdr.st.t > 0 && (hdr.st.g < 1 || hdr.st.g > h->p.l_max))
+  if (hdr.st.t > 0 && h->p.l_max > 0 && (hdr.st.g < 1 || hdr.st.g > h->p.l_max))
     return h->fail(COFIE_EINVAL, "saved state has a gap outside [1, l_max]");
   const uint8_t* b = static_cast<const uint8_t*>(buf);
-  const size_t ring_bytes = static_cast<size_t>(h->p.l_max) * h->fw * sizeof(uint32_t);
-  uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * h->p.l_max * h->fw;
+  const size_t ring_bytes = static_cast<size_t>(ring_rows(h)) * h->fw * sizeof(uint32_t);
+  uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * ring_rows(h) * h->fw;
   e = cudaMemcpyAsync(ring, b + kStateHeader, ring_bytes, cudaMemcpyDefault, st);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(h->d_state + stream, b + offsetof(StateHeader, st), sizeof(StreamState), cudaMemcpyDefault, st);
@@ -766,6 +774,8 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   if (!frames || !map_out || n == 0) return h->fail(COFIE_EINVAL, "frames and map_out are required, n >= 1");
   if (h->p.signal == COFIE_SIGNAL_SCD)  // a scene-change run can reach back past any halo
     return h->fail(COFIE_EINVAL, "streams of the scene-change signal cannot be sharded");
+  if (h->p.l_max == 0)  // without forced retention the reference frame can lie any distance back
+    return h->fail(COFIE_EINVAL, "streams with l_max = 0 cannot be sharded");
   const uint64_t want_halo = t0 < h->p.l_max ? t0 : h->p.l_max;
   if (n_halo != want_halo) return h->fail(COFIE_EINVAL, "n_halo must be min(t0, l_max)");
   if (static_cast<uint64_t>(n_halo) + n > h->p.max_frames_per_push)

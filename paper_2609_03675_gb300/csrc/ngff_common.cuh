@@ -8,6 +8,8 @@
 //   mask     uint32 [rows][W_m]       bit g-1 of row t: keep decision of frame t
 //                                     if its gap t - r(t) were g (W_m = ceil(L_max/32))
 //   ring     uint32 [streams][L_max][B]  histogram of frame t at slot t mod L_max
+//                                     (L_max = 0: [streams][2][B], the previous
+//                                     frame's and the reference frame's rows)
 //   state    StreamState [streams]    frames seen and current gap
 #pragma once
 
@@ -148,6 +150,8 @@ cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const Lum
                               uint32_t* err, int grid, cudaStream_t st);
 cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st);
 cudaError_t launch_wait_probe(uint64_t timeout_ns, uint32_t* err, cudaStream_t st);
+cudaError_t launch_lazy_select(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
+                               StreamState* state, cudaStream_t st);
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);

@@ -53,7 +53,7 @@ def test_defaults_are_the_papers(lib):
 
 
 @pytest.mark.parametrize("field,value,msg", [
-    ("width", 0, "width"), ("bins", 0, "bins"), ("bins", 257, "bins"), ("l_max", 0, "l_max"),
+    ("width", 0, "width"), ("bins", 0, "bins"), ("bins", 257, "bins"),
     ("l_max", 257, "l_max"), ("tau", float("nan"), "NaN"), ("luma_den", 999, "sum"), ("max_streams", 0, "streams"),
     ("max_frames_per_push", 0, "max_frames"),
 ])
