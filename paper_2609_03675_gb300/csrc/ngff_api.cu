@@ -64,6 +64,7 @@ struct cofie_ngff {
   bool size_fast = false;
   int hist_grid = 0;
   int cells_grid = 0;    // the TMA kernel's grid for the spatial signals (0: not usable)
+  unsigned long long x_tau = 0, x_cut = 0, x_grad = 0;  // integer forms of the fp32 decisions
   uint32_t m_gpr = 0, m_h = 0, m_gw = 0;  // its multiply-high divisors (16-pixel groups per row, height, grid columns)
   uint32_t* d_cells = nullptr;  // dHash only: [F][72] cell sums, kept zero between pushes
   float two_n = 0.f;
@@ -254,6 +255,23 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
   return launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
 }
 
+// The smallest numerator x with fp32(x) / den >= thr, or 2^64 - 1 if none.
+// fp32(x) and the correctly rounded division never decrease as x grows, so
+// "x >= result" is exactly the fp32 decision; found by bisection with the
+// host's IEEE arithmetic (the device's __ull2float_rn and __fdiv_rn round
+// the same way).
+unsigned long long numerator_threshold(float thr, float den) {
+  const auto reaches = [&](unsigned long long x) { return static_cast<float>(x) / den >= thr; };
+  if (reaches(0)) return 0;
+  unsigned long long lo = 0, hi = ~0ull;  // reaches(lo) false; reaches(hi) decides "never"
+  if (!reaches(hi)) return ~0ull;
+  while (hi - lo > 1) {
+    const unsigned long long mid = lo + (hi - lo) / 2;
+    (reaches(mid) ? hi : lo) = mid;
+  }
+  return hi;
+}
+
 // Ring rows per stream: the last L_max feature rows, or for L_max = 0 the
 // previous frame's row and the reference frame's row.
 uint32_t ring_rows(const cofie_ngff* h) { return h->p.l_max ? h->p.l_max : 2u; }
@@ -269,6 +287,9 @@ SelectArgs select_args(const cofie_ngff* h) {
   sa.scd = h->p.signal == COFIE_SIGNAL_SCD ? 1u : 0u;
   sa.scd_cut = h->p.scd_cut;
   sa.scd_grad = h->p.scd_gradual;
+  sa.x_tau = h->x_tau;
+  sa.x_cut = h->x_cut;
+  sa.x_grad = h->x_grad;
   return sa;
 }
 
@@ -512,6 +533,9 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     h->fw = p->bins;
     h->two_n = static_cast<float>(2ull * h->npix);
   }
+  h->x_tau = numerator_threshold(p->tau, h->two_n);
+  h->x_cut = numerator_threshold(p->scd_cut, h->two_n);
+  h->x_grad = numerator_threshold(p->scd_gradual, h->two_n);
   if (p->signal == COFIE_SIGNAL_LOWRES || p->signal == COFIE_SIGNAL_DHASH) {
     FeatArgs& fa = h->fa;
     fa.frame_bytes = 3ull * h->npix;

@@ -97,6 +97,9 @@ struct SelectArgs {
   uint32_t dist_kind;  // 0: sum of |differences| (histogram, low-res); 1: Hamming (dHash)
   uint32_t scd;        // twin-comparison scene changes are added to the rule
   float scd_cut, scd_grad;
+  // the same three decisions as integer thresholds on the L1 numerator: the
+  // smallest x with fp32(x) / two_n >= tau, T_b, T_s (2^64 - 1: never)
+  unsigned long long x_tau, x_cut, x_grad;
 };
 
 // The spatial signals: per-frame grayscale sums on a grid of cells.

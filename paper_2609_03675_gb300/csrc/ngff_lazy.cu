@@ -6,9 +6,9 @@
 // One CTA per stream segment. Warp 0 holds c_{t-1} and c_{r(t)} of its
 // stream in registers (lane l: feature words l, l + 32, ...) and walks the
 // frames of a tile of feature rows in shared memory: both distances with one
-// warp reduction each, the fp32 decision, and the reference update. The
+// warp reduction each, the decision, and the reference update. The
 // other warps meanwhile stage the next tile from the (L2-resident) feature
-// rows into the other shared-memory buffer. The stream's state between
+// rows into the other shared-memory buffer with asynchronous copies. The stream's state between
 // pushes is {t, the open scene-change run} and two ring rows: slot 0 holds
 // c_{t-1}, slot 1 holds c_{r(t)}.
 #include "ngff_common.cuh"
@@ -18,17 +18,34 @@ namespace {
 
 constexpr int kLazyThreads = 256;
 constexpr uint32_t kLazyTileWords = 8192;  // 32 KiB per buffer, two buffers
-constexpr uint32_t kPer = kMaxBins / 32;   // feature words per lane, at most
+constexpr uint32_t kLazyMaxRows = kLazyTileWords / 2;  // rows per tile at the smallest width (dHash, 2 words)
 
 __device__ __forceinline__ uint32_t word_dist(uint32_t x, uint32_t y, uint32_t kind) {
   return kind == 1 ? static_cast<uint32_t>(__popc(x ^ y)) : (x > y ? x - y : y - x);
 }
 
+// Per tile of feature rows (shared memory, double-buffered):
+//   all warps  adjacent distances d_adj[f] = |c_f - c_{f-1}| of the tile;
+//   warp 0     the serial walk: d_ref = |c_f - c_r| (one warp reduction), the
+//              decision as an integer compare against the host-computed
+//              thresholds (the smallest numerators whose fp32 quotient by 2N
+//              reaches tau_h, T_b, T_s; exact since that quotient never
+//              decreases as the numerator grows), the scene-change run, and
+//              the reference update; meanwhile the other warps stage the
+//              next tile with asynchronous copies;
+//   all warps  the tile's fp32 scores and keep codes to global memory.
+// kP feature words per lane in the walk (B <= 32 kP).
+template <int kP>
 __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs, SelectArgs a,
                                                                    const uint32_t* __restrict__ feat,
                                                                    uint32_t* __restrict__ ring,
                                                                    StreamState* __restrict__ state) {
-  extern __shared__ __align__(16) uint32_t tiles[];  // [2][kLazyTileWords]
+  extern __shared__ __align__(16) uint32_t smem[];
+  uint32_t* tiles = smem;                            // [2][kLazyTileWords]
+  uint32_t* sadj = tiles + 2 * kLazyTileWords;       // [rows_per_tile] adjacent numerators
+  uint32_t* sd = sadj + kLazyMaxRows;                // [rows_per_tile] max(d_adj, d_ref)
+  uint8_t* scode = reinterpret_cast<uint8_t*>(sd + kLazyMaxRows);  // [rows_per_tile]
+  uint32_t* sprev = reinterpret_cast<uint32_t*>(scode + kLazyMaxRows);  // [B] the row before the tile
   const Segment sg = segs.s[blockIdx.x];
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t B = a.bins, n = sg.n;
@@ -36,92 +53,118 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   const uint32_t n_tiles = (n + rows_per_tile - 1) / rows_per_tile;
   const unsigned long long t0 = state[sg.stream].t;
   uint32_t* sring = ring + static_cast<uint64_t>(sg.stream) * 2 * B;
+  if (n == 0) return;
 
+  // asynchronous 4-byte copies (all of a thread's words in flight at once),
+  // waited for by the staging threads before the block barrier
   auto stage = [&](uint32_t tile, uint32_t first_thread, uint32_t threads) {
     const uint32_t j0 = tile * rows_per_tile, m = min(rows_per_tile, n - j0);
     uint32_t* dst = tiles + (tile & 1) * kLazyTileWords;
     const uint32_t* src = feat + static_cast<uint64_t>(sg.row0 + j0) * B;
-    for (uint32_t i = tid - first_thread; i < m * B; i += threads) dst[i] = src[i];
+    for (uint32_t i = tid - first_thread; i < m * B; i += threads)
+      asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst + i))),
+                   "l"(src + i)
+                   : "memory");
+    asm volatile("cp.async.commit_group;\ncp.async.wait_all;" ::: "memory");
+  };
+  // adjacent numerators of a staged tile: warp w takes rows w, w + 8, ...
+  auto adjacent = [&](uint32_t tile) {
+    const uint32_t j0 = tile * rows_per_tile, m = min(rows_per_tile, n - j0);
+    const uint32_t* buf = tiles + (tile & 1) * kLazyTileWords;
+    for (uint32_t f = warp; f < m; f += kLazyThreads / 32) {
+      const uint32_t* c = buf + f * B;
+      const uint32_t* p = f ? c - B : sprev;
+      uint32_t part = 0;
+      for (uint32_t b = lane; b < B; b += 32) part += word_dist(c[b], p[b], a.dist_kind);
+      part = __reduce_add_sync(0xffffffffu, part);
+      if (lane == 0) sadj[f] = part;
+    }
   };
 
-  // warp 0's registers: previous frame, reference frame, and the run sum
-  uint32_t prev[kPer], ref[kPer];
+  uint32_t ref[kP];  // warp 0: the reference frame's row
   unsigned long long acc = 0;
   if (warp == 0) {
 #pragma unroll
-    for (uint32_t q = 0; q < kPer; ++q) {
+    for (int q = 0; q < kP; ++q) {
       const uint32_t b = lane + 32 * q;
-      prev[q] = (t0 > 0 && b < B) ? sring[b] : 0u;
       ref[q] = (t0 > 0 && b < B) ? sring[B + b] : 0u;
     }
     acc = t0 > 0 ? state[sg.stream].acc : 0ull;
   }
-  if (n_tiles > 0) stage(0, 0, kLazyThreads);
+  for (uint32_t b = tid; b < B; b += kLazyThreads) sprev[b] = t0 > 0 ? sring[b] : 0u;
+  stage(0, 0, kLazyThreads);
+  __syncthreads();
+  adjacent(0);
   __syncthreads();
   for (uint32_t tile = 0; tile < n_tiles; ++tile) {
+    const uint32_t j0 = tile * rows_per_tile, m = min(rows_per_tile, n - j0);
+    const uint32_t* buf = tiles + (tile & 1) * kLazyTileWords;
     if (warp != 0) {
       if (tile + 1 < n_tiles) stage(tile + 1, 32, kLazyThreads - 32);
     } else {
-      const uint32_t j0 = tile * rows_per_tile, m = min(rows_per_tile, n - j0);
-      const uint32_t* buf = tiles + (tile & 1) * kLazyTileWords;
-      for (uint32_t f = 0; f < m; ++f) {
-        const uint32_t j = j0 + f;
-        const unsigned long long t = t0 + j;
-        uint32_t cur[kPer];
-        uint32_t pa = 0, pr = 0;
+      uint32_t nxt[kP];
 #pragma unroll
-        for (uint32_t q = 0; q < kPer; ++q) {
+      for (int q = 0; q < kP; ++q) nxt[q] = (lane + 32 * q < B) ? buf[lane + 32 * q] : 0u;
+      for (uint32_t f = 0; f < m; ++f) {
+        uint32_t cur[kP];
+        uint32_t pr = 0;
+#pragma unroll
+        for (int q = 0; q < kP; ++q) {
+          cur[q] = nxt[q];
           const uint32_t b = lane + 32 * q;
-          cur[q] = b < B ? buf[f * B + b] : 0u;
-          pa += word_dist(cur[q], prev[q], a.dist_kind);
+          nxt[q] = (f + 1 < m && b < B) ? buf[(f + 1) * B + b] : 0u;  // the next row, off the chain
           pr += word_dist(cur[q], ref[q], a.dist_kind);
         }
-        const uint32_t d_adj = __reduce_add_sync(0xffffffffu, pa);
-        const uint32_t d_ref = __reduce_add_sync(0xffffffffu, pr);
-        float s = 0.0f;
+        const uint32_t d_adj = sadj[f];
+        const uint32_t d = max(d_adj, __reduce_add_sync(0xffffffffu, pr));
         uint8_t code;
-        if (t == 0) {
+        if (t0 + j0 + f == 0) {
           code = 3;  // the stream's first frame
         } else {
-          s = __fdiv_rn(static_cast<float>(max(d_adj, d_ref)), a.two_n);
           bool scene = false;
           if (a.scd) {  // twin comparison on the adjacent difference
-            const float sd = __fdiv_rn(static_cast<float>(d_adj), a.two_n);
-            if (sd >= a.scd_cut) {
+            if (d_adj >= a.x_cut) {
               scene = true;
               acc = 0;
-            } else if (sd >= a.scd_grad) {
-              const unsigned long long before = acc;
+            } else if (d_adj >= a.x_grad) {
+              scene = acc < a.x_cut && acc + d_adj >= a.x_cut;  // the run's sum first reaches T_b
               acc += d_adj;
-              scene = __fdiv_rn(__ull2float_rn(acc), a.two_n) >= a.scd_cut &&
-                      !(__fdiv_rn(__ull2float_rn(before), a.two_n) >= a.scd_cut);
             } else {
               acc = 0;
             }
           }
-          code = s >= a.tau ? 1 : (scene ? 4 : 0);
+          code = d >= a.x_tau ? 1 : (scene ? 4 : 0);
         }
         if (lane == 0) {
-          if (sg.scores) sg.scores[j] = s;
-          if (sg.keep) sg.keep[j] = code;
+          sd[f] = d;
+          scode[f] = code;
         }
 #pragma unroll
-        for (uint32_t q = 0; q < kPer; ++q) {
-          if (code) ref[q] = cur[q];
-          prev[q] = cur[q];
-        }
+        for (int q = 0; q < kP; ++q) ref[q] = code ? cur[q] : ref[q];
       }
     }
     __syncthreads();
+    for (uint32_t f = tid; f < m; f += kLazyThreads) {
+      const bool first = t0 + j0 + f == 0;
+      if (sg.scores) sg.scores[j0 + f] = first ? 0.0f : __fdiv_rn(static_cast<float>(sd[f]), a.two_n);
+      if (sg.keep) sg.keep[j0 + f] = scode[f];
+    }
+    if (tile + 1 < n_tiles) {
+      for (uint32_t b = tid; b < B; b += kLazyThreads) sprev[b] = buf[(m - 1) * B + b];
+      __syncthreads();
+      adjacent(tile + 1);
+    }
+    __syncthreads();
   }
-  if (warp == 0 && n > 0) {
+  // the ring: slot 0 the last frame's row, slot 1 the reference's
+  const uint32_t last = (n - 1) - (n_tiles - 1) * rows_per_tile;
+  const uint32_t* lbuf = tiles + ((n_tiles - 1) & 1) * kLazyTileWords;
+  for (uint32_t b = tid; b < B; b += kLazyThreads) sring[b] = lbuf[last * B + b];
+  if (warp == 0) {
 #pragma unroll
-    for (uint32_t q = 0; q < kPer; ++q) {
+    for (int q = 0; q < kP; ++q) {
       const uint32_t b = lane + 32 * q;
-      if (b < B) {
-        sring[b] = prev[q];
-        sring[B + b] = ref[q];
-      }
+      if (b < B) sring[B + b] = ref[q];
     }
     if (lane == 0) {
       state[sg.stream].t = t0 + n;
@@ -131,16 +174,26 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   }
 }
 
+template <int kP>
+cudaError_t launch_p(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
+                     StreamState* state, cudaStream_t st) {
+  const size_t smem = 2 * kLazyTileWords * 4 + kLazyMaxRows * (4 + 4 + 1) + kMaxBins * 4;
+  cudaError_t e = cudaFuncSetAttribute(lazy_select_kernel<kP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  lazy_select_kernel<kP><<<segs.count, kLazyThreads, smem, st>>>(segs, a, feat, ring, state);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_lazy_select(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
                                StreamState* state, cudaStream_t st) {
-  const size_t smem = 2 * kLazyTileWords * sizeof(uint32_t);
-  cudaError_t e = cudaFuncSetAttribute(lazy_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  lazy_select_kernel<<<segs.count, kLazyThreads, smem, st>>>(segs, a, feat, ring, state);
-  return cudaGetLastError();
+  const uint32_t per = (a.bins + 31) / 32;
+  if (per <= 1) return launch_p<1>(segs, a, feat, ring, state, st);
+  if (per <= 2) return launch_p<2>(segs, a, feat, ring, state, st);
+  if (per <= 4) return launch_p<4>(segs, a, feat, ring, state, st);
+  return launch_p<8>(segs, a, feat, ring, state, st);
 }
 
 }  // namespace cofie

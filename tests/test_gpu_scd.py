@@ -81,13 +81,14 @@ def test_two_ramps_closed_form_on_device():
     from paper_2609_03675_gb300 import NGFF, _abi
     pos = [16 * t for t in range(21)] + [320] * 3 + [320 + 16 * (t - 23) for t in range(24, 64)]
     dev = torch.from_numpy(_frames_from_positions(pos)).cuda()
-    for chunks in ([64], [1] * 64, [5, 30, 29]):
-        f = NGFF(W, H, tau=0.5, l_max=256, signal=_abi.SIGNAL_SCD, scd_cut=0.125, scd_gradual=0.01)
-        _, k = _run(f, dev, chunks)
-        assert {int(t): int(k[t]) for t in np.flatnonzero(k)} == {0: 3, 8: 4, 31: 4, 63: 1}, chunks
+    for l_max in (256, 0):  # the window + scan kernels, and the frame-order walk
+        for chunks in ([64], [1] * 64, [5, 30, 29]):
+            f = NGFF(W, H, tau=0.5, l_max=l_max, signal=_abi.SIGNAL_SCD, scd_cut=0.125, scd_gradual=0.01)
+            _, k = _run(f, dev, chunks)
+            assert {int(t): int(k[t]) for t in np.flatnonzero(k)} == {0: 3, 8: 4, 31: 4, 63: 1}, (l_max, chunks)
 
 
-@pytest.mark.parametrize("tau,l_max", [(0.5, 30), (1.5, 7), (0.2, 256)])
+@pytest.mark.parametrize("tau,l_max", [(0.5, 30), (1.5, 7), (0.2, 256), (0.5, 0)])
 def test_random_walk_long_stream(tau, l_max):
     """12,000 frames: several 4096-frame scan tiles, runs crossing tile and
     push boundaries, pushes through both the fused small-push kernel and the
