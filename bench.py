@@ -194,6 +194,27 @@ def oracle_sample(frames_u8_ptr, spec, target_s: float, signal: int = 0, l_max: 
     return k, dt
 
 
+def oracle_parallel_sample(frames_u8_ptr, spec, target_s: float, l_max: int = 30):
+    """The oracle's histogram routine mapped over all host cores (frames in
+    parallel), then its selection, on the first k frames; k sized to about
+    target_s seconds. Returns (k, seconds, cores)."""
+    import oracle as O
+    o = O.load()
+    p = O.Params(spec.width, spec.height, l_max=l_max)
+    cores = max(1, len(os.sched_getaffinity(0)))
+
+    def run(k):
+        t = time.perf_counter()
+        hist = o.histograms_parallel(frames_u8_ptr, k, p, nthreads=cores)
+        o.select(hist, p)
+        return time.perf_counter() - t
+
+    t1 = run(min(cores, spec.frames))
+    per = t1 / min(cores, spec.frames)
+    k = int(max(cores, min(spec.frames, target_s / max(per, 1e-6))))
+    return k, run(k), cores
+
+
 def bench_gb300(args):
     import numpy as np  # noqa: F401
     import torch
@@ -316,7 +337,14 @@ def bench_gb300(args):
                 3: "C oracle histograms + the scene-change oracle's rule (Python)"}.get(
             signal, f"numpy signals oracle ({args.signal} features + selection)")
         cpu = {"value": k / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"first {k} frames of the 1080p stream, {what}"}
+               "sample": f"first {k} frames of the 1080p stream, {what}",
+               "wall_s": dt, "pixel_gbs": k * spec.frame_bytes / dt / 1e9}
+        if signal == 0:
+            kp, dtp, cores = oracle_parallel_sample(host.data_ptr(), spec, args.cpu_seconds / 2, args.l_max)
+            cpu["all_cores"] = {"value": kp / dtp, "unit": UNIT, "cores": cores, "wall_s": dtp,
+                                "pixel_gbs": kp * spec.frame_bytes / dtp / 1e9,
+                                "sample": f"first {kp} frames, the oracle's histogram routine on {cores} threads "
+                                          "(frames in parallel), then its selection"}
 
     if rank == 0:
         line = {
@@ -664,15 +692,66 @@ def bench_qer(args):
         "n_evidence": int(len(ev))}), flush=True)
 
 
+def bench_shards_ranks(args):
+    """One 1080p stream split over the ranks of a torchrun job (strong
+    scaling): every rank generates and prepares its shard plus halo, the gap
+    maps are all-gathered (NCCL), every rank commits its shard. The time of a
+    step is the max over ranks; the value counts the stream's frames."""
+    import torch
+    import torch.distributed as dist
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF, shards
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    spec = synth.hd1080().with_(frames=min(3600, args.frames))
+    T = spec.frames
+    a, b, halo = shards.shard_bounds(T, world, rank, 30)
+    host = torch.empty((b - a + halo, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, a - halo, b, out=host.data_ptr())
+    dev = host.cuda()
+    f = NGFF(spec.width, spec.height, max_frames_per_push=b - a + halo)
+
+    def step():
+        f.reset()
+        m = f.shard_prepare(dev, n_halo=halo, t0=a)
+        maps = shards.exchange_maps(m, world)
+        return f.shard_commit(shards.entry_gaps([x.tolist() for x in maps])[rank], b - a)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    torch.cuda.synchronize()
+    el = max_over_ranks(time.perf_counter() - t0)
+    dist.barrier()
+    f.status()
+    if rank == 0:
+        print(json.dumps({"workload": f"shards over ranks: the {T}-frame 1080p stream split over {world} GPUs",
+                          "n_gpus": world, "scaling": "strong", "steps": args.steps,
+                          "frames_per_s": T * args.steps / el, "ms_per_step": el / args.steps * 1e3,
+                          "exchange": "one all-gather of the 30-entry gap maps per step (NCCL)",
+                          "timing": "host wall time, max over ranks, device synchronised"}), flush=True)
+    dist.destroy_process_group()
+
+
 def bench_shards(args):
     """One 1080p stream split into 4 shards: each prepared from its frames and
     an L_max-frame halo (independently; on several GPUs they would run in
     parallel), chained through the gap maps, and committed. Reports the cost
-    against one whole-stream push, and the checkpoint size and latency."""
+    against one whole-stream push, and the checkpoint size and latency.
+    Under torchrun (several ranks) the shards run one per GPU instead."""
     import torch
 
     import synth
     from paper_2609_03675_gb300 import NGFF
+    if dist_env()[1] > 1:
+        bench_shards_ranks(args)
+        return
     spec = synth.hd1080().with_(frames=min(3600, args.frames))
     T = spec.frames
     host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
