@@ -32,7 +32,7 @@ METRIC = "NGFF frames/s and pixel GB/s (fraction of HBM peak) at 1 GB300 vs CPU 
 UNIT = "frames/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-K1_SOURCE = os.path.join(REPO, "paper_2609_03675_gb300", "csrc", "ngff_hist.cu")
+K1_SOURCES = [os.path.join(REPO, "paper_2609_03675_gb300", "csrc", f) for f in ("ngff_hist.cu", "ngff_device.cuh")]
 K1_TRAFFIC = os.path.join(REPO, "profiles", "k1_hist_1080p_traffic.json")
 
 
@@ -95,13 +95,21 @@ def peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def k1_source_hash() -> str:
+    """sha256 over K1's sources (the kernel file and its device helpers)."""
+    h = hashlib.sha256()
+    for path in K1_SOURCES:
+        h.update(open(path, "rb").read())
+    return h.hexdigest()
+
+
 def k1_traffic_per_launch():
     """DRAM bytes per histogram launch from the committed ncu summary, or None
     when the kernel source changed since the counters were taken."""
     try:
         with open(K1_TRAFFIC) as fh:
             d = json.load(fh)
-        src = hashlib.sha256(open(K1_SOURCE, "rb").read()).hexdigest()
+        src = k1_source_hash()
         if d.get("source_sha256") != src:
             return None
         return float(d["dram_bytes_per_launch_full"])

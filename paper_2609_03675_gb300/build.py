@@ -18,8 +18,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(REPO, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcofie_ngff.so")
-SOURCES = ["ngff_api.cu", "ngff_hist.cu", "ngff_select.cu", "ngff_lazy.cu", "ngff_finalize.cu", "ngff_static.cu",
-           "qer.cu"]
+SOURCES = ["ngff_api.cu", "ngff_hist.cu", "ngff_features.cu", "ngff_select.cu", "ngff_lazy.cu", "ngff_finalize.cu",
+           "ngff_static.cu", "qer.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -37,6 +37,7 @@ def _flags(extra=()):
 
 def _inputs():
     files = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, "ngff_common.cuh"),
+                                                        os.path.join(CSRC, "ngff_device.cuh"),
                                                         os.path.join(INCLUDE, "cofie_ngff.h"), __file__]
     return files
 
