@@ -409,13 +409,27 @@ typedef struct {
   uint32_t tokens_per_frame; /* |V_f|, the same for every frame */
   float rho;                 /* keep ratio, [0, 1] */
   int32_t device;            /* CUDA device ordinal, or -1 for the current device */
+  uint32_t kernel;           /* scoring kernel: COFIE_QER_KERNEL_* */
 } cofie_qer_params;
+
+/* Scoring kernels: the paired-SM one (clusters of two CTAs, one M = 256 MMA
+ * per pair) needs n_text rounded up to 16 to be a multiple of 32; AUTO takes
+ * it when it applies and the 256-token tiles of a run exceed one wave of the
+ * one-SM kernel (one per SM). The results of the two agree up to the order of
+ * fp32 accumulation inside the tensor cores. */
+#define COFIE_QER_KERNEL_AUTO 0
+#define COFIE_QER_KERNEL_ONE_SM 1
+#define COFIE_QER_KERNEL_PAIR 2
 
 /* Validates *p and allocates the scratch (group-summed queries, per-token
  * maxima, frame scores). Synchronous. Errors: COFIE_EINVAL, COFIE_ENOMEM, COFIE_ECUDA. */
 int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out);
 
 void cofie_qer_destroy(cofie_qer_t* h);
+
+/* COFIE_QER_KERNEL_PAIR if the handle runs the paired-SM kernel for runs
+ * above one wave (or always, when asked for), else COFIE_QER_KERNEL_ONE_SM (0 for NULL). */
+uint32_t cofie_qer_kernel_in_use(const cofie_qer_t* h);
 
 /*
  * Ranks n_frames candidate frames (Eqs. 6-8).

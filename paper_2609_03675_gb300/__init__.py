@@ -250,16 +250,17 @@ class QER:
     max(1, round(rho m)) of them."""
 
     def __init__(self, n_text: int, n_heads: int, n_kv_heads: int, head_dim: int, max_frames: int,
-                 tokens_per_frame: int, rho: float, device: int | None = None):
+                 tokens_per_frame: int, rho: float, device: int | None = None, kernel: int = 0):
         lib = _abi.load()
         p = _abi.QerParams(n_text, n_heads, n_kv_heads, head_dim, max_frames, tokens_per_frame, rho,
-                           torch.cuda.current_device() if device is None else device)
+                           torch.cuda.current_device() if device is None else device, kernel)
         h = ctypes.c_void_p()
         rc = lib.cofie_qer_create(ctypes.byref(p), ctypes.byref(h))
         if rc != _abi.OK:
             raise NGFFError(rc, lib.cofie_qer_last_error(None).decode())
         self._lib, self._h, self.params = lib, h, p
         self.device = torch.device("cuda", p.device)
+        self.kernel = int(lib.cofie_qer_kernel_in_use(h))  # 1: one-SM, 2: paired-SM
 
     def _check(self, rc):
         if rc != _abi.OK:

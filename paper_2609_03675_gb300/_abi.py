@@ -48,6 +48,7 @@ EXPORTS = (
     "cofie_qer_destroy",
     "cofie_qer_run",
     "cofie_qer_status",
+    "cofie_qer_kernel_in_use",
     "cofie_qer_profile_reset",
     "cofie_qer_profile_read",
     "cofie_qer_last_error",
@@ -107,7 +108,11 @@ class QerParams(ctypes.Structure):
         ("tokens_per_frame", ctypes.c_uint32),
         ("rho", ctypes.c_float),
         ("device", ctypes.c_int32),
+        ("kernel", ctypes.c_uint32),
     ]
+
+
+QER_KERNEL_AUTO, QER_KERNEL_ONE_SM, QER_KERNEL_PAIR = 0, 1, 2
 
 
 class NGFFError(RuntimeError):
@@ -185,6 +190,8 @@ def load():
     lib.cofie_qer_run.restype = ctypes.c_int
     lib.cofie_qer_status.argtypes = [H, vp]
     lib.cofie_qer_status.restype = ctypes.c_int
+    lib.cofie_qer_kernel_in_use.argtypes = [H]
+    lib.cofie_qer_kernel_in_use.restype = ctypes.c_uint32
     lib.cofie_qer_profile_reset.argtypes = [H, ctypes.c_int]
     lib.cofie_qer_profile_reset.restype = ctypes.c_int
     pu64 = ctypes.POINTER(ctypes.c_uint64)

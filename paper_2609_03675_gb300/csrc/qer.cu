@@ -61,8 +61,7 @@ constexpr int kQerEpiWarps = 4;    // epilogue warps: TMEM lanes 0..127
 constexpr int kQerThreads = 32 * (2 + kQerEpiWarps);  // + TMA producer warp + MMA issuer warp
 constexpr uint32_t kQerMaxN = 256;  // text tokens (MMA N) per CTA
 constexpr int kSelThreads = 1024;
-constexpr int kRankThreads = 64;  // few warps per CTA: the O(m^2) ranking spreads over many SMs
-constexpr uint32_t kSelSmemFrames = 11264;  // frame scores staged in 44 KiB of shared memory (within the default limit)
+constexpr int kRankThreads = 256;  // 8 frames per CTA (a warp each): the O(m^2) ranking spreads over many SMs
 
 constexpr uint32_t kQerErrProducer = 16u, kQerErrMma = 32u, kQerErrEpilogue = 64u, kQerErrDrain = 128u;
 
@@ -174,6 +173,83 @@ __device__ __forceinline__ float tmem_row_max(uint32_t taddr, uint32_t n_pad, ui
     }
   }
   return best;
+}
+
+
+// ---- paired-SM helpers (clusters of two CTAs) ----
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// The address of the same shared variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// A wait on a barrier that the peer CTA also arrives on (cluster-scope acquire).
+__device__ __noinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  if (mbar_try_cluster(bar, parity)) return true;
+  const uint64_t t0 = gtimer();
+  for (;;) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_cluster(bar, parity)) return true;
+    if (gtimer() - t0 > timeout_ns) return false;
+  }
+}
+
+// A tile load into this CTA's shared memory whose completion is counted on a
+// barrier that may live in the peer CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int32_t x, int32_t y,
+                                                 uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%2, %3}], "
+      "[%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_pair_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+// Arrives on the barrier at this shared offset in both CTAs of the pair once
+// every MMA this thread issued so far has completed.
+__device__ __forceinline__ void umma_pair_commit_both(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
 }
 
 __global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H,
@@ -388,6 +464,190 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
   }
 }
 
+// Paired-SM scoring kernel (tcgen05 cta_group::2; clusters of two CTAs on two
+// SMs). The pair covers a 256-token tile with one M = 256 MMA per 16-wide K
+// step (a ring stage holds n_sub 64-wide K chunks, so 4 n_sub MMAs): CTA rank r stages key rows [128 r, 128 r + 128) of the tile (A) and
+// q~ rows [r n_pad / 2, (r + 1) n_pad / 2) (half of B); the MMA, issued by
+// rank 0, reads both CTAs' halves and writes each CTA's 128 token rows x
+// n_pad text columns into that CTA's TMEM. Against the one-SM kernel this
+// halves the shared-memory reads of q~ per SM (each half of B is read once
+// for both SMs) and needs one accumulator of acc_cols columns per tile, so
+// two of them overlap a tile's epilogue with the next tile's MMAs.
+// Synchronisation: each CTA's TMA thread fills its own ring slot, and both
+// CTAs' copies count their bytes on rank 0's full barrier (rank 1 through
+// the paired form of the tensor copy), which rank 0's producer arms with the
+// bytes of both; rank 0's MMA thread waits on it alone, and commits MMA
+// completion to the empty barriers and accumulator barriers of both CTAs at
+// once (multicast). The epilogue warps of both CTAs arrive on rank 0's
+// tempty barrier. Every wait is bounded, and both CTAs always meet at a
+// final cluster barrier before TMEM is freed.
+__global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_constant__ CUtensorMap map_k,
+                                                              const __grid_constant__ CUtensorMap map_qh,
+                                                              uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
+                                                              uint32_t acc_cols, uint32_t n_stages, uint32_t n_sub,
+                                                              uint32_t n_chunks, uint32_t n_tiles,
+                                                              float* __restrict__ colmax,
+                                                              uint32_t* __restrict__ err, uint64_t timeout_ns) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t tfull_bar[2];
+  __shared__ __align__(8) uint64_t tempty_bar[2];
+  __shared__ __align__(8) uint64_t done_bar;
+  __shared__ uint32_t tmem_slot;
+  __shared__ volatile uint32_t abort_flag;
+
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t n_pairs = gridDim.x / 2, pair = blockIdx.x / 2;
+  const uint32_t half_rows = n_pad / 2;
+  const uint32_t a_bytes = kQerM * 128, b_bytes = half_rows * 128;
+  const uint32_t sub_bytes = (a_bytes + b_bytes + 1023) & ~1023u;  // one 64-wide K chunk of A and B
+  const uint32_t stage_bytes = n_sub * sub_bytes;                    // a ring stage: n_sub chunks
+  const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t my_tiles = pair < n_tiles ? (n_tiles - 1 - pair) / n_pairs + 1 : 0;
+  const uint32_t tmem_total = 2 * acc_cols;  // two accumulators
+
+  if (warp == 0) {  // one warp in each CTA of the pair allocates, together
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
+                 "r"(tmem_total)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  if (threadIdx.x == 32) {
+    for (uint32_t s = 0; s < n_stages; ++s) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full_bar[s])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&empty_bar[s])) : "memory");
+    }
+    for (int b = 0; b < 2; ++b) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&tfull_bar[b])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(&tempty_bar[b])), "r"(2 * kQerEpiWarps)
+                   : "memory");
+    }
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&done_bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    abort_flag = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers exist before any remote arrive or multicast commit
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer (both CTAs)
+      uint32_t g = 0;
+      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
+        const uint32_t row0 = (pair + t * n_pairs) * kQerTile + rank * kQerM;
+        for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
+          const uint32_t s = g % n_stages, use = g / n_stages;
+          if (use > 0 && !mbar_wait_cluster(smem_u32(&empty_bar[s]), (use - 1) & 1, timeout_ns)) {
+            atomicOr(err, kQerErrProducer);
+            abort_flag = 1;
+            break;
+          }
+          if (abort_flag) break;
+          const uint32_t fb0 = map_to_rank(smem_u32(&full_bar[s]), 0);  // rank 0's full barrier
+          if (rank == 0)
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(&full_bar[s])),
+                         "r"(2 * n_sub * (a_bytes + b_bytes))
+                         : "memory");
+          const uint32_t base = smem_u32(smem + s * stage_bytes);
+          for (uint32_t sub = 0; sub < n_sub; ++sub) {
+            const int32_t x = static_cast<int32_t>((kc * n_sub + sub) * kQerKChunk);
+            const uint32_t b = base + sub * sub_bytes;
+            tma_load_2d_pair(b, &map_k, x, static_cast<int32_t>(row0), fb0);
+            tma_load_2d_pair(b + a_bytes, &map_qh, x, static_cast<int32_t>(rank * half_rows), fb0);
+          }
+        }
+      }
+      // no copy may still be writing shared memory when the CTA exits: the
+      // last copies of every slot were read by MMAs whose completion reached
+      // this CTA's empty barrier
+      for (uint32_t j = g > n_stages ? g - n_stages : 0; j < g; ++j)
+        if (!mbar_wait_cluster(smem_u32(&empty_bar[j % n_stages]), (j / n_stages) & 1, timeout_ns))
+          atomicOr(err, kQerErrDrain);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // ------------------------------------------------ MMA issuer (rank 0)
+      const uint32_t idesc = idesc_bf16_f32(2 * kQerM, n_pad);
+      uint32_t g = 0;
+      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
+        const uint32_t b = t & 1, ub = t >> 1;
+        if (ub > 0 && !mbar_wait_cluster(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
+          atomicOr(err, kQerErrMma);
+          abort_flag = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc = tmem + b * acc_cols;
+        bool stop = false;
+        for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
+          const uint32_t s = g % n_stages, use = g / n_stages;
+          if (!mbar_wait_cluster(smem_u32(&full_bar[s]), use & 1, timeout_ns) || abort_flag) {
+            atomicOr(err, kQerErrMma);
+            abort_flag = 1;
+            stop = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(smem + s * stage_bytes), b0 = a0 + a_bytes;
+          for (uint32_t sub = 0; sub < n_sub; ++sub) {
+#pragma unroll
+            for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk) {
+              const uint32_t o = sub * sub_bytes + kk * 32;
+              umma_pair_bf16(acc, sw128_desc(a0 + o), sw128_desc(b0 + o), idesc, (kc | sub | kk) != 0);
+            }
+          }
+          umma_pair_commit_both(smem_u32(&empty_bar[s]));  // both CTAs' slot s is free once read
+        }
+        if (stop) break;
+        umma_pair_commit_both(smem_u32(&tfull_bar[b]));  // accumulator b holds tile t in both CTAs
+      }
+      umma_pair_commit_both(smem_u32(&done_bar));  // every MMA of the pair is complete
+    }
+  } else {
+    // ------------------------------------------------------ epilogue (both CTAs)
+    const uint32_t quarter = warp & 3;
+    const uint32_t tempty0 = map_to_rank(smem_u32(&tempty_bar[0]), 0);
+    const uint32_t tempty1 = map_to_rank(smem_u32(&tempty_bar[1]), 0);
+    for (uint32_t t = 0; t < my_tiles; ++t) {
+      const uint32_t b = t & 1, ub = t >> 1;
+      bool ok = !abort_flag && mbar_wait_cluster(smem_u32(&tfull_bar[b]), ub & 1, timeout_ns);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) {
+        if (lane == 0) atomicOr(err, kQerErrEpilogue);
+        abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t taddr = tmem + b * acc_cols + ((quarter * 32u) << 16);
+      const float best = tmem_row_max(taddr, n_pad, n_text);
+      const uint32_t j = (pair + t * n_pairs) * kQerTile + rank * kQerM + quarter * 32 + lane;
+      if (j < n_visual) colmax[j] = best;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(b ? tempty1 : tempty0);
+    }
+  }
+  __syncwarp();
+  // TMEM is freed only after every MMA of the pair has completed, and only
+  // once both CTAs are past every remote arrive and multicast commit
+  if (warp == 0) {
+    const bool ok = mbar_wait_cluster(smem_u32(&done_bar), 0, timeout_ns);
+    if (!ok && lane == 0) atomicOr(err, kQerErrDrain);
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(tmem_total) : "memory");
+  }
+}
+
 // Eq. 7: w_f = mean over the frame's tokens of their max over text, times the
 // 1/(H sqrt(d)) of Eq. 6. One warp per frame.
 __global__ void __launch_bounds__(256) qer_mean(const float* __restrict__ colmax, uint32_t n_frames, uint32_t tpf,
@@ -402,26 +662,21 @@ __global__ void __launch_bounds__(256) qer_mean(const float* __restrict__ colmax
 }
 
 // Eq. 8: flag[f] = 1 when fewer than k frames rank above frame f (higher w,
-// or equal w and lower index). Each CTA stages all scores in shared memory
-// (or reads them from global memory when they do not fit); a thread per frame.
+// or equal w and lower index). A warp per frame: its lanes split the m scores
+// (coalesced reads of the L2-resident w) and one warp reduction counts them.
 __global__ void __launch_bounds__(kRankThreads) qer_rank(const float* __restrict__ w, uint32_t n_frames, uint32_t k,
                                                 uint8_t* __restrict__ flag) {
-  extern __shared__ float sw[];
-  const bool in_smem = n_frames <= kSelSmemFrames;
-  if (in_smem)
-    for (uint32_t g = threadIdx.x; g < n_frames; g += blockDim.x) sw[g] = w[g];
-  __syncthreads();
-  const float* ws = in_smem ? sw : w;
-  const uint32_t f = blockIdx.x * blockDim.x + threadIdx.x;
-  if (f >= n_frames) return;
-  const float wf = ws[f];
+  const uint32_t f = blockIdx.x * (kRankThreads / 32) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (f >= n_frames) return;  // uniform across the warp
+  const float wf = w[f];
   uint32_t above = 0;
-#pragma unroll 8
-  for (uint32_t g = 0; g < n_frames; ++g) {
-    const float wg = ws[g];  // the same word for the whole warp: a broadcast
+#pragma unroll 4
+  for (uint32_t g = lane; g < n_frames; g += 32) {
+    const float wg = __ldg(w + g);
     above += (wg > wf) | ((wg == wf) & (g < f));
   }
-  flag[f] = above < k;
+  above = __reduce_add_sync(0xffffffffu, above);
+  if (lane == 0) flag[f] = above < k;
 }
 
 // The flagged frames, in time order: block-wide compaction (ballot,
@@ -462,6 +717,16 @@ uint32_t qer_stage_bytes(uint32_t n_pad) { return 2 * kQerM * 128 + ((n_pad * 12
 
 uint32_t qer_stages(uint32_t n_pad) {
   const size_t n = kQerStageBudget / qer_stage_bytes(n_pad);
+  return static_cast<uint32_t>(n < kQerMaxStages ? n : kQerMaxStages);
+}
+
+// A ring stage of the paired kernel holds n_sub 64-wide K chunks of A and B.
+uint32_t qer_pair_stage_bytes(uint32_t n_pad, uint32_t n_sub) {
+  return n_sub * ((kQerM * 128 + (n_pad / 2) * 128 + 1023) & ~1023u);
+}
+
+uint32_t qer_pair_stages(uint32_t n_pad, uint32_t n_sub) {
+  const size_t n = kQerStageBudget / qer_pair_stage_bytes(n_pad, n_sub);
   return static_cast<uint32_t>(n < kQerMaxStages ? n : kQerMaxStages);
 }
 
@@ -506,6 +771,10 @@ struct cofie_qer {
   uint32_t n_pad = 0, D = 0, acc_cols = 0, n_buf = 1, n_stages = 0;
   int grid = 0;          // persistent CTAs
   size_t smem = 0;       // dynamic shared memory per CTA
+  bool pair = false;     // the paired-SM kernel (clusters of two CTAs)
+  uint32_t pair_stages = 0, pair_sub = 1;
+  int pair_clusters = 0;  // co-resident clusters
+  size_t pair_smem = 0;
   __nv_bfloat16_raw* d_qg = nullptr;
   float* d_colmax = nullptr;
   float* d_w = nullptr;
@@ -568,6 +837,7 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
       static_cast<uint64_t>(p->max_frames) * p->tokens_per_frame > 0x7fffffffull)
     return g_qer_error = "max_frames and tokens_per_frame must be >= 1 (product < 2^31)", COFIE_EINVAL;
   if (!(p->rho >= 0.f && p->rho <= 1.f)) return g_qer_error = "rho must be in [0, 1]", COFIE_EINVAL;
+  if (p->kernel > COFIE_QER_KERNEL_PAIR) return g_qer_error = "kernel must be one of COFIE_QER_KERNEL_*", COFIE_EINVAL;
   int dev = p->device;
   if (dev < 0 && cudaGetDevice(&dev) != cudaSuccess) return g_qer_error = "no CUDA device", COFIE_ECUDA;
   int prev = -1;
@@ -614,6 +884,43 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
   if (e == cudaSuccess && (per_sm_ctas < 1 || per_sm_ctas > max_ctas_by_tmem)) e = cudaErrorInvalidConfiguration;
   h->grid = n_sms * (per_sm_ctas > 0 ? per_sm_ctas : 1);
+  if (e == cudaSuccess && p->kernel != COFIE_QER_KERNEL_ONE_SM && h->n_pad % 32 == 0) {
+    // the paired-SM kernel: one accumulator of acc_cols columns per buffer,
+    // two buffers; the same TMEM residency rule through shared memory
+    // two 64-wide K chunks per ring stage when D allows: every stage costs a
+    // fixed synchronisation overhead, which more MMAs per stage amortise
+    h->pair_sub = (h->D / kQerKChunk) % 2 == 0 ? 2 : 1;
+    h->pair_stages = qer_pair_stages(h->n_pad, h->pair_sub);
+    h->pair_smem = static_cast<size_t>(h->pair_stages) * qer_pair_stage_bytes(h->n_pad, h->pair_sub) + 1024;
+    const int pair_ctas_by_tmem = static_cast<int>(512 / (2 * h->acc_cols));
+    while (per_sm / (h->pair_smem + 1024) > static_cast<size_t>(pair_ctas_by_tmem)) h->pair_smem += 1024;
+    cudaError_t pe = cudaFuncSetAttribute(qer_score_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          static_cast<int>(h->pair_smem));
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * n_sms, 1, 1);
+    cfg.blockDim = dim3(kQerThreads, 1, 1);
+    cfg.dynamicSmemBytes = h->pair_smem;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int clusters = 0;
+    if (pe == cudaSuccess) pe = cudaOccupancyMaxActiveClusters(&clusters, qer_score_pair, &cfg);
+    if (pe == cudaSuccess && clusters >= 1) {
+      h->pair = true;
+      h->pair_clusters = clusters;
+    } else {
+      cudaGetLastError();
+      if (p->kernel == COFIE_QER_KERNEL_PAIR) e = pe != cudaSuccess ? pe : cudaErrorInvalidConfiguration;
+    }
+  } else if (e == cudaSuccess && p->kernel == COFIE_QER_KERNEL_PAIR) {
+    if (prev >= 0) cudaSetDevice(prev);
+    qer_free(h);
+    return g_qer_error = "the paired-SM kernel needs n_text rounded up to 16 to be a multiple of 32", COFIE_EINVAL;
+  }
   if (prev >= 0) cudaSetDevice(prev);
   if (e != cudaSuccess) {
     g_qer_error = std::string("QER set-up failed: ") + cudaGetErrorString(e);
@@ -626,6 +933,10 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
 }
 
 void cofie_qer_destroy(cofie_qer_t* h) { qer_free(h); }
+
+uint32_t cofie_qer_kernel_in_use(const cofie_qer_t* h) {
+  return h ? (h->pair ? COFIE_QER_KERNEL_PAIR : COFIE_QER_KERNEL_ONE_SM) : 0u;
+}
 
 int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t n_frames, float* w_out,
                   uint32_t* sel_out, uint32_t* k_out, void* cuda_stream) {
@@ -649,7 +960,12 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   const uint64_t nv = static_cast<uint64_t>(n_frames) * p.tokens_per_frame;
   CUtensorMap map_k, map_q;
-  if (!make_map(&map_k, k, nv, h->D, kQerM) || !make_map(&map_q, h->d_qg, h->n_pad, h->D, h->n_pad))
+  const uint32_t tiles = static_cast<uint32_t>((nv + kQerTile - 1) / kQerTile);
+  // the paired kernel when asked for, or (automatic) when the tiles exceed
+  // one wave of the one-SM kernel: a single wave runs faster on twice the CTAs
+  const bool pair_run = h->pair && (p.kernel == COFIE_QER_KERNEL_PAIR || tiles > static_cast<uint32_t>(h->grid));
+  const uint32_t q_box = pair_run ? h->n_pad / 2 : h->n_pad;  // the pair's CTAs each stage half of q~
+  if (!make_map(&map_k, k, nv, h->D, kQerM) || !make_map(&map_q, h->d_qg, h->n_pad, h->D, q_box))
     return h->fail(COFIE_ECUDA, "tensor map encoding failed");
   if (p.head_dim % 8 == 0 && reinterpret_cast<uintptr_t>(q) % 16 == 0) {
     const uint64_t n8 = static_cast<uint64_t>(h->n_pad) * h->D / 8;
@@ -659,7 +975,6 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   } else {
     qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, h->n_pad, p.n_heads, p.n_kv_heads, p.head_dim, h->d_qg);
   }
-  const uint32_t tiles = static_cast<uint32_t>((nv + kQerTile - 1) / kQerTile);
   const uint32_t grid = tiles < static_cast<uint32_t>(h->grid) ? tiles : static_cast<uint32_t>(h->grid);
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (h->time_on && h->ev_used + 2 <= (1u << 16)) {
@@ -675,9 +990,28 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
       cudaEventRecord(e0, st);
     }
   }
-  qer_score<<<grid, kQerThreads, h->smem, st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
-                                                h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles,
-                                                h->d_colmax, h->d_err, 2000000000ull);
+  if (pair_run) {
+    const uint32_t clusters = std::min<uint32_t>(tiles, static_cast<uint32_t>(h->pair_clusters));
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * clusters, 1, 1);
+    cfg.blockDim = dim3(kQerThreads, 1, 1);
+    cfg.dynamicSmemBytes = h->pair_smem;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, qer_score_pair, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad, h->acc_cols,
+                       h->pair_stages, h->pair_sub, h->D / kQerKChunk / h->pair_sub, tiles, h->d_colmax, h->d_err,
+                       2000000000ull);
+  } else {
+    qer_score<<<grid, kQerThreads, h->smem, st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
+                                                  h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles,
+                                                  h->d_colmax, h->d_err, 2000000000ull);
+  }
   if (e1) cudaEventRecord(e1, st);
   h->launches += 1;
   h->flops += 2.0 * h->n_pad * static_cast<double>(nv) * h->D;
@@ -687,8 +1021,8 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   float* w = w_out ? w_out : h->d_w;
   uint32_t* kdev = is_device(k_out, h->device) ? k_out : h->d_k;
   qer_mean<<<(n_frames + 7) / 8, 256, 0, st>>>(h->d_colmax, n_frames, p.tokens_per_frame, scale, w);
-  const size_t rank_smem = n_frames <= kSelSmemFrames ? n_frames * sizeof(float) : 0;
-  qer_rank<<<(n_frames + kRankThreads - 1) / kRankThreads, kRankThreads, rank_smem, st>>>(w, n_frames, kk, h->d_flag);
+  qer_rank<<<(n_frames + kRankThreads / 32 - 1) / (kRankThreads / 32), kRankThreads, 0, st>>>(w, n_frames, kk,
+                                                                                              h->d_flag);
   qer_compact<<<1, kSelThreads, 0, st>>>(h->d_flag, n_frames, sel_out, kdev);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess && kdev != k_out) {

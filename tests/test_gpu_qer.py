@@ -21,10 +21,13 @@ def _cuda():
         pytest.skip("no CUDA device")
 
 
-def _run_gpu(spec, rho):
+def _run_gpu(spec, rho, kernel=0):
     from paper_2609_03675_gb300 import QER
     q, k, ev = S.generate(spec)
-    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, rho)
+    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, rho,
+            kernel=kernel)
+    if kernel:
+        assert f.kernel == kernel
     qd = torch.from_numpy(q.view(np.int16)).cuda()
     kd = torch.from_numpy(k.view(np.int16)).cuda()
     w, sel = f.run(qd, kd)
@@ -33,8 +36,8 @@ def _run_gpu(spec, rho):
     return q, k, ev, w.cpu().numpy().astype(np.float64), sel.cpu().numpy().astype(np.int64)
 
 
-def check(spec, rho, frames=None):
-    q, k, ev, w_gpu, sel_gpu = _run_gpu(spec, rho)
+def check(spec, rho, frames=None, kernel=0):
+    q, k, ev, w_gpu, sel_gpu = _run_gpu(spec, rho, kernel)
     rho32 = float(np.float32(rho))
     m = spec.n_frames
     kk = Q.keep_count(m, rho32)
@@ -70,7 +73,8 @@ def check(spec, rho, frames=None):
                seed=9), 0.5),
 ])
 def test_qer_small_and_ragged(spec, rho):
-    check(spec, rho)
+    check(spec, rho)  # the paired-SM kernel where n_text rounds up to a multiple of 32, else the one-SM kernel
+    check(spec, rho, kernel=1)
 
 
 @pytest.mark.parametrize("spec", [
@@ -87,6 +91,24 @@ def test_qer_exact_on_integer_inputs(spec):
     assert np.all(np.abs(w_gpu - w_o) <= 2.0 ** -21 * np.abs(w_o)), np.abs(w_gpu - w_o).max()
 
 
+@pytest.mark.parametrize("spec", [
+    S.QerSpec(n_text=256, n_heads=32, n_kv_heads=8, head_dim=128, n_frames=9, tokens_per_frame=256, integer=True,
+              seed=17),
+    S.QerSpec(n_text=90, n_heads=8, n_kv_heads=4, head_dim=64, n_frames=7, tokens_per_frame=150, integer=True,
+              seed=18),
+    S.QerSpec(n_text=32, n_heads=4, n_kv_heads=1, head_dim=64, n_frames=3, tokens_per_frame=700, integer=True,
+              seed=19),
+])
+def test_qer_pair_kernel_equals_one_sm_kernel(spec):
+    """On integer inputs every product and sum is exact, so the two scoring
+    kernels must give the same frame scores bit for bit, and the oracle's."""
+    q, k, _, w1, s1 = _run_gpu(spec, 0.5, kernel=1)
+    _, _, _, w2, s2 = _run_gpu(spec, 0.5, kernel=2)
+    assert np.array_equal(w1, w2) and np.array_equal(s1, s2)
+    w_o = Q.frame_relevance(Q.token_scores(q, k), spec.tokens_per_frame)
+    assert np.all(np.abs(w2 - w_o) <= 2.0 ** -21 * np.abs(w_o))
+
+
 def test_qer_planted_evidence_found():
     spec = S.QerSpec(n_text=64, n_heads=32, n_kv_heads=8, head_dim=128, n_frames=32, tokens_per_frame=64,
                      n_evidence=4, seed=6)
@@ -94,9 +116,14 @@ def test_qer_planted_evidence_found():
     assert list(sel) == list(ev)
 
 
-def test_qer_full_size_sampled():
-    """The benchmark's geometry: 256 text tokens, 128 frames x 256 tokens,
-    32/8 heads of 128; the oracle checks 12 sampled frames."""
-    spec = S.QerSpec()
+@pytest.mark.parametrize("n_frames", [128, 400])
+def test_qer_full_size_sampled(n_frames):
+    """The benchmark's geometry: 256 text tokens, frames of 256 tokens, 32/8
+    heads of 128; the oracle checks 12 sampled frames. 128 frames fit one
+    wave of the one-SM kernel; 400 frames take the paired-SM kernel."""
+    from paper_2609_03675_gb300 import QER
+    spec = S.QerSpec(n_frames=n_frames)
     frames = np.linspace(0, spec.n_frames - 1, 12).astype(int)
     check(spec, 0.3, frames=frames)
+    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3)
+    assert f.kernel == 2  # the handle can pair; a run switches to it above one wave
