@@ -317,6 +317,13 @@ int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_o
  *                                the handle stay usable.
  */
 void cofie_ngff_debug_fail_alloc(int32_t after);
+
+/* 1 if this library is the checked build (compiled with -DCOFIE_DEBUG_CHECKS=1):
+ * its kernels check computed indices against their launch arguments, skip an
+ * access that fails, and cofie_ngff_status then reports COFIE_EDEVICE (error
+ * bit 16). It stands in for a memory checker; normal builds return 0 and
+ * carry no checks. */
+int cofie_ngff_checked_build(void);
 int cofie_ngff_debug_wait(cofie_ngff_t* h, uint64_t timeout_ns, void* cuda_stream);
 
 /*

@@ -38,6 +38,7 @@ EXPORTS = (
     "cofie_ngff_frames_seen",
     "cofie_ngff_debug_bins",
     "cofie_ngff_debug_fail_alloc",
+    "cofie_ngff_checked_build",
     "cofie_ngff_debug_wait",
     "cofie_ngff_profile_reset",
     "cofie_ngff_profile_read",
@@ -172,6 +173,8 @@ def load():
     lib.cofie_ngff_frames_seen.restype = ctypes.c_int
     lib.cofie_ngff_debug_bins.argtypes = [H, vp, u64, vp, vp]
     lib.cofie_ngff_debug_bins.restype = ctypes.c_int
+    lib.cofie_ngff_checked_build.argtypes = []
+    lib.cofie_ngff_checked_build.restype = ctypes.c_int
     lib.cofie_ngff_debug_fail_alloc.argtypes = [ctypes.c_int32]
     lib.cofie_ngff_debug_fail_alloc.restype = None
     lib.cofie_ngff_debug_wait.argtypes = [H, u64, vp]

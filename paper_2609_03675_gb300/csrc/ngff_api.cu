@@ -22,6 +22,7 @@
 using namespace cofie;
 
 namespace cofie {
+bool checked_build() { return COFIE_DEBUG_CHECKS != 0; }
 std::atomic<int> g_fail_alloc{-1};
 }
 
@@ -917,10 +918,17 @@ int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream) {
   uint32_t word = 0;
   e = cudaMemcpy(&word, h->d_err, sizeof word, cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return h->cuda_fail(e, "error word read");
+  if (checked_build()) {  // the index checks of every kernel file (checked builds only)
+    const uint32_t b = take_bounds_errors_hist() | take_bounds_errors_features() | take_bounds_errors_select() |
+                       take_bounds_errors_lazy() | take_bounds_errors_finalize();
+    if (b) word |= kErrBounds;
+  }
   if (word) {
     cudaMemset(h->d_err, 0, sizeof word);
     char buf[128];
-    snprintf(buf, sizeof buf, "device-side failure (error bits 0x%x: 1/2/4 a wait ran out, 8 a bad gather index)",
+    snprintf(buf, sizeof buf,
+             "device-side failure (error bits 0x%x: 1/2/4 a wait ran out, 8 a bad gather index, 16 an index check "
+             "of the checked build)",
              word);
     return h->fail((word & (kErrConsumerTimeout | kErrProducerTimeout | kErrDrainTimeout)) ? COFIE_ETIMEOUT
                                                                                           : COFIE_EDEVICE,
@@ -934,6 +942,8 @@ int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_o
   *t_out = h->seen[stream];
   return COFIE_OK;
 }
+
+int cofie_ngff_checked_build(void) { return checked_build() ? 1 : 0; }
 
 void cofie_ngff_debug_fail_alloc(int32_t after) { g_fail_alloc.store(after < 0 ? -1 : after); }
 

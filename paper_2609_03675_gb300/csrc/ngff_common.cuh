@@ -67,11 +67,49 @@ struct StreamState {
   unsigned long long acc;  // scene-change signal: L1 numerator summed over the open gradual run (0: none)
 };
 
+// Index checks of the checked build (-DCOFIE_DEBUG_CHECKS=1), which stands in
+// for a memory checker: COFIE_BOUND(c) is true in normal builds (and
+// compiles away); in checked builds a false c sets this translation unit's
+// bounds error word and the guarded access is skipped. cofie_ngff_status
+// collects the words (COFIE_EDEVICE). Each check relates an index to the
+// kernel's own launch arguments (rows, L_max, bins, tile sizes).
+#ifndef COFIE_DEBUG_CHECKS
+#define COFIE_DEBUG_CHECKS 0
+#endif
+namespace {
+#if COFIE_DEBUG_CHECKS
+__device__ uint32_t g_bounds_err;
+__device__ __forceinline__ bool bound_ok(bool c) {
+  if (!c) atomicOr(&g_bounds_err, 1u);
+  return c;
+}
+#define COFIE_BOUND(c) (::cofie::bound_ok(static_cast<bool>(c)))
+// this translation unit's word, read and cleared (host; synchronous)
+inline uint32_t take_local_bounds_errors() {
+  uint32_t v = 0, z = 0;
+  if (cudaMemcpyFromSymbol(&v, g_bounds_err, sizeof v) != cudaSuccess) return 0;
+  cudaMemcpyToSymbol(g_bounds_err, &z, sizeof z);
+  return v;
+}
+#else
+#define COFIE_BOUND(c) true
+inline uint32_t take_local_bounds_errors() { return 0; }
+#endif
+}  // namespace
+// one reader per translation unit with checked kernels
+uint32_t take_bounds_errors_hist();
+uint32_t take_bounds_errors_features();
+uint32_t take_bounds_errors_select();
+uint32_t take_bounds_errors_lazy();
+uint32_t take_bounds_errors_finalize();
+bool checked_build();
+
 // Bits of the device error word.
 constexpr uint32_t kErrConsumerTimeout = 1u;
 constexpr uint32_t kErrProducerTimeout = 2u;
 constexpr uint32_t kErrDrainTimeout = 4u;
 constexpr uint32_t kErrBadIndex = 8u;  // a gather index outside the frame buffer
+constexpr uint32_t kErrBounds = 16u;   // checked build: an index check failed
 
 struct HistArgs {
   uint64_t frame_bytes;      // 3 W H

@@ -48,21 +48,22 @@ __global__ void __launch_bounds__(kFeatThreads) features_kernel(SegTable segs, F
       for (uint32_t i = 0; i < 16; ++i) {
         const uint32_t yv = fa.use_magic ? __umulhi(v[i], L.magic_y) : v[i] / L.den;
         if (x0 + i >= next) {
-          atomicAdd(&cell[cy * gw + cx], acc);
+          if (COFIE_BOUND(cy * gw + cx < gh * gw)) atomicAdd(&cell[cy * gw + cx], acc);
           acc = 0;
           ++cx;
           next = ((cx + 1) * W + gw - 1) / gw;
         }
         acc += yv;
       }
-      atomicAdd(&cell[cy * gw + cx], acc);
+      if (COFIE_BOUND(cy * gw + cx < gh * gw)) atomicAdd(&cell[cy * gw + cx], acc);
     }
   } else {
     for (uint32_t p = tid; p < fa.npix; p += kFeatThreads) {
       const uint8_t* px = frame + 3ull * p;
       const uint32_t yv = (L.w[0] * px[0] + L.w[1] * px[1] + L.w[2] * px[2] + L.half) / L.den;
       const uint32_t y = p / W, x = p - y * W;
-      atomicAdd(&cell[(y * gh / H) * gw + x * gw / W], yv);
+      const uint32_t ci = (y * gh / H) * gw + x * gw / W;
+      if (COFIE_BOUND(ci < gh * gw)) atomicAdd(&cell[ci], yv);
     }
   }
   __syncthreads();
@@ -161,5 +162,7 @@ cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaCo
     debug_bins_kernel<kBinTwoStep><<<grid, threads, 0, st>>>(px, n_groups, lc, bins_out);
   return cudaGetLastError();
 }
+
+uint32_t take_bounds_errors_features() { return take_local_bounds_errors(); }
 
 }  // namespace cofie

@@ -71,7 +71,7 @@ __global__ void __launch_bounds__(kFinThreads) candidates_kernel(const uint8_t* 
       if (lane == 31) s_total = x;
     }
     __syncthreads();
-    if (in) idx[base + wsum[warp] + before] = t;
+    if (in && COFIE_BOUND(base + wsum[warp] + before < T)) idx[base + wsum[warp] + before] = t;
     base += s_total;
     __syncthreads();
   }
@@ -139,5 +139,7 @@ cudaError_t launch_gather(const uint8_t* frames, uint32_t n_frames, uint64_t fra
   }
   return cudaGetLastError();
 }
+
+uint32_t take_bounds_errors_finalize() { return take_local_bounds_errors(); }
 
 }  // namespace cofie

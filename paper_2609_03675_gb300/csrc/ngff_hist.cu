@@ -162,21 +162,21 @@ __device__ __forceinline__ void cells_chunk(const uint8_t* buf, uint32_t groups,
 #pragma unroll
       for (int k = 0; k < 2; ++k) q[k] = (i & 4) ? q[2 * k + 1] : q[2 * k];
       const uint32_t lo = (i & 8) ? q[1] : q[0];
-      atomicAdd(&cells[crow + cx], lo);
-      if (i < 15) atomicAdd(&cells[crow + cx + 1], P[15] - lo);
+      if (COFIE_BOUND(crow + cx < gh * gw)) atomicAdd(&cells[crow + cx], lo);
+      if (i < 15 && COFIE_BOUND(crow + cx + 1 < gh * gw)) atomicAdd(&cells[crow + cx + 1], P[15] - lo);
     } else {
       uint32_t acc = 0;
 #pragma unroll
       for (uint32_t i = 0; i < 16; ++i) {
         if ((x0 + i) * gw >= edge) {
-          atomicAdd(&cells[crow + cx], acc);
+          if (COFIE_BOUND(crow + cx < gh * gw)) atomicAdd(&cells[crow + cx], acc);
           acc = 0;
           ++cx;
           edge += W;
         }
         acc += v[i];
       }
-      atomicAdd(&cells[crow + cx], acc);
+      if (COFIE_BOUND(crow + cx < gh * gw)) atomicAdd(&cells[crow + cx], acc);
     }
   }
 }
@@ -260,6 +260,9 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
         break;
       }
       const uint32_t bytes = cur.groups(gpf) * kGroupBytes;
+      // checked build: a chunk outside the push stops the producer (the
+      // consumers' bounded waits then end the launch with an error)
+      if (!COFIE_BOUND(cur.row < segs.rows && cur.k < cpf && bytes <= kChunkBytes)) break;
       mbar_arrive_expect_tx(full0 + 8 * slot, bytes);
       bulk_load(ring0 + slot * kChunkBytes, cur.src(sseg, a.frame_bytes), bytes, full0 + 8 * slot, pol);
       cur.advance(cpf, sseg, nseg);
@@ -314,7 +317,8 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
         for (uint32_t b = tid; b < n_cnt; b += kNC) {
           const uint32_t sum = cnt[b];
           cnt[b] = 0;
-          if (sum && ok) atomicAdd(hist + static_cast<uint64_t>(row) * n_cnt + b, sum);
+          if (sum && ok && COFIE_BOUND(row < segs.rows))
+            atomicAdd(hist + static_cast<uint64_t>(row) * n_cnt + b, sum);
         }
       } else {
         for (uint32_t b = tid; b < L.bins; b += kNC) {
@@ -326,7 +330,8 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
             sum += rowp[idx];
             rowp[idx] = 0;
           }
-          if (sum && ok) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, sum);
+          if (sum && ok && COFIE_BOUND(row < segs.rows))
+            atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, sum);
         }
       }
       consumer_bar<kNC>();
@@ -355,11 +360,11 @@ __global__ void __launch_bounds__(kGenericThreads) hist_generic_kernel(SegTable 
     const uint8_t* px = frame + 3 * p;
     const uint32_t v = L.w[0] * px[0] + L.w[1] * px[1] + L.w[2] * px[2] + L.half;
     const uint32_t y = v / L.den;
-    atomicAdd(&cnt[(y * L.bins) >> 8], 1u);
+    if (COFIE_BOUND(((y * L.bins) >> 8) < L.bins)) atomicAdd(&cnt[(y * L.bins) >> 8], 1u);
   }
   __syncthreads();
   for (uint32_t b = threadIdx.x; b < L.bins; b += blockDim.x)
-    if (cnt[b]) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, cnt[b]);
+    if (cnt[b] && COFIE_BOUND(row < segs.rows)) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, cnt[b]);
 }
 
 }  // namespace
@@ -429,5 +434,7 @@ cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const L
   hist_generic_kernel<<<grid, kGenericThreads, 0, st>>>(segs, a, lc, hist);
   return cudaGetLastError();
 }
+
+uint32_t take_bounds_errors_hist() { return take_local_bounds_errors(); }
 
 }  // namespace cofie

@@ -77,7 +77,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
       uint32_t part = 0;
       for (uint32_t b = lane; b < B; b += 32) part += word_dist(c[b], p[b], a.dist_kind);
       part = __reduce_add_sync(0xffffffffu, part);
-      if (lane == 0) sadj[f] = part;
+      if (lane == 0 && COFIE_BOUND(f < kLazyMaxRows)) sadj[f] = part;
     }
   };
 
@@ -135,7 +135,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
           }
           code = d >= a.x_tau ? 1 : (scene ? 4 : 0);
         }
-        if (lane == 0) {
+        if (lane == 0 && COFIE_BOUND(f < kLazyMaxRows && (f + 1) * B <= kLazyTileWords)) {
           sd[f] = d;
           scode[f] = code;
         }
@@ -195,5 +195,7 @@ cudaError_t launch_lazy_select(const SegTable& segs, const SelectArgs& a, const 
   if (per <= 4) return launch_p<4>(segs, a, feat, ring, state, st);
   return launch_p<8>(segs, a, feat, ring, state, st);
 }
+
+uint32_t take_bounds_errors_lazy() { return take_local_bounds_errors(); }
 
 }  // namespace cofie

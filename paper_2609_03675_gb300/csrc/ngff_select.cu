@@ -59,7 +59,7 @@ __device__ __forceinline__ void window_row(uint32_t row, uint32_t lane, const Se
     const bool valid = k <= L && k <= t;
     const uint32_t* src = ct;
     if (valid)
-      src = (k <= j + sg.halo) ? hist + static_cast<uint64_t>(row - k) * B
+      src = (k <= j + sg.halo) ? (COFIE_BOUND(k <= row) ? hist + static_cast<uint64_t>(row - k) * B : ct)
                                : ring + (static_cast<uint64_t>(stream) * L + (t - k) % L) * B;
     uint32_t d = 0;
     if (kVec4) {
@@ -244,6 +244,7 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
       uint32_t g = gin;
 #pragma unroll 4
       for (uint32_t f = f0; f < f1; ++f) g = step_gap<kOneWord>(smask + f * W, g);
+      (void)COFIE_BOUND(g >= 1 && g <= L);  // a gap stays in [1, L_max]
       sexit[warp * L + gin - 1] = static_cast<uint16_t>(g);
     }
     __syncthreads();
@@ -268,7 +269,8 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
 #pragma unroll 4
     for (uint32_t f = tid; f < m; f += kScanThreads) {
       const uint32_t jj = tile0 + f;
-      const uint32_t g = sgap[f];
+      uint32_t g = sgap[f];
+      if (!COFIE_BOUND(g >= 1 && g <= L)) g = 1;  // checked build: keep the L1 read in its row
       const uint64_t r = static_cast<uint64_t>(row0 + jj) * L;
       const uint32_t lm = max(l1[r], l1[r + g - 1]);
       const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
@@ -385,6 +387,7 @@ __global__ void __launch_bounds__(kScanThreads) gap_map_kernel(Segment sg, Selec
     for (uint32_t gin = lane + 1; gin <= L; gin += 32) {
       uint32_t g = gin;
       for (uint32_t f = f0; f < f1; ++f) g = step_gap<kOneWord>(smask + f * W, g);
+      (void)COFIE_BOUND(g >= 1 && g <= L);  // a gap stays in [1, L_max]
       sexit[warp * L + gin - 1] = static_cast<uint16_t>(g);
     }
     __syncthreads();
@@ -492,5 +495,7 @@ cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint3
     select_small_kernel<false, false><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
   return cudaGetLastError();
 }
+
+uint32_t take_bounds_errors_select() { return take_local_bounds_errors(); }
 
 }  // namespace cofie
