@@ -4,7 +4,8 @@ Eq. 6 against a brute-force loop on tiny inputs and against the equivalent
 layout with every key head repeated per query head; Eq. 7 against closed
 forms (identical tokens, duplicated or permuted text tokens, positive
 scaling); Eq. 8 against its definition on special cases (rho = 0 and 1,
-halfway counts, ties) and a planted-evidence stream."""
+halfway counts, ties) and a planted-evidence stream; the score error bound
+against honest rounding and a case that reaches it."""
 import math
 
 import numpy as np
@@ -108,3 +109,22 @@ def test_score_bound_covers_bf16_group_sums():
     w_approx = approx.max(axis=0).reshape(-1, 8).mean(axis=1)
     w, _ = Q.run(q, k, 8, 0.5)
     assert np.all(np.abs(w_approx - w) <= Q.score_bound(q, k, 8))
+
+
+def test_score_bound_reached_by_a_rounding_worst_case():
+    """Two query heads in one group, 1 and 2^-8 in every component, sum to
+    1 + 2^-8, halfway between two bf16 values: the group sum rounds to 1 (half
+    to even) and every product has the same sign, so the error is the whole
+    2^-8 relative term: w = 1 + 2^-8 exactly, the group-sum path gives 1."""
+    d = 4
+    q = np.zeros((1, 2, d), dtype=np.float32)
+    q[:, 0, :], q[:, 1, :] = 1.0, 2.0 ** -8
+    q_bits = S.to_bf16_bits(q)
+    k_bits = S.to_bf16_bits(np.ones((3, 1, d), dtype=np.float32))
+    qg = Q.bf16_to_f64(S.to_bf16_bits(Q.bf16_to_f64(q_bits).sum(axis=1).astype(np.float32)))
+    assert qg[0, 0] == 1.0
+    w_group = (qg @ Q.bf16_to_f64(k_bits)[:, 0, :].T / (2 * np.sqrt(d))).max(axis=0).mean()
+    w, _ = Q.run(q_bits, k_bits, 3, 1.0)
+    assert w[0] == 1 + 2.0 ** -8 and w_group == 1.0
+    bound = Q.score_bound(q_bits, k_bits, 3)[0]
+    assert bound >= w[0] - w_group >= 0.99 * bound

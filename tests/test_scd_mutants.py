@@ -1,12 +1,10 @@
 """Plants one-spot mistakes in a copy of the scene-change oracle (on the CPU)
 and checks that the pins of test_scd_oracle catch each of them."""
-import inspect
-import types
-
 import pytest
 
 from oracle import scd_oracle as SC
 from tests import test_scd_oracle as PINS
+from tests.mutation import call, caught_by, mutant, pins
 
 MUTANTS = {
     "cut does not end the run": ("            flags[t] = True\n            acc = 0\n",
@@ -31,46 +29,13 @@ MUTANTS = {
 }
 
 
-def _mutant(src_from, src_to):
-    src = inspect.getsource(SC)
-    assert src_from in src, "mutation site not found"
-    mod = types.ModuleType("scd_mutant")
-    mod.__dict__["__name__"] = "scd_mutant"
-    exec(compile(src.replace(src_from, src_to, 1), "scd_mutant", "exec"), mod.__dict__)
-    return mod
-
-
-def _pins():
-    return [(n, f) for n, f in inspect.getmembers(PINS, inspect.isfunction) if n.startswith("test_")]
-
-
-def _call(fn):
-    marks = getattr(fn, "pytestmark", [])
-    params = [m for m in marks if m.name == "parametrize"]
-    if not params:
-        fn()
-        return
-    names = [s.strip() for s in params[0].args[0].split(",")]
-    for vals in params[0].args[1]:
-        vals = vals if isinstance(vals, tuple) else (vals,)
-        fn(**dict(zip(names, vals)))
-
-
 @pytest.mark.parametrize("name", sorted(MUTANTS))
 def test_each_mutant_is_caught(name, monkeypatch):
-    mod = _mutant(*MUTANTS[name])
-    monkeypatch.setattr(PINS, "SC", mod)
-    caught = []
-    for pin, fn in _pins():
-        try:
-            _call(fn)
-        except AssertionError:
-            caught.append(pin)
-    assert caught, f"mutant '{name}' passes every pin"
+    monkeypatch.setattr(PINS, "SC", mutant(SC, *MUTANTS[name]))
+    assert caught_by(PINS), f"mutant '{name}' passes every pin"
 
 
 def test_unmutated_copy_passes_every_pin(monkeypatch):
-    mod = _mutant("KEEP_SCENE = 4", "KEEP_SCENE = 4")
-    monkeypatch.setattr(PINS, "SC", mod)
-    for _, fn in _pins():
-        _call(fn)
+    monkeypatch.setattr(PINS, "SC", mutant(SC, "KEEP_SCENE = 4", "KEEP_SCENE = 4"))
+    for _, fn in pins(PINS):
+        call(fn)

@@ -72,3 +72,41 @@ def test_rule_special_cases(kind):
     for cut in (1, 9, 25):
         f2, s2, k2 = SO.run(frames[:cut], O.Params(W, H, tau=0.2), kind)
         assert np.array_equal(k2, k[:cut]) and np.array_equal(s2, s[:cut])
+
+
+def test_flat_frames_closed_forms():
+    """A flat frame has equal cell means everywhere: no dHash bit is set
+    (strict comparison), even where cells hold different pixel counts
+    (64 x 48 over 9 columns: 7 or 8 pixels). Black against white is the
+    largest low-res difference: d = 255 W H / (255 W H) = 1."""
+    H, W = 48, 64
+    p = O.Params(W, H)
+    for v in (0, 37, 255):
+        assert SO.features(_gray(np.full((H, W), v)), p, SO.DHASH).sum() == 0
+    black, white = _gray(np.zeros((H, W))), _gray(np.full((H, W), 255))
+    fa, fb = SO.features(black, p, SO.LOWRES), SO.features(white, p, SO.LOWRES)
+    assert SO.numerator(fa, fb, SO.LOWRES) / SO.denominator(p, SO.LOWRES) == 1.0
+
+
+def _hashes(*bit_sets):
+    """dHash feature rows with the given bits set."""
+    f = np.zeros((len(bit_sets), 64), dtype=np.int64)
+    for i, bits in enumerate(bit_sets):
+        f[i, list(bits)] = 1
+    return f
+
+
+def test_rule_terms_on_constructed_hashes():
+    """Only the adjacent term crosses tau: X and Y each differ from the
+    reference A in 16 bits (d = 0.25) and from each other in 32 (d = 0.5).
+    Only the reference term crosses: a drift of 8 bits per frame (adjacent
+    d = 0.125) reaches 24 bits from the reference (0.375) at frame 3, kept
+    also at tau = 0.375 (s >= tau, Eq. 5)."""
+    p = O.Params(16, 16, tau=0.4, l_max=100)
+    _, keep = SO.select(_hashes([], range(16), range(16, 32)), p, SO.DHASH)
+    assert list(keep) == [O.KEEP_FIRST, O.KEEP_DROP, O.KEEP_NOVELTY]
+    for tau in (0.3, 0.375):
+        p = O.Params(16, 16, tau=tau, l_max=100)
+        score, keep = SO.select(_hashes([], range(8), range(16), range(24), range(32)), p, SO.DHASH)
+        assert list(keep) == [O.KEEP_FIRST, O.KEEP_DROP, O.KEEP_DROP, O.KEEP_NOVELTY, O.KEEP_DROP]
+        assert list(score[1:]) == [0.125, 0.25, 0.375, 0.125]
