@@ -98,6 +98,12 @@ __device__ __noinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, uint64
   }
 }
 
+// The common case inline (the phase has already completed), the bounded
+// wait loop out of line.
+__device__ __forceinline__ bool mbar_wait_fast(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
+  return mbar_try(bar, parity) || mbar_wait_for(bar, parity, timeout_ns);
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int32_t x, int32_t y, uint32_t bar) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
@@ -360,25 +366,30 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
   if (warp == 0) {
     if (lane == 0) {
       // --------------------------------------------------------- TMA producer
-      uint32_t g = 0;  // chunk counter over all of this CTA's tiles
-      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
-        const uint32_t row0 = (blockIdx.x + t * gridDim.x) * kQerTile;
+      const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
+      uint32_t g = 0, s = 0, ph = 0;  // chunk counter over all of this CTA's tiles; ring slot and phase
+      bool stop = false;
+      for (uint32_t t = 0; t < my_tiles && !stop; ++t) {
+        const int32_t row0 = static_cast<int32_t>((blockIdx.x + t * gridDim.x) * kQerTile);
         for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
-          const uint32_t s = g % n_stages, use = g / n_stages;
-          if (use > 0 && !mbar_wait_for(smem_u32(&empty_bar[s]), (use - 1) & 1, timeout_ns)) {
+          if (g >= n_stages && !mbar_wait_fast(empty0 + 8 * s, ph ^ 1, timeout_ns)) {
             atomicOr(err, kQerErrProducer);
             abort_flag = 1;
+            stop = true;
             break;
           }
-          if (abort_flag) break;
-          const uint32_t fb = smem_u32(&full_bar[s]);
+          const uint32_t fb = full0 + 8 * s;
           asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(fb), "r"(a_bytes + b_bytes)
                        : "memory");
-          const uint32_t base = smem_u32(smem + s * stage_bytes);
+          const uint32_t base = ring0 + s * stage_bytes;
           const int32_t x = static_cast<int32_t>(kc * kQerKChunk);
-          tma_load_2d(base, &map_k, x, static_cast<int32_t>(row0), fb);
-          tma_load_2d(base + half_bytes, &map_k, x, static_cast<int32_t>(row0 + kQerM), fb);
+          tma_load_2d(base, &map_k, x, row0, fb);
+          tma_load_2d(base + half_bytes, &map_k, x, row0 + kQerM, fb);
           tma_load_2d(base + a_bytes, &map_q, x, 0, fb);
+          if (++s == n_stages) {
+            s = 0;
+            ph ^= 1;
+          }
         }
       }
       // no copy may still be writing shared memory when the CTA exits
@@ -389,35 +400,44 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
   } else if (warp == 1) {
     if (lane == 0) {
       // ----------------------------------------------------------- MMA issuer
+      // Per stage: one inline try of the full barrier, descriptors formed
+      // once and stepped by the 32-byte K offset (the ring lies below 256
+      // KiB, so the descriptor's 14-bit address field never carries).
       const uint32_t idesc = idesc_bf16_f32(kQerM, n_pad);
-      uint32_t g = 0;
-      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
+      const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
+      uint32_t s = 0, ph = 0;
+      bool stop = false;
+      for (uint32_t t = 0; t < my_tiles && !stop && !abort_flag; ++t) {
         const uint32_t b = t % n_buf, ub = t / n_buf;
-        if (ub > 0 && !mbar_wait_for(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
+        if (ub > 0 && !mbar_wait_fast(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
           atomicOr(err, kQerErrMma);
           abort_flag = 1;
           break;
         }
         tc_fence_after();
         const uint32_t acc0 = tmem + b * 2 * acc_cols, acc1 = acc0 + acc_cols;
-        bool stop = false;
-        for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
-          const uint32_t s = g % n_stages, use = g / n_stages;
-          if (!mbar_wait_for(smem_u32(&full_bar[s]), use & 1, timeout_ns) || abort_flag) {
+        for (uint32_t kc = 0; kc < n_chunks; ++kc) {
+          if (!mbar_wait_fast(full0 + 8 * s, ph, timeout_ns)) {
             atomicOr(err, kQerErrMma);
             abort_flag = 1;
             stop = true;
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(smem + s * stage_bytes), a1 = a0 + half_bytes, b0 = a0 + a_bytes;
+          const uint32_t a0 = ring0 + s * stage_bytes;
+          const uint64_t da0 = sw128_desc(a0), da1 = sw128_desc(a0 + half_bytes), db = sw128_desc(a0 + a_bytes);
+          const uint32_t first = kc != 0;  // 0: the tile's first MMAs overwrite the accumulators
 #pragma unroll
           for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk) {
-            const uint64_t bd = sw128_desc(b0 + kk * 32);
-            umma_bf16(acc0, sw128_desc(a0 + kk * 32), bd, idesc, (kc | kk) != 0);
-            umma_bf16(acc1, sw128_desc(a1 + kk * 32), bd, idesc, (kc | kk) != 0);
+            const uint64_t o = kk * (kQerUmmaK * 2 / 16);
+            umma_bf16(acc0, da0 + o, db + o, idesc, kk ? 1u : first);
+            umma_bf16(acc1, da1 + o, db + o, idesc, kk ? 1u : first);
           }
-          umma_commit(smem_u32(&empty_bar[s]));  // the stage is free once these MMAs have read it
+          umma_commit(empty0 + 8 * s);  // the stage is free once these MMAs have read it
+          if (++s == n_stages) {
+            s = 0;
+            ph ^= 1;
+          }
         }
         if (stop) break;
         umma_commit(smem_u32(&tfull_bar[b]));  // accumulator pair b holds tile t
@@ -466,8 +486,8 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
 
 // Paired-SM scoring kernel (tcgen05 cta_group::2; clusters of two CTAs on two
 // SMs). The pair covers a 256-token tile with one M = 256 MMA per 16-wide K
-// step (a ring stage holds n_sub 64-wide K chunks, so 4 n_sub MMAs): CTA rank r stages key rows [128 r, 128 r + 128) of the tile (A) and
-// q~ rows [r n_pad / 2, (r + 1) n_pad / 2) (half of B); the MMA, issued by
+// step (a ring stage holds kSub 64-wide K chunks, so 4 kSub MMAs): CTA rank
+// r stages key rows [128 r, 128 r + 128) of the tile (A) and q~ rows [r n_pad / 2, (r + 1) n_pad / 2) (half of B); the MMA, issued by
 // rank 0, reads both CTAs' halves and writes each CTA's 128 token rows x
 // n_pad text columns into that CTA's TMEM. Against the one-SM kernel this
 // halves the shared-memory reads of q~ per SM (each half of B is read once
@@ -478,15 +498,17 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
 // the paired form of the tensor copy), which rank 0's producer arms with the
 // bytes of both; rank 0's MMA thread waits on it alone, and commits MMA
 // completion to the empty barriers and accumulator barriers of both CTAs at
-// once (multicast). The epilogue warps of both CTAs arrive on rank 0's
-// tempty barrier. Every wait is bounded, and both CTAs always meet at a
+// once (multicast). The ring barriers are completed by the asynchronous
+// proxy only (copy bytes, MMA commits), so their waits are CTA-scoped; the
+// tempty barrier, on which the epilogue warps of both CTAs arrive, is waited
+// on at cluster scope. Every wait is bounded, and both CTAs always meet at a
 // final cluster barrier before TMEM is freed.
+template <uint32_t kSub>
 __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_constant__ CUtensorMap map_k,
                                                               const __grid_constant__ CUtensorMap map_qh,
                                                               uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
-                                                              uint32_t acc_cols, uint32_t n_stages, uint32_t n_sub,
-                                                              uint32_t n_chunks, uint32_t n_tiles,
-                                                              float* __restrict__ colmax,
+                                                              uint32_t acc_cols, uint32_t n_stages, uint32_t n_chunks,
+                                                              uint32_t n_tiles, float* __restrict__ colmax,
                                                               uint32_t* __restrict__ err, uint64_t timeout_ns) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kQerMaxStages];
@@ -503,7 +525,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
   const uint32_t half_rows = n_pad / 2;
   const uint32_t a_bytes = kQerM * 128, b_bytes = half_rows * 128;
   const uint32_t sub_bytes = (a_bytes + b_bytes + 1023) & ~1023u;  // one 64-wide K chunk of A and B
-  const uint32_t stage_bytes = n_sub * sub_bytes;                    // a ring stage: n_sub chunks
+  const uint32_t stage_bytes = kSub * sub_bytes;                     // a ring stage: kSub chunks
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t my_tiles = pair < n_tiles ? (n_tiles - 1 - pair) / n_pairs + 1 : 0;
   const uint32_t tmem_total = 2 * acc_cols;  // two accumulators
@@ -537,28 +559,34 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------ TMA producer (both CTAs)
-      uint32_t g = 0;
-      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
-        const uint32_t row0 = (pair + t * n_pairs) * kQerTile + rank * kQerM;
+      // The ring slot s and its phase ph advance incrementally; a wait that
+      // runs out stops this thread (the other roles then run out on theirs).
+      const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
+      const uint32_t full0_rank0 = map_to_rank(full0, 0);  // rank 0's full barriers count both CTAs' bytes
+      const uint32_t tx = 2 * kSub * (a_bytes + b_bytes);
+      uint32_t g = 0, s = 0, ph = 0;
+      bool stop = false;
+      for (uint32_t t = 0; t < my_tiles && !stop; ++t) {
+        const int32_t row0 = static_cast<int32_t>((pair + t * n_pairs) * kQerTile + rank * kQerM);
         for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
-          const uint32_t s = g % n_stages, use = g / n_stages;
-          if (use > 0 && !mbar_wait_cluster(smem_u32(&empty_bar[s]), (use - 1) & 1, timeout_ns)) {
+          if (g >= n_stages && !mbar_wait_fast(empty0 + 8 * s, ph ^ 1, timeout_ns)) {
             atomicOr(err, kQerErrProducer);
             abort_flag = 1;
+            stop = true;
             break;
           }
-          if (abort_flag) break;
-          const uint32_t fb0 = map_to_rank(smem_u32(&full_bar[s]), 0);  // rank 0's full barrier
           if (rank == 0)
-            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(&full_bar[s])),
-                         "r"(2 * n_sub * (a_bytes + b_bytes))
-                         : "memory");
-          const uint32_t base = smem_u32(smem + s * stage_bytes);
-          for (uint32_t sub = 0; sub < n_sub; ++sub) {
-            const int32_t x = static_cast<int32_t>((kc * n_sub + sub) * kQerKChunk);
-            const uint32_t b = base + sub * sub_bytes;
-            tma_load_2d_pair(b, &map_k, x, static_cast<int32_t>(row0), fb0);
-            tma_load_2d_pair(b + a_bytes, &map_qh, x, static_cast<int32_t>(rank * half_rows), fb0);
+            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(full0 + 8 * s), "r"(tx) : "memory");
+          const uint32_t base = ring0 + s * stage_bytes, fb = full0_rank0 + 8 * s;
+#pragma unroll
+          for (uint32_t sub = 0; sub < kSub; ++sub) {
+            const int32_t x = static_cast<int32_t>((kc * kSub + sub) * kQerKChunk);
+            tma_load_2d_pair(base + sub * sub_bytes, &map_k, x, row0, fb);
+            tma_load_2d_pair(base + sub * sub_bytes + a_bytes, &map_qh, x, static_cast<int32_t>(rank * half_rows), fb);
+          }
+          if (++s == n_stages) {
+            s = 0;
+            ph ^= 1;
           }
         }
       }
@@ -572,9 +600,18 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
       // ------------------------------------------------ MMA issuer (rank 0)
+      // One thread issues every MMA of the pair, so its per-stage work is
+      // kept small: the ring slot and phase advance incrementally, the first
+      // try of each wait is inline, and each stage's shared-memory
+      // descriptors are formed once and stepped by the 32-byte K offset
+      // (2 in the descriptor's 16-byte address units; the ring lies below
+      // 256 KiB, so the 14-bit address field never carries).
       const uint32_t idesc = idesc_bf16_f32(2 * kQerM, n_pad);
-      uint32_t g = 0;
-      for (uint32_t t = 0; t < my_tiles && !abort_flag; ++t) {
+      const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
+      const uint64_t sub16 = sub_bytes >> 4;
+      uint32_t s = 0, ph = 0;
+      bool stop = false;
+      for (uint32_t t = 0; t < my_tiles && !stop && !abort_flag; ++t) {
         const uint32_t b = t & 1, ub = t >> 1;
         if (ub > 0 && !mbar_wait_cluster(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
           atomicOr(err, kQerErrMma);
@@ -583,25 +620,29 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
         }
         tc_fence_after();
         const uint32_t acc = tmem + b * acc_cols;
-        bool stop = false;
-        for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
-          const uint32_t s = g % n_stages, use = g / n_stages;
-          if (!mbar_wait_cluster(smem_u32(&full_bar[s]), use & 1, timeout_ns) || abort_flag) {
+        for (uint32_t kc = 0; kc < n_chunks; ++kc) {
+          if (!mbar_wait_fast(full0 + 8 * s, ph, timeout_ns)) {
             atomicOr(err, kQerErrMma);
             abort_flag = 1;
             stop = true;
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(smem + s * stage_bytes), b0 = a0 + a_bytes;
-          for (uint32_t sub = 0; sub < n_sub; ++sub) {
+          const uint32_t a0 = ring0 + s * stage_bytes;
+          const uint64_t da = sw128_desc(a0), db = sw128_desc(a0 + a_bytes);
+          const uint32_t first = kc != 0;  // 0: the tile's first MMA overwrites the accumulator
+#pragma unroll
+          for (uint32_t sub = 0; sub < kSub; ++sub)
 #pragma unroll
             for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk) {
-              const uint32_t o = sub * sub_bytes + kk * 32;
-              umma_pair_bf16(acc, sw128_desc(a0 + o), sw128_desc(b0 + o), idesc, (kc | sub | kk) != 0);
+              const uint64_t o = sub * sub16 + kk * (kQerUmmaK * 2 / 16);
+              umma_pair_bf16(acc, da + o, db + o, idesc, (sub | kk) ? 1u : first);
             }
+          umma_pair_commit_both(empty0 + 8 * s);  // both CTAs' slot s is free once read
+          if (++s == n_stages) {
+            s = 0;
+            ph ^= 1;
           }
-          umma_pair_commit_both(smem_u32(&empty_bar[s]));  // both CTAs' slot s is free once read
         }
         if (stop) break;
         umma_pair_commit_both(smem_u32(&tfull_bar[b]));  // accumulator b holds tile t in both CTAs
@@ -894,7 +935,8 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
     h->pair_smem = static_cast<size_t>(h->pair_stages) * qer_pair_stage_bytes(h->n_pad, h->pair_sub) + 1024;
     const int pair_ctas_by_tmem = static_cast<int>(512 / (2 * h->acc_cols));
     while (per_sm / (h->pair_smem + 1024) > static_cast<size_t>(pair_ctas_by_tmem)) h->pair_smem += 1024;
-    cudaError_t pe = cudaFuncSetAttribute(qer_score_pair, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    const auto pair_fn = h->pair_sub == 2 ? qer_score_pair<2> : qer_score_pair<1>;  // the one launched
+    cudaError_t pe = cudaFuncSetAttribute(pair_fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           static_cast<int>(h->pair_smem));
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -908,7 +950,7 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int clusters = 0;
-    if (pe == cudaSuccess) pe = cudaOccupancyMaxActiveClusters(&clusters, qer_score_pair, &cfg);
+    if (pe == cudaSuccess) pe = cudaOccupancyMaxActiveClusters(&clusters, pair_fn, &cfg);
     if (pe == cudaSuccess && clusters >= 1) {
       h->pair = true;
       h->pair_clusters = clusters;
@@ -1004,9 +1046,13 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
     cfg.stream = st;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, qer_score_pair, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad, h->acc_cols,
-                       h->pair_stages, h->pair_sub, h->D / kQerKChunk / h->pair_sub, tiles, h->d_colmax, h->d_err,
-                       2000000000ull);
+    const uint32_t n_chunks = h->D / kQerKChunk / h->pair_sub;
+    if (h->pair_sub == 2)
+      cudaLaunchKernelEx(&cfg, qer_score_pair<2>, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
+                         h->acc_cols, h->pair_stages, n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
+    else
+      cudaLaunchKernelEx(&cfg, qer_score_pair<1>, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
+                         h->acc_cols, h->pair_stages, n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
   } else {
     qer_score<<<grid, kQerThreads, h->smem, st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
                                                   h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles,
