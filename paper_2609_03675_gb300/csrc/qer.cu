@@ -59,6 +59,9 @@ constexpr size_t kQerStageBudget = 200 * 1024;  // shared memory for the ring
 constexpr int kQerUmmaK = 16;       // K of one tcgen05.mma for 16-bit inputs
 constexpr int kQerEpiWarps = 4;    // epilogue warps: TMEM lanes 0..127
 constexpr int kQerThreads = 32 * (2 + kQerEpiWarps);  // + TMA producer warp + MMA issuer warp
+constexpr int kQerPairThreads = kQerThreads + 32;     // paired kernel: + a second producer warp (q~)
+constexpr size_t kQerPairRingBudget = 224 * 1024;     // paired kernel: both rings (one CTA per SM)
+constexpr uint32_t kQerPairQSlots = 3;                // q~ slots: enough to cover its L2 latency
 constexpr uint32_t kQerMaxN = 256;  // text tokens (MMA N) per CTA
 constexpr int kSelThreads = 1024;
 constexpr int kRankThreads = 256;  // 8 frames per CTA (a warp each): the O(m^2) ranking spreads over many SMs
@@ -486,17 +489,25 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
 
 // Paired-SM scoring kernel (tcgen05 cta_group::2; clusters of two CTAs on two
 // SMs). The pair covers a 256-token tile with one M = 256 MMA per 16-wide K
-// step (a ring stage holds kSub 64-wide K chunks, so 4 kSub MMAs): CTA rank
-// r stages key rows [128 r, 128 r + 128) of the tile (A) and q~ rows [r n_pad / 2, (r + 1) n_pad / 2) (half of B); the MMA, issued by
+// step: CTA rank r stages key rows [128 r, 128 r + 128) of the tile (A) and
+// q~ rows [r n_pad / 2, (r + 1) n_pad / 2) (half of B); the MMA, issued by
 // rank 0, reads both CTAs' halves and writes each CTA's 128 token rows x
 // n_pad text columns into that CTA's TMEM. Against the one-SM kernel this
 // halves the shared-memory reads of q~ per SM (each half of B is read once
 // for both SMs) and needs one accumulator of acc_cols columns per tile, so
 // two of them overlap a tile's epilogue with the next tile's MMAs.
-// Synchronisation: each CTA's TMA thread fills its own ring slot, and both
-// CTAs' copies count their bytes on rank 0's full barrier (rank 1 through
-// the paired form of the tensor copy), which rank 0's producer arms with the
-// bytes of both; rank 0's MMA thread waits on it alone, and commits MMA
+//
+// Keys and q~ stream through two rings of kSub 64-wide K chunks per slot:
+// keys come from DRAM and want as many bytes in flight as shared memory
+// allows, q~ (the same for every tile) comes from L2 and needs only the few
+// slots that cover its L2 latency, so the q~ chunks do not take key slots.
+// Warp 0 streams keys, the last warp q~, warp 1 (rank 0) issues the MMAs,
+// warps 2..5 are the epilogue.
+//
+// Synchronisation: each CTA's producers fill their own ring slots, and both
+// CTAs' copies count their bytes on rank 0's full barriers (rank 1 through
+// the paired form of the tensor copy), which rank 0's producers arm with the
+// bytes of both; rank 0's MMA thread waits on them alone, and commits MMA
 // completion to the empty barriers and accumulator barriers of both CTAs at
 // once (multicast). The ring barriers are completed by the asynchronous
 // proxy only (copy bytes, MMA commits), so their waits are CTA-scoped; the
@@ -504,15 +515,15 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
 // on at cluster scope. Every wait is bounded, and both CTAs always meet at a
 // final cluster barrier before TMEM is freed.
 template <uint32_t kSub>
-__global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_constant__ CUtensorMap map_k,
-                                                              const __grid_constant__ CUtensorMap map_qh,
-                                                              uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
-                                                              uint32_t acc_cols, uint32_t n_stages, uint32_t n_chunks,
-                                                              uint32_t n_tiles, float* __restrict__ colmax,
-                                                              uint32_t* __restrict__ err, uint64_t timeout_ns) {
+__global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
+    const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_qh, uint32_t n_visual,
+    uint32_t n_text, uint32_t n_pad, uint32_t acc_cols, uint32_t n_kst, uint32_t n_qst, uint32_t n_chunks,
+    uint32_t n_tiles, float* __restrict__ colmax, uint32_t* __restrict__ err, uint64_t timeout_ns) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t full_bar[kQerMaxStages];
-  __shared__ __align__(8) uint64_t empty_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t kfull_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t kempty_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t qfull_bar[kQerMaxStages];
+  __shared__ __align__(8) uint64_t qempty_bar[kQerMaxStages];
   __shared__ __align__(8) uint64_t tfull_bar[2];
   __shared__ __align__(8) uint64_t tempty_bar[2];
   __shared__ __align__(8) uint64_t done_bar;
@@ -523,12 +534,12 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
   const uint32_t rank = cluster_ctarank();
   const uint32_t n_pairs = gridDim.x / 2, pair = blockIdx.x / 2;
   const uint32_t half_rows = n_pad / 2;
-  const uint32_t a_bytes = kQerM * 128, b_bytes = half_rows * 128;
-  const uint32_t sub_bytes = (a_bytes + b_bytes + 1023) & ~1023u;  // one 64-wide K chunk of A and B
-  const uint32_t stage_bytes = kSub * sub_bytes;                     // a ring stage: kSub chunks
+  const uint32_t a_chunk = kQerM * 128, b_chunk = half_rows * 128;  // one 64-wide K chunk of A / of half of B
+  const uint32_t kslot = kSub * a_chunk, qslot = kSub * b_chunk;
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t my_tiles = pair < n_tiles ? (n_tiles - 1 - pair) / n_pairs + 1 : 0;
   const uint32_t tmem_total = 2 * acc_cols;  // two accumulators
+  const uint32_t kring0 = smem_u32(smem), qring0 = kring0 + n_kst * kslot;
 
   if (warp == 0) {  // one warp in each CTA of the pair allocates, together
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
@@ -537,9 +548,13 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
   if (threadIdx.x == 32) {
-    for (uint32_t s = 0; s < n_stages; ++s) {
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&full_bar[s])) : "memory");
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&empty_bar[s])) : "memory");
+    for (uint32_t i = 0; i < n_kst; ++i) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&kfull_bar[i])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&kempty_bar[i])) : "memory");
+    }
+    for (uint32_t i = 0; i < n_qst; ++i) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&qfull_bar[i])) : "memory");
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&qempty_bar[i])) : "memory");
     }
     for (int b = 0; b < 2; ++b) {
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(&tfull_bar[b])) : "memory");
@@ -556,20 +571,26 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
   tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
-  if (warp == 0) {
+  if (warp == 0 || warp == kQerPairThreads / 32 - 1) {
     if (lane == 0) {
-      // ------------------------------------------------ TMA producer (both CTAs)
-      // The ring slot s and its phase ph advance incrementally; a wait that
-      // runs out stops this thread (the other roles then run out on theirs).
-      const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
+      // ----------------------------- producers (both CTAs): warp 0 keys, last warp q~
+      // Slot s and its phase ph advance incrementally; a wait that runs out
+      // stops this thread (the other roles then run out on theirs).
+      const bool keys = warp == 0;
+      const uint32_t n_slots = keys ? n_kst : n_qst, slot_bytes = keys ? kslot : qslot;
+      const uint32_t chunk = keys ? a_chunk : b_chunk, ring0 = keys ? kring0 : qring0;
+      const uint32_t empty0 = smem_u32(keys ? &kempty_bar[0] : &qempty_bar[0]);
+      const uint32_t full0 = smem_u32(keys ? &kfull_bar[0] : &qfull_bar[0]);
       const uint32_t full0_rank0 = map_to_rank(full0, 0);  // rank 0's full barriers count both CTAs' bytes
-      const uint32_t tx = 2 * kSub * (a_bytes + b_bytes);
+      const CUtensorMap* map = keys ? &map_k : &map_qh;
+      const uint32_t tx = 2 * kSub * chunk;
       uint32_t g = 0, s = 0, ph = 0;
       bool stop = false;
       for (uint32_t t = 0; t < my_tiles && !stop; ++t) {
-        const int32_t row0 = static_cast<int32_t>((pair + t * n_pairs) * kQerTile + rank * kQerM);
+        const int32_t y = keys ? static_cast<int32_t>((pair + t * n_pairs) * kQerTile + rank * kQerM)
+                               : static_cast<int32_t>(rank * half_rows);
         for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
-          if (g >= n_stages && !mbar_wait_fast(empty0 + 8 * s, ph ^ 1, timeout_ns)) {
+          if (g >= n_slots && !mbar_wait_fast(empty0 + 8 * s, ph ^ 1, timeout_ns)) {
             atomicOr(err, kQerErrProducer);
             abort_flag = 1;
             stop = true;
@@ -577,14 +598,11 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
           }
           if (rank == 0)
             asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(full0 + 8 * s), "r"(tx) : "memory");
-          const uint32_t base = ring0 + s * stage_bytes, fb = full0_rank0 + 8 * s;
+          const uint32_t base = ring0 + s * slot_bytes, fb = full0_rank0 + 8 * s;
 #pragma unroll
-          for (uint32_t sub = 0; sub < kSub; ++sub) {
-            const int32_t x = static_cast<int32_t>((kc * kSub + sub) * kQerKChunk);
-            tma_load_2d_pair(base + sub * sub_bytes, &map_k, x, row0, fb);
-            tma_load_2d_pair(base + sub * sub_bytes + a_bytes, &map_qh, x, static_cast<int32_t>(rank * half_rows), fb);
-          }
-          if (++s == n_stages) {
+          for (uint32_t sub = 0; sub < kSub; ++sub)
+            tma_load_2d_pair(base + sub * chunk, map, static_cast<int32_t>((kc * kSub + sub) * kQerKChunk), y, fb);
+          if (++s == n_slots) {
             s = 0;
             ph ^= 1;
           }
@@ -593,23 +611,23 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
       // no copy may still be writing shared memory when the CTA exits: the
       // last copies of every slot were read by MMAs whose completion reached
       // this CTA's empty barrier
-      for (uint32_t j = g > n_stages ? g - n_stages : 0; j < g; ++j)
-        if (!mbar_wait_cluster(smem_u32(&empty_bar[j % n_stages]), (j / n_stages) & 1, timeout_ns))
-          atomicOr(err, kQerErrDrain);
+      for (uint32_t j = g > n_slots ? g - n_slots : 0; j < g; ++j)
+        if (!mbar_wait_cluster(empty0 + 8 * (j % n_slots), (j / n_slots) & 1, timeout_ns)) atomicOr(err, kQerErrDrain);
     }
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
       // ------------------------------------------------ MMA issuer (rank 0)
       // One thread issues every MMA of the pair, so its per-stage work is
-      // kept small: the ring slot and phase advance incrementally, the first
-      // try of each wait is inline, and each stage's shared-memory
-      // descriptors are formed once and stepped by the 32-byte K offset
-      // (2 in the descriptor's 16-byte address units; the ring lies below
-      // 256 KiB, so the 14-bit address field never carries).
+      // kept small: slots and phases advance incrementally, the first try of
+      // each wait is inline, and each stage's shared-memory descriptors are
+      // formed once and stepped by the 32-byte K offset (2 in the
+      // descriptor's 16-byte address units; the rings lie below 256 KiB, so
+      // the 14-bit address field never carries).
       const uint32_t idesc = idesc_bf16_f32(2 * kQerM, n_pad);
-      const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
-      const uint64_t sub16 = sub_bytes >> 4;
-      uint32_t s = 0, ph = 0;
+      const uint32_t kfull0 = smem_u32(&kfull_bar[0]), kempty0 = smem_u32(&kempty_bar[0]);
+      const uint32_t qfull0 = smem_u32(&qfull_bar[0]), qempty0 = smem_u32(&qempty_bar[0]);
+      const uint64_t a16 = a_chunk >> 4, b16 = b_chunk >> 4;
+      uint32_t ks = 0, kph = 0, qs = 0, qph = 0;
       bool stop = false;
       for (uint32_t t = 0; t < my_tiles && !stop && !abort_flag; ++t) {
         const uint32_t b = t & 1, ub = t >> 1;
@@ -621,27 +639,31 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
         tc_fence_after();
         const uint32_t acc = tmem + b * acc_cols;
         for (uint32_t kc = 0; kc < n_chunks; ++kc) {
-          if (!mbar_wait_fast(full0 + 8 * s, ph, timeout_ns)) {
+          if (!mbar_wait_fast(kfull0 + 8 * ks, kph, timeout_ns) || !mbar_wait_fast(qfull0 + 8 * qs, qph, timeout_ns)) {
             atomicOr(err, kQerErrMma);
             abort_flag = 1;
             stop = true;
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = ring0 + s * stage_bytes;
-          const uint64_t da = sw128_desc(a0), db = sw128_desc(a0 + a_bytes);
+          const uint64_t da = sw128_desc(kring0 + ks * kslot), db = sw128_desc(qring0 + qs * qslot);
           const uint32_t first = kc != 0;  // 0: the tile's first MMA overwrites the accumulator
 #pragma unroll
           for (uint32_t sub = 0; sub < kSub; ++sub)
 #pragma unroll
             for (uint32_t kk = 0; kk < kQerKChunk / kQerUmmaK; ++kk) {
-              const uint64_t o = sub * sub16 + kk * (kQerUmmaK * 2 / 16);
-              umma_pair_bf16(acc, da + o, db + o, idesc, (sub | kk) ? 1u : first);
+              const uint64_t o = kk * (kQerUmmaK * 2 / 16);
+              umma_pair_bf16(acc, da + sub * a16 + o, db + sub * b16 + o, idesc, (sub | kk) ? 1u : first);
             }
-          umma_pair_commit_both(empty0 + 8 * s);  // both CTAs' slot s is free once read
-          if (++s == n_stages) {
-            s = 0;
-            ph ^= 1;
+          umma_pair_commit_both(kempty0 + 8 * ks);  // both CTAs' slots are free once read
+          umma_pair_commit_both(qempty0 + 8 * qs);
+          if (++ks == n_kst) {
+            ks = 0;
+            kph ^= 1;
+          }
+          if (++qs == n_qst) {
+            qs = 0;
+            qph ^= 1;
           }
         }
         if (stop) break;
@@ -651,7 +673,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score_pair(const __grid_const
     }
   } else {
     // ------------------------------------------------------ epilogue (both CTAs)
-    const uint32_t quarter = warp & 3;
+    const uint32_t quarter = warp & 3;  // warps 2..5: TMEM lanes 32 (warp % 4) ..
     const uint32_t tempty0 = map_to_rank(smem_u32(&tempty_bar[0]), 0);
     const uint32_t tempty1 = map_to_rank(smem_u32(&tempty_bar[1]), 0);
     for (uint32_t t = 0; t < my_tiles; ++t) {
@@ -761,14 +783,17 @@ uint32_t qer_stages(uint32_t n_pad) {
   return static_cast<uint32_t>(n < kQerMaxStages ? n : kQerMaxStages);
 }
 
-// A ring stage of the paired kernel holds n_sub 64-wide K chunks of A and B.
-uint32_t qer_pair_stage_bytes(uint32_t n_pad, uint32_t n_sub) {
-  return n_sub * ((kQerM * 128 + (n_pad / 2) * 128 + 1023) & ~1023u);
+// Key slots of the paired kernel: as many n_sub-chunk slots of 128 key rows
+// as fit the ring budget beside kQerPairQSlots q~ slots (n_sub chunks of
+// n_pad / 2 rows), at most kQerMaxStages.
+uint32_t qer_pair_key_slots(uint32_t n_pad, uint32_t n_sub) {
+  const size_t kslot = static_cast<size_t>(n_sub) * kQerM * 128, qslot = static_cast<size_t>(n_sub) * (n_pad / 2) * 128;
+  const size_t n = (kQerPairRingBudget - kQerPairQSlots * qslot) / kslot;
+  return static_cast<uint32_t>(n < kQerMaxStages ? n : kQerMaxStages);
 }
 
-uint32_t qer_pair_stages(uint32_t n_pad, uint32_t n_sub) {
-  const size_t n = kQerStageBudget / qer_pair_stage_bytes(n_pad, n_sub);
-  return static_cast<uint32_t>(n < kQerMaxStages ? n : kQerMaxStages);
+size_t qer_pair_smem_bytes(uint32_t n_pad, uint32_t n_sub, uint32_t key_slots) {
+  return static_cast<size_t>(n_sub) * (key_slots * kQerM * 128 + kQerPairQSlots * (n_pad / 2) * 128) + 1024;
 }
 
 size_t qer_smem_bytes(uint32_t n_pad) {
@@ -813,7 +838,7 @@ struct cofie_qer {
   int grid = 0;          // persistent CTAs
   size_t smem = 0;       // dynamic shared memory per CTA
   bool pair = false;     // the paired-SM kernel (clusters of two CTAs)
-  uint32_t pair_stages = 0, pair_sub = 1;
+  uint32_t pair_key_slots = 0, pair_sub = 1;
   int pair_clusters = 0;  // co-resident clusters
   size_t pair_smem = 0;
   __nv_bfloat16_raw* d_qg = nullptr;
@@ -931,8 +956,8 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
     // two 64-wide K chunks per ring stage when D allows: every stage costs a
     // fixed synchronisation overhead, which more MMAs per stage amortise
     h->pair_sub = (h->D / kQerKChunk) % 2 == 0 ? 2 : 1;
-    h->pair_stages = qer_pair_stages(h->n_pad, h->pair_sub);
-    h->pair_smem = static_cast<size_t>(h->pair_stages) * qer_pair_stage_bytes(h->n_pad, h->pair_sub) + 1024;
+    h->pair_key_slots = qer_pair_key_slots(h->n_pad, h->pair_sub);
+    h->pair_smem = qer_pair_smem_bytes(h->n_pad, h->pair_sub, h->pair_key_slots);
     const int pair_ctas_by_tmem = static_cast<int>(512 / (2 * h->acc_cols));
     while (per_sm / (h->pair_smem + 1024) > static_cast<size_t>(pair_ctas_by_tmem)) h->pair_smem += 1024;
     const auto pair_fn = h->pair_sub == 2 ? qer_score_pair<2> : qer_score_pair<1>;  // the one launched
@@ -945,7 +970,7 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
     attr[0].val.clusterDim.z = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * n_sms, 1, 1);
-    cfg.blockDim = dim3(kQerThreads, 1, 1);
+    cfg.blockDim = dim3(kQerPairThreads, 1, 1);
     cfg.dynamicSmemBytes = h->pair_smem;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
@@ -1041,7 +1066,7 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
     attr[0].val.clusterDim.z = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * clusters, 1, 1);
-    cfg.blockDim = dim3(kQerThreads, 1, 1);
+    cfg.blockDim = dim3(kQerPairThreads, 1, 1);
     cfg.dynamicSmemBytes = h->pair_smem;
     cfg.stream = st;
     cfg.attrs = attr;
@@ -1049,10 +1074,12 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
     const uint32_t n_chunks = h->D / kQerKChunk / h->pair_sub;
     if (h->pair_sub == 2)
       cudaLaunchKernelEx(&cfg, qer_score_pair<2>, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
-                         h->acc_cols, h->pair_stages, n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
+                         h->acc_cols, h->pair_key_slots, kQerPairQSlots, n_chunks, tiles, h->d_colmax, h->d_err,
+                         2000000000ull);
     else
       cudaLaunchKernelEx(&cfg, qer_score_pair<1>, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
-                         h->acc_cols, h->pair_stages, n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
+                         h->acc_cols, h->pair_key_slots, kQerPairQSlots, n_chunks, tiles, h->d_colmax, h->d_err,
+                         2000000000ull);
   } else {
     qer_score<<<grid, kQerThreads, h->smem, st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
                                                   h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles,
