@@ -14,7 +14,7 @@
 // that is kept: the text-by-vision score matrix is never written to memory,
 // which is the point of the paper's tiled computation.
 //
-// Kernels:
+// Kernels (one QER call launches four):
 //   qer_prepare_q   q [n_text][H][d] -> q~ [N][D] bf16 (fp32 sums rounded to
 //                   nearest even; rows n_text..N-1 zero, N = n_text rounded up to 16)
 //   qer_score       persistent CTAs over tiles of 256 visual tokens: TMA
@@ -24,13 +24,16 @@
 //                   half tile, N, K = 16) into TMEM accumulators (128 lanes x N
 //                   fp32 columns per half) and commits each stage back to the
 //                   producer; four epilogue warps read the accumulators
-//                   (tcgen05.ld) and keep each token's max over the n_text real
-//                   columns.
+//                   (tcgen05.ld) and keep each token's max over the n_text
+//                   real columns;
+//   qer_score_pair  the same over pairs of SMs (tcgen05 cta_group::2), for
+//                   runs longer than one wave of qer_score;
 //   qer_mean        w_f = (sum of the frame's token maxima) / (|V_f| H sqrt(d)),
 //                   a warp per frame;
 //   qer_rank        the k best frames by rank (ties to the lower index), a
-//                   thread per frame against all scores staged in shared memory;
-//   qer_compact     the kept frames in time order (one CTA).
+//                   warp per frame; the last CTA writes them in time order.
+// Every kernel after the first is a programmatic dependent of the one before
+// it, so its launch and set-up overlap that kernel's tail.
 // Every mbarrier wait is bounded by the global timer; a wait that runs out
 // sets an error bit, stops issuing, lets the work already issued finish
 // (bounded) and frees TMEM before the CTA exits.
@@ -63,7 +66,6 @@ constexpr int kQerPairThreads = kQerThreads + 32;     // paired kernel: + a seco
 constexpr size_t kQerPairRingBudget = 224 * 1024;     // paired kernel: both rings (one CTA per SM)
 constexpr uint32_t kQerPairQSlots = 3;                // q~ slots: enough to cover its L2 latency
 constexpr uint32_t kQerMaxN = 256;  // text tokens (MMA N) per CTA
-constexpr int kSelThreads = 1024;
 constexpr int kRankThreads = 256;  // 8 frames per CTA (a warp each): the O(m^2) ranking spreads over many SMs
 
 constexpr uint32_t kQerErrProducer = 16u, kQerErrMma = 32u, kQerErrEpilogue = 64u, kQerErrDrain = 128u;
@@ -144,6 +146,12 @@ __device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t a, uint64_t 
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
+
+// Programmatic dependent launch: let the next kernel in the stream be
+// scheduled now / wait until the previous one has completed and its memory
+// is visible (a no-op when the kernel was not launched as a dependent).
+__device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -263,6 +271,7 @@ __device__ __forceinline__ void umma_pair_commit_both(uint32_t bar) {
 
 __global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H,
                               uint32_t H_kv, uint32_t d, __nv_bfloat16_raw* __restrict__ qg) {
+  grid_dependents_launch();  // the scoring kernel may start; its q~ loads wait for this grid
   const uint32_t D = H_kv * d, G = H / H_kv;
   const uint64_t total = static_cast<uint64_t>(n_pad) * D;
   for (uint64_t e = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; e < total;
@@ -280,6 +289,7 @@ __global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, u
 // The same with 8 consecutive channels per thread (d % 8 == 0, 16-byte aligned q).
 __global__ void qer_prepare_q8(const uint4* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H, uint32_t H_kv,
                                uint32_t d, uint4* __restrict__ qg) {
+  grid_dependents_launch();  // the scoring kernel may start; its q~ loads wait for this grid
   const uint32_t d8 = d / 8, D8 = H_kv * d8, G = H / H_kv;
   const uint64_t total = static_cast<uint64_t>(n_pad) * D8;
   for (uint64_t e = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; e < total;
@@ -369,6 +379,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
   if (warp == 0) {
     if (lane == 0) {
       // --------------------------------------------------------- TMA producer
+      grid_dependency_wait();  // q~ is written by the kernel before this one
       const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
       uint32_t g = 0, s = 0, ph = 0;  // chunk counter over all of this CTA's tiles; ring slot and phase
       bool stop = false;
@@ -584,6 +595,7 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
       const uint32_t full0_rank0 = map_to_rank(full0, 0);  // rank 0's full barriers count both CTAs' bytes
       const CUtensorMap* map = keys ? &map_k : &map_qh;
       const uint32_t tx = 2 * kSub * chunk;
+      if (!keys) grid_dependency_wait();  // q~ is written by the kernel before this one; keys stream at once
       uint32_t g = 0, s = 0, ph = 0;
       bool stop = false;
       for (uint32_t t = 0; t < my_tiles && !stop; ++t) {
@@ -712,9 +724,11 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
 }
 
 // Eq. 7: w_f = mean over the frame's tokens of their max over text, times the
-// 1/(H sqrt(d)) of Eq. 6. One warp per frame.
+// 1/(H sqrt(d)) of Eq. 6. One warp per frame; a programmatic dependent of the
+// scoring kernel, whose maxima it waits for.
 __global__ void __launch_bounds__(256) qer_mean(const float* __restrict__ colmax, uint32_t n_frames, uint32_t tpf,
                                                 float scale, float* __restrict__ w) {
+  grid_dependency_wait();
   const uint32_t f = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (f >= n_frames) return;
   float s = 0.f;
@@ -727,53 +741,68 @@ __global__ void __launch_bounds__(256) qer_mean(const float* __restrict__ colmax
 // Eq. 8: flag[f] = 1 when fewer than k frames rank above frame f (higher w,
 // or equal w and lower index). A warp per frame: its lanes split the m scores
 // (coalesced reads of the L2-resident w) and one warp reduction counts them.
+// The last CTA to finish (a ticket taken after a fence) then writes the flagged frames
+// in time order (ballot, popcount and a scan of the warp totals per pass of
+// kRankThreads frames), the count to k_out, and returns the ticket counter
+// to zero. Launched as a programmatic dependent of the mean kernel, so every
+// thread first waits for that grid's completion and memory.
 __global__ void __launch_bounds__(kRankThreads) qer_rank(const float* __restrict__ w, uint32_t n_frames, uint32_t k,
-                                                uint8_t* __restrict__ flag) {
-  const uint32_t f = blockIdx.x * (kRankThreads / 32) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (f >= n_frames) return;  // uniform across the warp
-  const float wf = w[f];
-  uint32_t above = 0;
-#pragma unroll 4
-  for (uint32_t g = lane; g < n_frames; g += 32) {
-    const float wg = __ldg(w + g);
-    above += (wg > wf) | ((wg == wf) & (g < f));
-  }
-  above = __reduce_add_sync(0xffffffffu, above);
-  if (lane == 0) flag[f] = above < k;
-}
-
-// The flagged frames, in time order: block-wide compaction (ballot,
-// popcount, a scan of the 32 warp totals), 1024 frames per pass.
-__global__ void __launch_bounds__(kSelThreads) qer_compact(const uint8_t* __restrict__ flag, uint32_t n_frames,
-                                                           uint32_t* __restrict__ sel, uint32_t* __restrict__ k_out) {
-  __shared__ uint32_t wsum[32];
-  __shared__ uint32_t s_total;
+                                                uint8_t* __restrict__ flag, uint32_t* __restrict__ done,
+                                                uint32_t* __restrict__ sel,
+                                                uint32_t* __restrict__ k_out) {
+  constexpr uint32_t kWarps = kRankThreads / 32;
+  __shared__ uint32_t wsum[kWarps];
+  __shared__ uint32_t s_total, s_last;
+  grid_dependency_wait();
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t f = blockIdx.x * kWarps + warp;
+  if (f < n_frames) {  // uniform across the warp
+    const float wf = w[f];
+    uint32_t above = 0;
+#pragma unroll 4
+    for (uint32_t g = lane; g < n_frames; g += 32) {
+      const float wg = __ldg(w + g);
+      above += (wg > wf) | ((wg == wf) & (g < f));
+    }
+    above = __reduce_add_sync(0xffffffffu, above);
+    if (lane == 0) flag[f] = above < k;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();  // this CTA's flags are visible before its ticket
+    s_last = atomicAdd(done, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();  // every CTA's flags are visible to the last one
   uint32_t base = 0;
-  for (uint32_t f0 = 0; f0 < n_frames; f0 += kSelThreads) {
-    const uint32_t f = f0 + tid;
-    const bool in = f < n_frames && flag[f];
+  for (uint32_t f0 = 0; f0 < n_frames; f0 += kRankThreads) {
+    const uint32_t g = f0 + tid;
+    const bool in = g < n_frames && __ldcg(flag + g) != 0;
     const uint32_t bal = __ballot_sync(0xffffffffu, in);
     const uint32_t before = __popc(bal & ((1u << lane) - 1u));
     if (lane == 0) wsum[warp] = __popc(bal);
     __syncthreads();
     if (warp == 0) {
-      const uint32_t v = wsum[lane];
+      const uint32_t v = lane < kWarps ? wsum[lane] : 0u;
       uint32_t x = v;
 #pragma unroll
       for (int dd = 1; dd < 32; dd <<= 1) {
         const uint32_t y = __shfl_up_sync(0xffffffffu, x, dd);
         if (lane >= static_cast<uint32_t>(dd)) x += y;
       }
-      wsum[lane] = x - v;
+      if (lane < kWarps) wsum[lane] = x - v;
       if (lane == 31) s_total = x;
     }
     __syncthreads();
-    if (in) sel[base + wsum[warp] + before] = f;
+    if (in) sel[base + wsum[warp] + before] = g;
     base += s_total;
     __syncthreads();
   }
-  if (tid == 0) *k_out = base;
+  if (tid == 0) {
+    *k_out = base;
+    *done = 0;
+  }
 }
 
 uint32_t qer_stage_bytes(uint32_t n_pad) { return 2 * kQerM * 128 + ((n_pad * 128 + 1023) & ~1023u); }
@@ -846,6 +875,7 @@ struct cofie_qer {
   float* d_w = nullptr;
   uint8_t* d_flag = nullptr;
   uint32_t* d_k = nullptr;
+  uint32_t* d_done = nullptr;  // CTAs of the ranking kernel that have finished
   uint32_t* d_err = nullptr;
   std::string err;
   // launch counter and optional event timing of the scoring kernel
@@ -877,7 +907,7 @@ void qer_free(cofie_qer* h) {
   cudaGetDevice(&prev);
   cudaSetDevice(h->device);
   cudaDeviceSynchronize();
-  void* bufs[] = {h->d_qg, h->d_colmax, h->d_w, h->d_k, h->d_err, h->d_flag};
+  void* bufs[] = {h->d_qg, h->d_colmax, h->d_w, h->d_k, h->d_err, h->d_flag, h->d_done};
   for (void* b : bufs)
     if (b) cudaFree(b);
   for (cudaEvent_t e : h->ev) cudaEventDestroy(e);
@@ -941,6 +971,8 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   if (e == cudaSuccess) e = cudaMalloc(&h->d_w, static_cast<size_t>(p->max_frames) * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_k, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_flag, p->max_frames);
+  if (e == cudaSuccess) e = cudaMalloc(&h->d_done, sizeof(uint32_t));
+  if (e == cudaSuccess) e = cudaMemset(h->d_done, 0, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_err, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
   if (e == cudaSuccess)
@@ -1043,6 +1075,10 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
     qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, h->n_pad, p.n_heads, p.n_kv_heads, p.head_dim, h->d_qg);
   }
   const uint32_t grid = tiles < static_cast<uint32_t>(h->grid) ? tiles : static_cast<uint32_t>(h->grid);
+  const uint32_t kk = static_cast<uint32_t>(std::max(1.0, std::nearbyint(static_cast<double>(p.rho) * n_frames)));
+  const float scale = static_cast<float>(1.0 / (static_cast<double>(p.n_heads) * std::sqrt(static_cast<double>(p.head_dim))));
+  float* w = w_out ? w_out : h->d_w;
+  uint32_t* kdev = is_device(k_out, h->device) ? k_out : h->d_k;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (h->time_on && h->ev_used + 2 <= (1u << 16)) {
     while (h->ev.size() < h->ev_used + 2) {
@@ -1057,46 +1093,52 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
       cudaEventRecord(e0, st);
     }
   }
+  // The scoring, mean and ranking kernels are programmatic dependents of the
+  // kernel before them: each may be scheduled while its predecessor still
+  // runs, and waits for it (griddepcontrol.wait) only where it reads that
+  // kernel's output (the scoring kernel's q~ producer; every thread of the
+  // mean and ranking kernels). With the timing events in between, the
+  // scoring kernel's launch serialises as usual.
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.stream = st;
+  cfg.attrs = attr;
   if (pair_run) {
     const uint32_t clusters = std::min<uint32_t>(tiles, static_cast<uint32_t>(h->pair_clusters));
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 2;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * clusters, 1, 1);
     cfg.blockDim = dim3(kQerPairThreads, 1, 1);
     cfg.dynamicSmemBytes = h->pair_smem;
-    cfg.stream = st;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     const uint32_t n_chunks = h->D / kQerKChunk / h->pair_sub;
-    if (h->pair_sub == 2)
-      cudaLaunchKernelEx(&cfg, qer_score_pair<2>, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
-                         h->acc_cols, h->pair_key_slots, kQerPairQSlots, n_chunks, tiles, h->d_colmax, h->d_err,
-                         2000000000ull);
-    else
-      cudaLaunchKernelEx(&cfg, qer_score_pair<1>, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
-                         h->acc_cols, h->pair_key_slots, kQerPairQSlots, n_chunks, tiles, h->d_colmax, h->d_err,
-                         2000000000ull);
+    cudaLaunchKernelEx(&cfg, h->pair_sub == 2 ? qer_score_pair<2> : qer_score_pair<1>, map_k, map_q,
+                       static_cast<uint32_t>(nv), p.n_text, h->n_pad, h->acc_cols, h->pair_key_slots, kQerPairQSlots,
+                       n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
   } else {
-    qer_score<<<grid, kQerThreads, h->smem, st>>>(map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad,
-                                                  h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles,
-                                                  h->d_colmax, h->d_err, 2000000000ull);
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(kQerThreads, 1, 1);
+    cfg.dynamicSmemBytes = h->smem;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, qer_score, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad, h->acc_cols,
+                       h->n_buf, h->n_stages, h->D / kQerKChunk, tiles, h->d_colmax, h->d_err, 2000000000ull);
   }
   if (e1) cudaEventRecord(e1, st);
   h->launches += 1;
   h->flops += 2.0 * h->n_pad * static_cast<double>(nv) * h->D;
   h->key_bytes += 2.0 * static_cast<double>(nv) * h->D;
-  const uint32_t kk = static_cast<uint32_t>(std::max(1.0, std::nearbyint(static_cast<double>(p.rho) * n_frames)));
-  const float scale = static_cast<float>(1.0 / (static_cast<double>(p.n_heads) * std::sqrt(static_cast<double>(p.head_dim))));
-  float* w = w_out ? w_out : h->d_w;
-  uint32_t* kdev = is_device(k_out, h->device) ? k_out : h->d_k;
-  qer_mean<<<(n_frames + 7) / 8, 256, 0, st>>>(h->d_colmax, n_frames, p.tokens_per_frame, scale, w);
-  qer_rank<<<(n_frames + kRankThreads / 32 - 1) / (kRankThreads / 32), kRankThreads, 0, st>>>(w, n_frames, kk,
-                                                                                              h->d_flag);
-  qer_compact<<<1, kSelThreads, 0, st>>>(h->d_flag, n_frames, sel_out, kdev);
+  cfg.gridDim = dim3((n_frames + 7) / 8, 1, 1);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.dynamicSmemBytes = 0;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, qer_mean, static_cast<const float*>(h->d_colmax), n_frames, p.tokens_per_frame, scale, w);
+  cfg.gridDim = dim3((n_frames + kRankThreads / 32 - 1) / (kRankThreads / 32), 1, 1);
+  cfg.blockDim = dim3(kRankThreads, 1, 1);
+  cudaLaunchKernelEx(&cfg, qer_rank, static_cast<const float*>(w), n_frames, kk, h->d_flag, h->d_done, sel_out, kdev);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess && kdev != k_out) {
     e = cudaMemcpyAsync(k_out, kdev, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);

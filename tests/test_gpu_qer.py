@@ -127,3 +127,33 @@ def test_qer_full_size_sampled(n_frames):
     check(spec, 0.3, frames=frames)
     f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3)
     assert f.kernel == 2  # the handle can pair; a run switches to it above one wave
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_qer_repeated_calls_on_one_handle(kernel):
+    """One handle, calls over prefixes of one stream of different lengths and
+    a repeat: every call equals a fresh handle's call bit for bit (the frame
+    counters of the epilogue and the ranking kernel's ticket return to zero),
+    and the scores are reproducible. 24 tokens per frame: an epilogue warp's
+    32 tokens span two frames."""
+    from paper_2609_03675_gb300 import QER
+    spec = S.QerSpec(n_text=64, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=40, tokens_per_frame=24,
+                     n_evidence=3, seed=21)
+    q, k, _ = S.generate(spec)
+    qd = torch.from_numpy(q.view(np.int16)).cuda()
+    kd = torch.from_numpy(k.view(np.int16)).cuda()
+    args = (spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.25)
+    f = QER(*args, kernel=kernel)
+    for n in (40, 7, 40, 1, 23, 40):
+        w, sel = f.run(qd, kd, n_frames=n)
+        g = QER(*args, kernel=kernel)
+        w2, sel2 = g.run(qd, kd, n_frames=n)
+        torch.cuda.synchronize()
+        f.status()
+        g.status()
+        assert torch.equal(w, w2) and torch.equal(sel, sel2), n
+        rho32 = float(np.float32(0.25))
+        assert list(sel.cpu().numpy()) == list(Q.select(w.cpu().numpy().astype(np.float64), rho32)), n
+        w_o = Q.frame_relevance_subset(q, k, spec.tokens_per_frame, range(n))
+        bound = Q.score_bound(q, k, spec.tokens_per_frame, range(n)) + 2.0 ** -18 * np.abs(w_o)
+        assert np.all(np.abs(w.cpu().numpy() - w_o) <= bound), n
