@@ -452,7 +452,10 @@ uint32_t cofie_qer_kernel_in_use(const cofie_qer_t* h);
 int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t n_frames, float* w_out,
                   uint32_t* sel_out, uint32_t* k_out, void* cuda_stream);
 
-/* Synchronises cuda_stream; COFIE_ETIMEOUT if a bounded device wait ran out. */
+/* Synchronises cuda_stream; COFIE_ETIMEOUT if a bounded device wait ran out;
+ * in a build with -DCOFIE_DEBUG_CHECKS=1, COFIE_EDEVICE if a kernel found its
+ * shared-memory rings or TMEM accumulators outside what the launch gave it
+ * (it then ran no tile). */
 int cofie_qer_status(cofie_qer_t* h, void* cuda_stream);
 
 /* Launch counter and CUDA-event timing of the scoring (tensor-core) kernel:

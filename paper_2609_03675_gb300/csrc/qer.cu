@@ -103,6 +103,13 @@ __device__ __noinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, uint64
   }
 }
 
+// Bytes of dynamic shared memory this launch gave the CTA.
+__device__ __forceinline__ uint32_t dynamic_smem_bytes() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%dynamic_smem_size;" : "=r"(r));
+  return r;
+}
+
 // The common case inline (the phase has already completed), the bounded
 // wait loop out of line.
 __device__ __forceinline__ bool mbar_wait_fast(uint32_t bar, uint32_t parity, uint64_t timeout_ns) {
@@ -350,6 +357,13 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
   const uint32_t tmem_total = 2 * acc_cols * n_buf;
+  // checked build: the ring ends inside this launch's dynamic shared memory,
+  // its slots fit the barrier arrays, and each accumulator's n_pad columns
+  // lie inside its acc_cols (a failed check runs no tile: my_tiles = 0)
+  const bool layout_ok = COFIE_BOUND(smem_u32(smem) + n_stages * stage_bytes <=
+                                         smem_u32(smem_raw) + dynamic_smem_bytes() &&
+                                     n_stages >= 1 && n_stages <= kQerMaxStages && n_pad <= acc_cols &&
+                                     n_buf >= 1 && n_buf <= 2);
 
   if (warp == 0) {  // the whole warp allocates the accumulators
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
@@ -383,7 +397,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
       const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
       uint32_t g = 0, s = 0, ph = 0;  // chunk counter over all of this CTA's tiles; ring slot and phase
       bool stop = false;
-      for (uint32_t t = 0; t < my_tiles && !stop; ++t) {
+      for (uint32_t t = 0; t < (layout_ok ? my_tiles : 0u) && !stop; ++t) {
         const int32_t row0 = static_cast<int32_t>((blockIdx.x + t * gridDim.x) * kQerTile);
         for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
           if (g >= n_stages && !mbar_wait_fast(empty0 + 8 * s, ph ^ 1, timeout_ns)) {
@@ -421,7 +435,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
       const uint32_t ring0 = smem_u32(smem), empty0 = smem_u32(&empty_bar[0]), full0 = smem_u32(&full_bar[0]);
       uint32_t s = 0, ph = 0;
       bool stop = false;
-      for (uint32_t t = 0; t < my_tiles && !stop && !abort_flag; ++t) {
+      for (uint32_t t = 0; t < (layout_ok ? my_tiles : 0u) && !stop && !abort_flag; ++t) {
         const uint32_t b = t % n_buf, ub = t / n_buf;
         if (ub > 0 && !mbar_wait_fast(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
           atomicOr(err, kQerErrMma);
@@ -461,7 +475,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
   } else {
     // --------------------------------------------------------------- epilogue
     const uint32_t quarter = warp & 3;  // TMEM lanes this warp may read
-    for (uint32_t t = 0; t < my_tiles; ++t) {
+    for (uint32_t t = 0; t < (layout_ok ? my_tiles : 0u); ++t) {
       const uint32_t b = t % n_buf, ub = t / n_buf;
       bool ok = !abort_flag && mbar_wait_for(smem_u32(&tfull_bar[b]), ub & 1, timeout_ns);
       ok = __all_sync(0xffffffffu, ok);
@@ -551,6 +565,14 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
   const uint32_t my_tiles = pair < n_tiles ? (n_tiles - 1 - pair) / n_pairs + 1 : 0;
   const uint32_t tmem_total = 2 * acc_cols;  // two accumulators
   const uint32_t kring0 = smem_u32(smem), qring0 = kring0 + n_kst * kslot;
+  // checked build: both rings end inside this launch's dynamic shared memory,
+  // their slots fit the barrier arrays, the accumulators' n_pad columns lie
+  // inside acc_cols, and the grid is whole clusters of two (a failed check
+  // runs no tile: my_tiles = 0 in both CTAs, which see the same arguments)
+  const bool layout_ok = COFIE_BOUND(qring0 + n_qst * qslot <= smem_u32(smem_raw) + dynamic_smem_bytes() &&
+                                     n_kst >= 1 && n_kst <= kQerMaxStages && n_qst >= 1 && n_qst <= kQerMaxStages &&
+                                     n_pad <= acc_cols && n_pad % 32 == 0 && gridDim.x % 2 == 0);
+  const uint32_t run_tiles = layout_ok ? my_tiles : 0u;
 
   if (warp == 0) {  // one warp in each CTA of the pair allocates, together
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_slot)),
@@ -598,7 +620,7 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
       if (!keys) grid_dependency_wait();  // q~ is written by the kernel before this one; keys stream at once
       uint32_t g = 0, s = 0, ph = 0;
       bool stop = false;
-      for (uint32_t t = 0; t < my_tiles && !stop; ++t) {
+      for (uint32_t t = 0; t < run_tiles && !stop; ++t) {
         const int32_t y = keys ? static_cast<int32_t>((pair + t * n_pairs) * kQerTile + rank * kQerM)
                                : static_cast<int32_t>(rank * half_rows);
         for (uint32_t kc = 0; kc < n_chunks; ++kc, ++g) {
@@ -641,7 +663,7 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
       const uint64_t a16 = a_chunk >> 4, b16 = b_chunk >> 4;
       uint32_t ks = 0, kph = 0, qs = 0, qph = 0;
       bool stop = false;
-      for (uint32_t t = 0; t < my_tiles && !stop && !abort_flag; ++t) {
+      for (uint32_t t = 0; t < run_tiles && !stop && !abort_flag; ++t) {
         const uint32_t b = t & 1, ub = t >> 1;
         if (ub > 0 && !mbar_wait_cluster(smem_u32(&tempty_bar[b]), (ub - 1) & 1, timeout_ns)) {
           atomicOr(err, kQerErrMma);
@@ -688,7 +710,7 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
     const uint32_t quarter = warp & 3;  // warps 2..5: TMEM lanes 32 (warp % 4) ..
     const uint32_t tempty0 = map_to_rank(smem_u32(&tempty_bar[0]), 0);
     const uint32_t tempty1 = map_to_rank(smem_u32(&tempty_bar[1]), 0);
-    for (uint32_t t = 0; t < my_tiles; ++t) {
+    for (uint32_t t = 0; t < run_tiles; ++t) {
       const uint32_t b = t & 1, ub = t >> 1;
       bool ok = !abort_flag && mbar_wait_cluster(smem_u32(&tfull_bar[b]), ub & 1, timeout_ns);
       ok = __all_sync(0xffffffffu, ok);
@@ -1158,7 +1180,9 @@ int cofie_qer_status(cofie_qer_t* h, void* cuda_stream) {
   if (e == cudaSuccess) e = cudaMemcpy(&word, h->d_err, sizeof word, cudaMemcpyDeviceToHost);
   if (e == cudaSuccess && word) cudaMemset(h->d_err, 0, sizeof word);
   if (prev >= 0) cudaSetDevice(prev);
+  const uint32_t bounds = take_local_bounds_errors();  // checked build only; 0 otherwise
   if (e != cudaSuccess) return h->fail(COFIE_ECUDA, cudaGetErrorString(e));
+  if (bounds) return h->fail(COFIE_EDEVICE, "a layout check of the QER kernels failed (checked build)");
   if (word) return h->fail(COFIE_ETIMEOUT, "a device-side wait of the QER kernels ran out");
   return COFIE_OK;
 }

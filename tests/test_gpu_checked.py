@@ -3,7 +3,8 @@ check every computed index against their launch arguments and report a
 failed check through cofie_ngff_status) run over representative workloads:
 the fast and generic histogram kernels, one- and two-word gap masks, the
 spatial signals on both of their kernels, scene changes across scan tiles,
-the frame-order walk (L_max = 0), batches, shards, candidates and gather.
+the frame-order walk (L_max = 0), batches, shards, candidates and gather,
+and QER on both scoring kernels.
 Every result must still equal the oracle's and no check may fail. A memory
 checker is not available on the GPUs this is tested on; these checks stand in
 for it. The workloads run in a child process that loads the checked library."""
@@ -137,6 +138,26 @@ want = O.load().candidates(ko, 4)
 assert np.array_equal(idx.cpu().numpy(), want)
 assert torch.equal(out, dev[idx.long()])
 n += 1
+# QER: the one-SM and the paired kernel, and the benchmark geometry at one wave
+from paper_2609_03675_gb300 import QER
+from oracle import qer_oracle as Q
+from synth import qer as SQ
+for spec, kernel in ((SQ.QerSpec(n_text=40, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=6, tokens_per_frame=40,
+                                 n_evidence=2, seed=31), 1),
+                     (SQ.QerSpec(n_text=64, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=9, tokens_per_frame=24,
+                                 n_evidence=2, seed=32), 2),
+                     (SQ.QerSpec(n_frames=128), 0)):
+    q, k, _ = SQ.generate(spec)
+    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3,
+            kernel=kernel)
+    w, sel = f.run(torch.from_numpy(q.view(np.int16)).cuda(), torch.from_numpy(k.view(np.int16)).cuda())
+    torch.cuda.synchronize()
+    f.status()  # raises on a failed layout check
+    frames = np.linspace(0, spec.n_frames - 1, min(spec.n_frames, 6)).astype(int)
+    w_o = Q.frame_relevance_subset(q, k, spec.tokens_per_frame, frames)
+    bound = Q.score_bound(q, k, spec.tokens_per_frame, frames) + 2.0 ** -18 * np.abs(w_o)
+    assert np.all(np.abs(w.cpu().numpy()[frames] - w_o) <= bound), f"QER kernel {kernel}"
+    n += 1
 print("checked workloads", n)
 '''
 
@@ -155,4 +176,4 @@ def test_checked_build_runs_clean_and_matches_the_oracle():
                   build_dir=os.path.join(d, "obj"))
     r = subprocess.run([sys.executable, "-c", CHILD, lib, REPO], capture_output=True, text=True, timeout=900)
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
-    assert "checked workloads 22" in r.stdout, r.stdout[-2000:]
+    assert "checked workloads 25" in r.stdout, r.stdout[-2000:]
