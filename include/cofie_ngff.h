@@ -403,12 +403,15 @@ int cofie_ngff_select_static(const cofie_ngff_params* p, const uint32_t* hist, u
  * the attention). The query heads of each group are summed in fp32 and
  * rounded to bf16; the contraction runs on the tensor cores in bf16 with fp32
  * accumulation. round() rounds half to even; equal scores rank by lower
- * frame index; S_e is returned in time order.
+ * frame index; S_e is returned in time order. A query of more than 256 text
+ * tokens is split into ceil(n_text / 256) equal blocks scored in successive
+ * passes over the keys, each pass keeping the running max of Eq. 7's inner
+ * max (the keys are read once per pass).
  * ------------------------------------------------------------------------ */
 typedef struct cofie_qer cofie_qer_t;
 
 typedef struct {
-  uint32_t n_text;           /* text tokens |Q|, 1..256 */
+  uint32_t n_text;           /* text tokens |Q|, 1..4096 (scored in passes of at most 256) */
   uint32_t n_heads;          /* H query heads */
   uint32_t n_kv_heads;       /* H_kv key heads, divides H */
   uint32_t head_dim;         /* d_h; H_kv * d_h a multiple of 64, at most 16384 */
@@ -420,7 +423,8 @@ typedef struct {
 } cofie_qer_params;
 
 /* Scoring kernels: the paired-SM one (clusters of two CTAs, one M = 256 MMA
- * per pair) needs n_text rounded up to 16 to be a multiple of 32; AUTO takes
+ * per pair) needs the text block (n_text, or for n_text > 256 its blocks,
+ * which are padded to 32) rounded up to 16 to be a multiple of 32; AUTO takes
  * it when it applies and the 256-token tiles of a run exceed one wave of the
  * one-SM kernel (one per SM). The results of the two agree up to the order of
  * fp32 accumulation inside the tensor cores. */

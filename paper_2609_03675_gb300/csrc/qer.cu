@@ -65,7 +65,8 @@ constexpr int kQerThreads = 32 * (2 + kQerEpiWarps);  // + TMA producer warp + M
 constexpr int kQerPairThreads = kQerThreads + 32;     // paired kernel: + a second producer warp (q~)
 constexpr size_t kQerPairRingBudget = 224 * 1024;     // paired kernel: both rings (one CTA per SM)
 constexpr uint32_t kQerPairQSlots = 3;                // q~ slots: enough to cover its L2 latency
-constexpr uint32_t kQerMaxN = 256;  // text tokens (MMA N) per CTA
+constexpr uint32_t kQerMaxN = 256;      // text tokens (MMA N) per scoring pass
+constexpr uint32_t kQerMaxText = 4096;  // text tokens per query: up to 16 passes
 constexpr int kRankThreads = 256;  // 8 frames per CTA (a warp each): the O(m^2) ranking spreads over many SMs
 
 constexpr uint32_t kQerErrProducer = 16u, kQerErrMma = 32u, kQerErrEpilogue = 64u, kQerErrDrain = 128u;
@@ -103,12 +104,14 @@ __device__ __noinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, uint64
   }
 }
 
-// Bytes of dynamic shared memory this launch gave the CTA.
+#if COFIE_DEBUG_CHECKS
+// Bytes of dynamic shared memory this launch gave the CTA (checked build).
 __device__ __forceinline__ uint32_t dynamic_smem_bytes() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%dynamic_smem_size;" : "=r"(r));
   return r;
 }
+#endif
 
 // The common case inline (the phase has already completed), the bounded
 // wait loop out of line.
@@ -276,14 +279,23 @@ __device__ __forceinline__ void umma_pair_commit_both(uint32_t bar) {
       : "memory");
 }
 
-__global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H,
-                              uint32_t H_kv, uint32_t d, __nv_bfloat16_raw* __restrict__ qg) {
+// q~ row p of n_rows belongs to text block p / bp, row p % bp of it; block b
+// holds text tokens [b per_blk, (b + 1) per_blk), the rest of its bp rows are
+// zero. Returns the text token, or n_text for a zero row.
+__device__ __forceinline__ uint32_t qer_text_of_row(uint32_t p, uint32_t bp, uint32_t per_blk, uint32_t n_text) {
+  const uint32_t b = p / bp, r = p % bp, i = b * per_blk + r;
+  return (r < per_blk && i < n_text) ? i : n_text;
+}
+
+__global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, uint32_t n_rows, uint32_t bp,
+                              uint32_t per_blk, uint32_t H, uint32_t H_kv, uint32_t d,
+                              __nv_bfloat16_raw* __restrict__ qg) {
   grid_dependents_launch();  // the scoring kernel may start; its q~ loads wait for this grid
   const uint32_t D = H_kv * d, G = H / H_kv;
-  const uint64_t total = static_cast<uint64_t>(n_pad) * D;
+  const uint64_t total = static_cast<uint64_t>(n_rows) * D;
   for (uint64_t e = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<uint64_t>(gridDim.x) * blockDim.x) {
-    const uint32_t i = static_cast<uint32_t>(e / D), r = static_cast<uint32_t>(e % D);
+    const uint32_t i = qer_text_of_row(static_cast<uint32_t>(e / D), bp, per_blk, n_text), r = static_cast<uint32_t>(e % D);
     const uint32_t g = r / d, c = r % d;
     float s = 0.f;
     if (i < n_text)
@@ -294,14 +306,14 @@ __global__ void qer_prepare_q(const uint16_t* __restrict__ q, uint32_t n_text, u
 }
 
 // The same with 8 consecutive channels per thread (d % 8 == 0, 16-byte aligned q).
-__global__ void qer_prepare_q8(const uint4* __restrict__ q, uint32_t n_text, uint32_t n_pad, uint32_t H, uint32_t H_kv,
-                               uint32_t d, uint4* __restrict__ qg) {
+__global__ void qer_prepare_q8(const uint4* __restrict__ q, uint32_t n_text, uint32_t n_rows, uint32_t bp,
+                               uint32_t per_blk, uint32_t H, uint32_t H_kv, uint32_t d, uint4* __restrict__ qg) {
   grid_dependents_launch();  // the scoring kernel may start; its q~ loads wait for this grid
   const uint32_t d8 = d / 8, D8 = H_kv * d8, G = H / H_kv;
-  const uint64_t total = static_cast<uint64_t>(n_pad) * D8;
+  const uint64_t total = static_cast<uint64_t>(n_rows) * D8;
   for (uint64_t e = blockIdx.x * static_cast<uint64_t>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<uint64_t>(gridDim.x) * blockDim.x) {
-    const uint32_t i = static_cast<uint32_t>(e / D8), r = static_cast<uint32_t>(e % D8);
+    const uint32_t i = qer_text_of_row(static_cast<uint32_t>(e / D8), bp, per_blk, n_text), r = static_cast<uint32_t>(e % D8);
     const uint32_t g = r / d8, c8 = r % d8;
     float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
     if (i < n_text)
@@ -338,7 +350,8 @@ __global__ void qer_prepare_q8(const uint4* __restrict__ q, uint32_t n_text, uin
 __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__ CUtensorMap map_k,
                                                          const __grid_constant__ CUtensorMap map_q,
                                                          uint32_t n_visual, uint32_t n_text, uint32_t n_pad,
-                                                         uint32_t acc_cols, uint32_t n_buf, uint32_t n_stages,
+                                                         uint32_t fold, uint32_t acc_cols, uint32_t n_buf,
+                                                         uint32_t n_stages,
                                                          uint32_t n_chunks, uint32_t n_tiles,
                                                          float* __restrict__ colmax, uint32_t* __restrict__ err,
                                                          uint64_t timeout_ns) {
@@ -491,7 +504,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
         const uint32_t taddr = tmem + (b * 2 + half) * acc_cols + ((quarter * 32u) << 16);
         const float best = tmem_row_max(taddr, n_pad, n_text);
         const uint32_t j = row0 + half * kQerM + quarter * 32 + lane;
-        if (j < n_visual) colmax[j] = best;
+        if (j < n_visual) colmax[j] = fold ? fmaxf(colmax[j], best) : best;
       }
       tc_fence_before();
       __syncwarp();
@@ -542,7 +555,7 @@ __global__ void __launch_bounds__(kQerThreads) qer_score(const __grid_constant__
 template <uint32_t kSub>
 __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
     const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_qh, uint32_t n_visual,
-    uint32_t n_text, uint32_t n_pad, uint32_t acc_cols, uint32_t n_kst, uint32_t n_qst, uint32_t n_chunks,
+    uint32_t n_text, uint32_t n_pad, uint32_t fold, uint32_t acc_cols, uint32_t n_kst, uint32_t n_qst, uint32_t n_chunks,
     uint32_t n_tiles, float* __restrict__ colmax, uint32_t* __restrict__ err, uint64_t timeout_ns) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t kfull_bar[kQerMaxStages];
@@ -723,7 +736,7 @@ __global__ void __launch_bounds__(kQerPairThreads) qer_score_pair(
       const uint32_t taddr = tmem + b * acc_cols + ((quarter * 32u) << 16);
       const float best = tmem_row_max(taddr, n_pad, n_text);
       const uint32_t j = (pair + t * n_pairs) * kQerTile + rank * kQerM + quarter * 32 + lane;
-      if (j < n_visual) colmax[j] = best;
+      if (j < n_visual) colmax[j] = fold ? fmaxf(colmax[j], best) : best;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(b ? tempty1 : tempty0);
@@ -885,6 +898,9 @@ using namespace cofie;
 struct cofie_qer {
   cofie_qer_params p{};
   int device = 0;
+  // the text is scored in n_blk passes of per_blk tokens (the last may have
+  // fewer), each padded to n_pad q~ rows; q~ holds n_blk * n_pad rows
+  uint32_t n_blk = 1, per_blk = 0;
   uint32_t n_pad = 0, D = 0, acc_cols = 0, n_buf = 1, n_stages = 0;
   int grid = 0;          // persistent CTAs
   size_t smem = 0;       // dynamic shared memory per CTA
@@ -945,7 +961,7 @@ extern "C" {
 
 int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   if (!p || !out) return g_qer_error = "params or out is NULL", COFIE_EINVAL;
-  if (p->n_text < 1 || p->n_text > kQerMaxN) return g_qer_error = "n_text must be in [1, 256]", COFIE_EINVAL;
+  if (p->n_text < 1 || p->n_text > kQerMaxText) return g_qer_error = "n_text must be in [1, 4096]", COFIE_EINVAL;
   if (p->n_heads < 1 || p->n_kv_heads < 1 || p->n_heads % p->n_kv_heads != 0)
     return g_qer_error = "n_kv_heads must divide n_heads", COFIE_EINVAL;
   const uint64_t D = static_cast<uint64_t>(p->n_kv_heads) * p->head_dim;
@@ -970,7 +986,12 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   h->p = *p;
   h->device = dev;
   h->D = static_cast<uint32_t>(D);
-  h->n_pad = (p->n_text + 15) / 16 * 16;
+  h->n_blk = (p->n_text + kQerMaxN - 1) / kQerMaxN;  // balanced blocks of at most 256 tokens
+  h->per_blk = (p->n_text + h->n_blk - 1) / h->n_blk;
+  // rows of a block: a multiple of 16 (the MMA's N step), of 32 when there are
+  // several blocks so that the paired kernel (half of q~ per CTA) stays open
+  const uint32_t row_step = h->n_blk > 1 ? 32u : 16u;
+  h->n_pad = (h->per_blk + row_step - 1) / row_step * row_step;
   h->acc_cols = 32;
   while (h->acc_cols < h->n_pad) h->acc_cols <<= 1;
   // Each tile needs two accumulators of acc_cols TMEM columns; double
@@ -988,7 +1009,7 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   while (max_ctas_by_tmem >= 1 && per_sm / (h->smem + 1024) > static_cast<size_t>(max_ctas_by_tmem))
     h->smem += 1024;
   const uint64_t nv = static_cast<uint64_t>(p->max_frames) * p->tokens_per_frame;
-  cudaError_t e = cudaMalloc(&h->d_qg, static_cast<size_t>(h->n_pad) * D * 2);
+  cudaError_t e = cudaMalloc(&h->d_qg, static_cast<size_t>(h->n_blk) * h->n_pad * D * 2);
   if (e == cudaSuccess) e = cudaMalloc(&h->d_colmax, nv * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_w, static_cast<size_t>(p->max_frames) * sizeof(float));
   if (e == cudaSuccess) e = cudaMalloc(&h->d_k, sizeof(uint32_t));
@@ -1040,7 +1061,9 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out) {
   } else if (e == cudaSuccess && p->kernel == COFIE_QER_KERNEL_PAIR) {
     if (prev >= 0) cudaSetDevice(prev);
     qer_free(h);
-    return g_qer_error = "the paired-SM kernel needs n_text rounded up to 16 to be a multiple of 32", COFIE_EINVAL;
+    return g_qer_error = "the paired-SM kernel needs the text block (n_text, or its blocks of at most 256) rounded up "
+                         "to 16 to be a multiple of 32",
+           COFIE_EINVAL;
   }
   if (prev >= 0) cudaSetDevice(prev);
   if (e != cudaSuccess) {
@@ -1086,15 +1109,16 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   // one wave of the one-SM kernel: a single wave runs faster on twice the CTAs
   const bool pair_run = h->pair && (p.kernel == COFIE_QER_KERNEL_PAIR || tiles > static_cast<uint32_t>(h->grid));
   const uint32_t q_box = pair_run ? h->n_pad / 2 : h->n_pad;  // the pair's CTAs each stage half of q~
-  if (!make_map(&map_k, k, nv, h->D, kQerM) || !make_map(&map_q, h->d_qg, h->n_pad, h->D, q_box))
-    return h->fail(COFIE_ECUDA, "tensor map encoding failed");
+  if (!make_map(&map_k, k, nv, h->D, kQerM)) return h->fail(COFIE_ECUDA, "tensor map encoding failed");
+  const uint32_t n_rows = h->n_blk * h->n_pad;
   if (p.head_dim % 8 == 0 && reinterpret_cast<uintptr_t>(q) % 16 == 0) {
-    const uint64_t n8 = static_cast<uint64_t>(h->n_pad) * h->D / 8;
+    const uint64_t n8 = static_cast<uint64_t>(n_rows) * h->D / 8;
     const uint32_t blocks = static_cast<uint32_t>(std::min<uint64_t>((n8 + 255) / 256, 1024));
-    qer_prepare_q8<<<blocks, 256, 0, st>>>(reinterpret_cast<const uint4*>(q), p.n_text, h->n_pad, p.n_heads,
-                                           p.n_kv_heads, p.head_dim, reinterpret_cast<uint4*>(h->d_qg));
+    qer_prepare_q8<<<blocks, 256, 0, st>>>(reinterpret_cast<const uint4*>(q), p.n_text, n_rows, h->n_pad, h->per_blk,
+                                           p.n_heads, p.n_kv_heads, p.head_dim, reinterpret_cast<uint4*>(h->d_qg));
   } else {
-    qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, h->n_pad, p.n_heads, p.n_kv_heads, p.head_dim, h->d_qg);
+    qer_prepare_q<<<256, 256, 0, st>>>(q, p.n_text, n_rows, h->n_pad, h->per_blk, p.n_heads, p.n_kv_heads,
+                                       p.head_dim, h->d_qg);
   }
   const uint32_t grid = tiles < static_cast<uint32_t>(h->grid) ? tiles : static_cast<uint32_t>(h->grid);
   const uint32_t kk = static_cast<uint32_t>(std::max(1.0, std::nearbyint(static_cast<double>(p.rho) * n_frames)));
@@ -1130,32 +1154,45 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   attr[1].val.clusterDim.z = 1;
   cudaLaunchConfig_t cfg = {};
   cfg.stream = st;
-  cfg.attrs = attr;
-  if (pair_run) {
-    const uint32_t clusters = std::min<uint32_t>(tiles, static_cast<uint32_t>(h->pair_clusters));
-    cfg.gridDim = dim3(2 * clusters, 1, 1);
-    cfg.blockDim = dim3(kQerPairThreads, 1, 1);
-    cfg.dynamicSmemBytes = h->pair_smem;
-    cfg.numAttrs = 2;
-    const uint32_t n_chunks = h->D / kQerKChunk / h->pair_sub;
-    cudaLaunchKernelEx(&cfg, h->pair_sub == 2 ? qer_score_pair<2> : qer_score_pair<1>, map_k, map_q,
-                       static_cast<uint32_t>(nv), p.n_text, h->n_pad, h->acc_cols, h->pair_key_slots, kQerPairQSlots,
-                       n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
-  } else {
-    cfg.gridDim = dim3(grid, 1, 1);
-    cfg.blockDim = dim3(kQerThreads, 1, 1);
-    cfg.dynamicSmemBytes = h->smem;
-    cfg.numAttrs = 1;
-    cudaLaunchKernelEx(&cfg, qer_score, map_k, map_q, static_cast<uint32_t>(nv), p.n_text, h->n_pad, h->acc_cols,
-                       h->n_buf, h->n_stages, h->D / kQerKChunk, tiles, h->d_colmax, h->d_err, 2000000000ull);
+  // One scoring pass per text block; passes after the first fold their
+  // maxima into colmax (Eq. 7's max over all text tokens) and are ordered
+  // after the pass before them as usual (no programmatic launch), so each
+  // reads that pass's maxima complete.
+  for (uint32_t blk = 0; blk < h->n_blk; ++blk) {
+    if (!make_map(&map_q, h->d_qg + static_cast<size_t>(blk) * h->n_pad * h->D, h->n_pad, h->D, q_box))
+      return h->fail(COFIE_ECUDA, "tensor map encoding failed");
+    const uint32_t text_b = std::min(h->per_blk, p.n_text - blk * h->per_blk);  // real columns of this pass
+    const uint32_t fold = blk > 0;
+    if (pair_run) {
+      const uint32_t clusters = std::min<uint32_t>(tiles, static_cast<uint32_t>(h->pair_clusters));
+      cfg.gridDim = dim3(2 * clusters, 1, 1);
+      cfg.blockDim = dim3(kQerPairThreads, 1, 1);
+      cfg.dynamicSmemBytes = h->pair_smem;
+      cfg.attrs = fold ? &attr[1] : attr;
+      cfg.numAttrs = fold ? 1 : 2;
+      const uint32_t n_chunks = h->D / kQerKChunk / h->pair_sub;
+      cudaLaunchKernelEx(&cfg, h->pair_sub == 2 ? qer_score_pair<2> : qer_score_pair<1>, map_k, map_q,
+                         static_cast<uint32_t>(nv), text_b, h->n_pad, fold, h->acc_cols, h->pair_key_slots,
+                         kQerPairQSlots, n_chunks, tiles, h->d_colmax, h->d_err, 2000000000ull);
+    } else {
+      cfg.gridDim = dim3(grid, 1, 1);
+      cfg.blockDim = dim3(kQerThreads, 1, 1);
+      cfg.dynamicSmemBytes = h->smem;
+      cfg.attrs = attr;
+      cfg.numAttrs = fold ? 0 : 1;
+      cudaLaunchKernelEx(&cfg, qer_score, map_k, map_q, static_cast<uint32_t>(nv), text_b, h->n_pad, fold,
+                         h->acc_cols, h->n_buf, h->n_stages, h->D / kQerKChunk, tiles, h->d_colmax, h->d_err,
+                         2000000000ull);
+    }
   }
   if (e1) cudaEventRecord(e1, st);
   h->launches += 1;
-  h->flops += 2.0 * h->n_pad * static_cast<double>(nv) * h->D;
-  h->key_bytes += 2.0 * static_cast<double>(nv) * h->D;
+  h->flops += 2.0 * n_rows * static_cast<double>(nv) * h->D;
+  h->key_bytes += 2.0 * static_cast<double>(nv) * h->D * h->n_blk;  // each pass reads the keys
   cfg.gridDim = dim3((n_frames + 7) / 8, 1, 1);
   cfg.blockDim = dim3(256, 1, 1);
   cfg.dynamicSmemBytes = 0;
+  cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaLaunchKernelEx(&cfg, qer_mean, static_cast<const float*>(h->d_colmax), n_frames, p.tokens_per_frame, scale, w);
   cfg.gridDim = dim3((n_frames + kRankThreads / 32 - 1) / (kRankThreads / 32), 1, 1);

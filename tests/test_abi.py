@@ -104,3 +104,20 @@ def test_create_rejects_nan_scene_thresholds(lib, field):
     h = ctypes.c_void_p()
     assert lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h)) == _abi.EINVAL
     assert "NaN" in lib.cofie_ngff_global_error().decode()
+
+
+@pytest.mark.parametrize("field,value,msg", [
+    ("n_text", 0, "n_text"), ("n_text", 4097, "n_text"), ("n_kv_heads", 3, "divide"), ("head_dim", 36, "multiple of 64"),
+    ("rho", 1.5, "rho"), ("kernel", 3, "kernel"), ("max_frames", 0, "max_frames"),
+])
+def test_qer_create_rejects_bad_params_without_gpu(lib, field, value, msg):
+    """QER's parameters are validated before any CUDA call: n_text runs to
+    4096 (scored in passes of at most 256), n_kv_heads divides n_heads,
+    H_kv * d_h is a multiple of 64, rho lies in [0, 1]."""
+    from paper_2609_03675_gb300 import _abi
+    p = _abi.QerParams(256, 32, 8, 128, 16, 256, 0.3, -1, 0)
+    setattr(p, field, value)
+    h = ctypes.c_void_p()
+    assert lib.cofie_qer_create(ctypes.byref(p), ctypes.byref(h)) == _abi.EINVAL
+    assert msg in lib.cofie_qer_last_error(None).decode()
+    assert not h.value

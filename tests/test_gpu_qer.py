@@ -157,3 +157,27 @@ def test_qer_repeated_calls_on_one_handle(kernel):
         w_o = Q.frame_relevance_subset(q, k, spec.tokens_per_frame, range(n))
         bound = Q.score_bound(q, k, spec.tokens_per_frame, range(n)) + 2.0 ** -18 * np.abs(w_o)
         assert np.all(np.abs(w.cpu().numpy() - w_o) <= bound), n
+
+
+@pytest.mark.parametrize("n_text", [257, 300, 600, 1000])
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_qer_long_queries_in_text_blocks(n_text, kernel):
+    """More than 256 text tokens: ceil(n_text / 256) blocks scored in passes
+    that keep a running max; the scores stay within the oracle's bound (the
+    bound is per token pair, so it holds for any split of the text) and the
+    selection is the TopK of the GPU's scores and the oracle's away from the
+    cut. 24 tokens per frame (ragged warps)."""
+    spec = S.QerSpec(n_text=n_text, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=10, tokens_per_frame=24,
+                     n_evidence=2, seed=40 + n_text)
+    check(spec, 0.3, kernel=kernel)
+
+
+def test_qer_long_query_integer_inputs_exact():
+    """Integer inputs (every product and sum exact): a 600-token query split
+    into 3 blocks gives exactly the oracle's scores on both kernels."""
+    spec = S.QerSpec(n_text=600, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=7, tokens_per_frame=40, integer=True,
+                     seed=44)
+    for kernel in (1, 2):
+        q, k, _, w_gpu, _ = _run_gpu(spec, 0.5, kernel)
+        w_o = Q.frame_relevance(Q.token_scores(q, k), spec.tokens_per_frame)
+        assert np.allclose(w_gpu, w_o, rtol=2.0 ** -21, atol=0), kernel
