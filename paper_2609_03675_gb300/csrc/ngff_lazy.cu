@@ -3,14 +3,22 @@
 // distance back, so the windowed distances of K2/K3 do not apply; the rule
 // is walked in frame order instead, computing d(c_t, c_{r(t)}) on the fly.
 //
-// One CTA per stream segment. Warp 0 holds c_{t-1} and c_{r(t)} of its
-// stream in registers (lane l: feature words l, l + 32, ...) and walks the
-// frames of a tile of feature rows in shared memory: both distances with one
-// warp reduction each, the decision, and the reference update. The
-// other warps meanwhile stage the next tile from the (L2-resident) feature
-// rows into the other shared-memory buffer with asynchronous copies. The stream's state between
-// pushes is {t, the open scene-change run} and two ring rows: slot 0 holds
-// c_{t-1}, slot 1 holds c_{r(t)}.
+// One CTA per stream segment. Warp 0 walks the frames of a tile of feature
+// rows in shared memory while the other warps stage the next tile from the
+// (L2-resident) feature rows into the other buffer with asynchronous copies.
+// Two walks:
+//   windowed (B <= 64, no scene changes): the reference stays fixed until
+//     the next keep, so lane l scores frame f + l against it (the whole row,
+//     read from a per-lane rotated word so the lanes hit distinct banks);
+//     one ballot finds the first keep in the window, the frames up to it
+//     stand, it becomes the reference, and the next window starts after it.
+//     With a keep every few frames this replaces a warp reduction per frame
+//     by a fraction of one;
+//   serial (otherwise): warp 0 holds c_{r(t)} in registers (lane l: feature
+//     words l, l + 32, ...), one warp reduction per frame, the twin
+//     comparison of scene changes inline.
+// The stream's state between pushes is {t, the open scene-change run} and
+// two ring rows: slot 0 holds c_{t-1}, slot 1 holds c_{r(t)}.
 #include "ngff_common.cuh"
 
 namespace cofie {
@@ -46,6 +54,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   uint32_t* sd = sadj + kLazyMaxRows;                // [rows_per_tile] max(d_adj, d_ref)
   uint8_t* scode = reinterpret_cast<uint8_t*>(sd + kLazyMaxRows);  // [rows_per_tile]
   uint32_t* sprev = reinterpret_cast<uint32_t*>(scode + kLazyMaxRows);  // [B] the row before the tile
+  uint32_t* sref = sprev + kMaxBins;                                    // [B] the reference row (windowed walk)
   const Segment sg = segs.s[blockIdx.x];
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t B = a.bins, n = sg.n;
@@ -81,8 +90,11 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     }
   };
 
-  uint32_t ref[kP];  // warp 0: the reference frame's row
+  const bool windowed = !a.scd && B <= 64;  // uniform
+  uint32_t ref[kP];  // warp 0: the reference frame's row (serial walk)
   unsigned long long acc = 0;
+  if (windowed)
+    for (uint32_t b = tid; b < B; b += kLazyThreads) sref[b] = t0 > 0 ? sring[B + b] : 0u;
   if (warp == 0) {
 #pragma unroll
     for (int q = 0; q < kP; ++q) {
@@ -101,6 +113,35 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     const uint32_t* buf = tiles + (tile & 1) * kLazyTileWords;
     if (warp != 0) {
       if (tile + 1 < n_tiles) stage(tile + 1, 32, kLazyThreads - 32);
+    } else if (windowed) {
+      for (uint32_t f = 0; f < m;) {
+        const uint32_t fl = f + lane;
+        uint32_t dref = 0;
+        if (fl < m) {
+          const uint32_t* row = buf + fl * B;
+          uint32_t b = lane % B;
+          for (uint32_t i = 0; i < B; ++i) {
+            dref += word_dist(row[b], sref[b], a.dist_kind);
+            b = (b + 1 == B) ? 0u : b + 1;
+          }
+        }
+        const uint32_t d = fl < m ? max(sadj[fl], dref) : 0u;
+        const bool first = t0 + j0 + fl == 0;
+        const bool keep = fl < m && (first || d >= a.x_tau);
+        const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+        const uint32_t upto = bal ? static_cast<uint32_t>(__ffs(bal)) - 1 : 31u;  // the last lane whose result stands
+        if (lane <= upto && fl < m && COFIE_BOUND(fl < kLazyMaxRows)) {
+          sd[fl] = d;
+          scode[fl] = first ? 3 : (keep ? 1 : 0);
+        }
+        if (bal) {  // frame f + upto is kept: it becomes the reference
+          __syncwarp();
+          const uint32_t* krow = buf + (f + upto) * B;
+          for (uint32_t bb = lane; bb < B; bb += 32) sref[bb] = krow[bb];
+          __syncwarp();
+        }
+        f += upto + 1;
+      }
     } else {
       uint32_t nxt[kP];
 #pragma unroll
@@ -164,7 +205,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
 #pragma unroll
     for (int q = 0; q < kP; ++q) {
       const uint32_t b = lane + 32 * q;
-      if (b < B) sring[B + b] = ref[q];
+      if (b < B) sring[B + b] = windowed ? sref[b] : ref[q];
     }
     if (lane == 0) {
       state[sg.stream].t = t0 + n;
@@ -177,7 +218,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
 template <int kP>
 cudaError_t launch_p(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
                      StreamState* state, cudaStream_t st) {
-  const size_t smem = 2 * kLazyTileWords * 4 + kLazyMaxRows * (4 + 4 + 1) + kMaxBins * 4;
+  const size_t smem = 2 * kLazyTileWords * 4 + kLazyMaxRows * (4 + 4 + 1) + 2 * kMaxBins * 4;
   cudaError_t e = cudaFuncSetAttribute(lazy_select_kernel<kP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
