@@ -25,7 +25,7 @@ def _frames(w, h, T, seed, mean=9):
     return synth.generate(synth.medium(seed=seed).with_(width=w, height=h, frames=T, mean_scene_len=mean))
 
 
-@pytest.mark.parametrize("bins,tau", [(32, 0.05), (32, 0.3), (7, 0.08), (256, 0.1), (1, 0.0)])
+@pytest.mark.parametrize("bins,tau", [(32, 0.05), (32, 0.3), (7, 0.08), (256, 0.1), (1, 0.0), (32, 1.5)])
 def test_histogram_rule_without_gap(bins, tau):
     from paper_2609_03675_gb300 import NGFF
     w, h, T = 64, 48, 700
