@@ -34,6 +34,10 @@
  *     is enqueued, so they leave the stream state unchanged; a COFIE_ECUDA
  *     from a failed launch may leave earlier pieces of the call enqueued.
  *   - A handle is not thread-safe: calls on one handle must be serialised.
+ *     Its device scratch is shared by all of its calls, so work it enqueues
+ *     on different CUDA streams must also be ordered on the device (one
+ *     stream per handle, or events between the streams); otherwise it races.
+ *     The same holds for a QER handle (cofie_qer_*).
  *   - Nothing aborts, traps or prints. Device-side waits are bounded; a wait
  *     that runs out sets an error word that cofie_ngff_status() reports.
  */
