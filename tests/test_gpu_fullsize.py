@@ -63,6 +63,42 @@ def test_hd1080_whole_stream_push():
     print(f"1080p: {len(cuts)} cuts, {int((got30[cuts] != 0).sum())} retained at tau 0.30")
 
 
+def test_hd1080_without_gap_and_with_scene_changes():
+    """The two other rules the benchmark times on the 1080p stream
+    (`--l-max 0`, `--signal 3`): no forced retention, walked in frame order
+    (the windowed walk), and scene-change detection + H-diff (twin comparison
+    over several 4096-frame scan tiles), against the oracle's rules on the
+    oracle's histograms; keep codes exact, scores within the fp32 bound. The
+    scene-change thresholds sit inside the stream's adjacent-difference
+    distribution so that cuts and gradual runs both occur."""
+    from oracle import scd_oracle as SC
+    from paper_2609_03675_gb300 import NGFF, _abi
+    spec = synth.hd1080()
+    buf = _pinned_stream(spec)
+    dev = buf.cuda()
+    o = O.load()
+    hist_o = o.histograms_parallel(buf.data_ptr(), spec.frames, O.Params(spec.width, spec.height))
+    del buf
+    # L_max = 0
+    p0 = O.Params(spec.width, spec.height, tau=0.30, l_max=0)
+    so, ko = o.select(hist_o, p0)
+    f = NGFF(spec.width, spec.height, tau=0.30, l_max=0, max_frames_per_push=spec.frames)
+    assert_parity(run_stream(f, dev, [spec.frames]), (hist_o, so, ko), 0.30, "1080p L_max=0")
+    assert (ko == O.KEEP_NOVELTY).any() and not (ko == O.KEEP_GAP).any()
+    f.close()
+    # scene changes + H-diff
+    two_n = 2 * spec.width * spec.height
+    sd = np.array([SC.l1(hist_o[t], hist_o[t - 1]) for t in range(1, spec.frames)]) / two_n
+    t_grad, t_cut = float(np.quantile(sd, 0.6)), float(np.quantile(sd, 0.995))
+    p3 = O.Params(spec.width, spec.height, tau=0.30, l_max=30)
+    so, ko = SC.select(hist_o, p3, t_cut, t_grad)
+    assert (ko == SC.KEEP_SCENE).any()
+    f = NGFF(spec.width, spec.height, tau=0.30, l_max=30, signal=_abi.SIGNAL_SCD, scd_cut=t_cut, scd_gradual=t_grad,
+             max_frames_per_push=spec.frames)
+    assert_parity(run_stream(f, dev, [spec.frames]), (hist_o, so, ko), 0.30, "1080p scene changes")
+    f.close()
+
+
 def test_rare_event_720p():
     from paper_2609_03675_gb300 import NGFF
     spec = synth.rare_event()
