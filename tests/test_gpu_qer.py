@@ -116,11 +116,12 @@ def test_qer_planted_evidence_found():
     assert list(sel) == list(ev)
 
 
-@pytest.mark.parametrize("n_frames", [128, 400])
+@pytest.mark.parametrize("n_frames", [128, 400, 1024])
 def test_qer_full_size_sampled(n_frames):
     """The benchmark's geometry: 256 text tokens, frames of 256 tokens, 32/8
     heads of 128; the oracle checks 12 sampled frames. 128 frames fit one
-    wave of the one-SM kernel; 400 frames take the paired-SM kernel."""
+    wave of the one-SM kernel; 400 and 1024 frames (the benchmark's size)
+    take the paired-SM kernel."""
     from paper_2609_03675_gb300 import QER
     spec = S.QerSpec(n_frames=n_frames)
     frames = np.linspace(0, spec.n_frames - 1, 12).astype(int)
