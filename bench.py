@@ -51,6 +51,8 @@ def parse():
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
     ap.add_argument("--qer-frames", type=int, default=128, help="candidate frames of the qer workload")
+    ap.add_argument("--qer-kernel", type=int, default=0, choices=[0, 1, 2],
+                    help="qer scoring kernel: 0 automatic, 1 one-SM, 2 paired-SM")
     ap.add_argument("--l-max", type=int, default=30,
                     help="L_max of the hd1080 workload (0: no forced retention, the rule walked in frame order)")
     ap.add_argument("--signal", choices=["histogram", "lowres", "dhash", "scd"], default="histogram",
@@ -663,7 +665,8 @@ def bench_qer(args):
     q, k, ev = SQ.generate(spec)
     qd = torch.from_numpy(q.view(np.int16)).cuda()
     kd = torch.from_numpy(k.view(np.int16)).cuda()
-    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3)
+    f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3,
+            kernel=args.qer_kernel)
     w = torch.empty(spec.n_frames, dtype=torch.float32, device="cuda")
     sel_all = torch.empty(spec.n_frames, dtype=torch.int32, device="cuda")
     k_dev = torch.zeros(1, dtype=torch.int32, device="cuda")
@@ -702,6 +705,7 @@ def bench_qer(args):
                    "flops_per_launch": pr["flops"] / pr["launches"]},
         "hbm": {"achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
                 "peak_kind": f"{hbm_kind} copy bandwidth", "key_bytes_per_launch": pr["key_bytes"] / pr["launches"]},
+        "kernel_request": {0: "automatic", 1: "one-SM", 2: "paired-SM"}[args.qer_kernel],
         "selected": int(sel.numel()), "evidence_recovered": int(np.isin(ev, sel.cpu().numpy()).sum()),
         "n_evidence": int(len(ev))}), flush=True)
 

@@ -429,9 +429,10 @@ typedef struct {
 /* Scoring kernels: the paired-SM one (clusters of two CTAs, one M = 256 MMA
  * per pair) needs the text block (n_text, or for n_text > 256 its blocks,
  * which are padded to 32) rounded up to 16 to be a multiple of 32; AUTO takes
- * it when it applies and the 256-token tiles of a run exceed one wave of the
- * one-SM kernel (one per SM). The results of the two agree up to the order of
- * fp32 accumulation inside the tensor cores. */
+ * it when it applies and the 256-token tiles of a run either fit one per
+ * co-resident pair (76 on GB300) or exceed one wave of the one-SM kernel (one
+ * per SM). The results of the two agree up to the order of fp32 accumulation
+ * inside the tensor cores. */
 #define COFIE_QER_KERNEL_AUTO 0
 #define COFIE_QER_KERNEL_ONE_SM 1
 #define COFIE_QER_KERNEL_PAIR 2
@@ -442,8 +443,9 @@ int cofie_qer_create(const cofie_qer_params* p, cofie_qer_t** out);
 
 void cofie_qer_destroy(cofie_qer_t* h);
 
-/* COFIE_QER_KERNEL_PAIR if the handle runs the paired-SM kernel for runs
- * above one wave (or always, when asked for), else COFIE_QER_KERNEL_ONE_SM (0 for NULL). */
+/* COFIE_QER_KERNEL_PAIR if the handle can run the paired-SM kernel (AUTO
+ * then picks it per run as described above; PAIR always), else
+ * COFIE_QER_KERNEL_ONE_SM (0 for NULL). */
 uint32_t cofie_qer_kernel_in_use(const cofie_qer_t* h);
 
 /*

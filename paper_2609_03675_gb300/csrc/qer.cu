@@ -1105,9 +1105,12 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   const uint64_t nv = static_cast<uint64_t>(n_frames) * p.tokens_per_frame;
   CUtensorMap map_k, map_q;
   const uint32_t tiles = static_cast<uint32_t>((nv + kQerTile - 1) / kQerTile);
-  // the paired kernel when asked for, or (automatic) when the tiles exceed
-  // one wave of the one-SM kernel: a single wave runs faster on twice the CTAs
-  const bool pair_run = h->pair && (p.kernel == COFIE_QER_KERNEL_PAIR || tiles > static_cast<uint32_t>(h->grid));
+  // the paired kernel when asked for, or (automatic) when every tile gets a
+  // pair of its own (each tile's MMAs split over two SMs: 14 us against 18 us
+  // for up to 76 tiles) or the tiles exceed one wave of the one-SM kernel; in
+  // between (one wave of that kernel, two of the pairs) the two run alike
+  const bool pair_run = h->pair && (p.kernel == COFIE_QER_KERNEL_PAIR || tiles > static_cast<uint32_t>(h->grid) ||
+                                    tiles <= static_cast<uint32_t>(h->pair_clusters));
   const uint32_t q_box = pair_run ? h->n_pad / 2 : h->n_pad;  // the pair's CTAs each stage half of q~
   if (!make_map(&map_k, k, nv, h->D, kQerM)) return h->fail(COFIE_ECUDA, "tensor map encoding failed");
   const uint32_t n_rows = h->n_blk * h->n_pad;

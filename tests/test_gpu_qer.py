@@ -119,15 +119,16 @@ def test_qer_planted_evidence_found():
 @pytest.mark.parametrize("n_frames", [128, 400, 1024])
 def test_qer_full_size_sampled(n_frames):
     """The benchmark's geometry: 256 text tokens, frames of 256 tokens, 32/8
-    heads of 128; the oracle checks 12 sampled frames. 128 frames fit one
-    wave of the one-SM kernel; 400 and 1024 frames (the benchmark's size)
-    take the paired-SM kernel."""
+    heads of 128; the oracle checks 12 sampled frames. 128 frames (128
+    tiles) fit one wave of the one-SM kernel, which the automatic choice
+    takes; 400 and 1024 frames (the benchmark's size) take the paired-SM
+    kernel."""
     from paper_2609_03675_gb300 import QER
     spec = S.QerSpec(n_frames=n_frames)
     frames = np.linspace(0, spec.n_frames - 1, 12).astype(int)
     check(spec, 0.3, frames=frames)
     f = QER(spec.n_text, spec.n_heads, spec.n_kv_heads, spec.head_dim, spec.n_frames, spec.tokens_per_frame, 0.3)
-    assert f.kernel == 2  # the handle can pair; a run switches to it above one wave
+    assert f.kernel == 2  # the handle can pair; a run takes it for one tile per pair or above one wave
 
 
 @pytest.mark.parametrize("kernel", [1, 2])
