@@ -190,6 +190,16 @@ __device__ __forceinline__ float tmem_row_max(uint32_t taddr, uint32_t n_pad, ui
     const bool two = c0 + 32 < n_pad;
     if (two) tmem_ld32_nowait(taddr + c0 + 32, r1);
     tmem_wait_ld();
+    if (c0 + 64 <= n_text) {  // every column of the block is a real text token: no mask
+      float m0 = __uint_as_float(r0[0]), m1 = __uint_as_float(r1[0]);
+#pragma unroll
+      for (uint32_t c = 1; c < 32; ++c) {
+        m0 = fmaxf(m0, __uint_as_float(r0[c]));
+        m1 = fmaxf(m1, __uint_as_float(r1[c]));
+      }
+      best = fmaxf(best, fmaxf(m0, m1));
+      continue;
+    }
 #pragma unroll
     for (uint32_t c = 0; c < 32; ++c)
       if (c0 + c < n_text) best = fmaxf(best, __uint_as_float(r0[c]));
