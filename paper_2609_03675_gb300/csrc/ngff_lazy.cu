@@ -32,9 +32,63 @@ __device__ __forceinline__ uint32_t word_dist(uint32_t x, uint32_t y, uint32_t k
   return kind == 1 ? static_cast<uint32_t>(__popc(x ^ y)) : (x > y ? x - y : y - x);
 }
 
+// The same for B = 4 kQ (kQ a power of two), fully unrolled: every load's
+// address is known up front, so all 2 kQ 16-byte loads are in flight at once.
+template <uint32_t kQ>
+__device__ __forceinline__ uint32_t row_dist_q(const uint32_t* x, const uint32_t* y, uint32_t start, uint32_t kind) {
+  static_assert((kQ & (kQ - 1)) == 0, "kQ must be a power of two");
+  const uint4* x4 = reinterpret_cast<const uint4*>(x);
+  const uint4* y4 = reinterpret_cast<const uint4*>(y);
+  uint32_t s0 = 0, s1 = 0, s2 = 0, s3 = 0;
+#pragma unroll
+  for (uint32_t i = 0; i < kQ; ++i) {
+    const uint32_t q = (start + i) & (kQ - 1);
+    const uint4 u = x4[q], v = y4[q];
+    s0 += word_dist(u.x, v.x, kind);
+    s1 += word_dist(u.y, v.y, kind);
+    s2 += word_dist(u.z, v.z, kind);
+    s3 += word_dist(u.w, v.w, kind);
+  }
+  return (s0 + s1) + (s2 + s3);
+}
+
+// The distance numerator between two feature rows of B words in shared
+// memory, taken by one thread. With B % 4 == 0, 16-byte words starting at
+// the rotated word `start` (lanes that read rows B words apart then touch
+// distinct banks), four independent sums so the loads of four words are in
+// flight together; otherwise word by word from `start`.
+__device__ __forceinline__ uint32_t row_dist(const uint32_t* x, const uint32_t* y, uint32_t B, uint32_t start,
+                                             uint32_t kind) {
+  if (B == 32) return row_dist_q<8>(x, y, start, kind);   // the paper's B
+  if (B == 64) return row_dist_q<16>(x, y, start, kind);
+  if (B % 4 == 0) {
+    const uint32_t Q = B / 4;
+    const uint4* x4 = reinterpret_cast<const uint4*>(x);
+    const uint4* y4 = reinterpret_cast<const uint4*>(y);
+    uint32_t q = start % Q, s0 = 0, s1 = 0, s2 = 0, s3 = 0;
+#pragma unroll 4
+    for (uint32_t i = 0; i < Q; ++i) {
+      const uint4 u = x4[q], v = y4[q];
+      s0 += word_dist(u.x, v.x, kind);
+      s1 += word_dist(u.y, v.y, kind);
+      s2 += word_dist(u.z, v.z, kind);
+      s3 += word_dist(u.w, v.w, kind);
+      q = (q + 1 == Q) ? 0u : q + 1;
+    }
+    return (s0 + s1) + (s2 + s3);
+  }
+  uint32_t b = start % B, sum = 0;
+  for (uint32_t i = 0; i < B; ++i) {
+    sum += word_dist(x[b], y[b], kind);
+    b = (b + 1 == B) ? 0u : b + 1;
+  }
+  return sum;
+}
+
 // Per tile of feature rows (shared memory, double-buffered):
-//   all warps  adjacent distances d_adj[f] = |c_f - c_{f-1}| of the tile;
-//   warp 0     the serial walk: d_ref = |c_f - c_r| (one warp reduction), the
+//   all warps  adjacent distances d_adj[f] = |c_f - c_{f-1}| of the tile (a
+//              thread per row for B <= 64, else a warp per row);
+//   warp 0     the walk (windowed as above, or serial): d_ref = |c_f - c_r|, the
 //              decision as an integer compare against the host-computed
 //              thresholds (the smallest numerators whose fp32 quotient by 2N
 //              reaches tau_h, T_b, T_s; exact since that quotient never
@@ -64,22 +118,43 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   uint32_t* sring = ring + static_cast<uint64_t>(sg.stream) * 2 * B;
   if (n == 0) return;
 
-  // asynchronous 4-byte copies (all of a thread's words in flight at once),
-  // waited for by the staging threads before the block barrier
+  // asynchronous copies (all of a thread's copies in flight at once), 16
+  // bytes when B % 4 == 0 (the rows of the tile are then 16-byte aligned:
+  // the feature array and the tile buffers are), else 4; waited for by the
+  // staging threads before the block barrier
+  const bool vec16 = B % 4 == 0;
   auto stage = [&](uint32_t tile, uint32_t first_thread, uint32_t threads) {
     const uint32_t j0 = tile * rows_per_tile, m = min(rows_per_tile, n - j0);
     uint32_t* dst = tiles + (tile & 1) * kLazyTileWords;
     const uint32_t* src = feat + static_cast<uint64_t>(sg.row0 + j0) * B;
-    for (uint32_t i = tid - first_thread; i < m * B; i += threads)
-      asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst + i))),
-                   "l"(src + i)
-                   : "memory");
+    if (vec16) {
+      for (uint32_t i = 4 * (tid - first_thread); i < m * B; i += 4 * threads)
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                         static_cast<uint32_t>(__cvta_generic_to_shared(dst + i))),
+                     "l"(src + i)
+                     : "memory");
+    } else {
+      for (uint32_t i = tid - first_thread; i < m * B; i += threads)
+        asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                         static_cast<uint32_t>(__cvta_generic_to_shared(dst + i))),
+                     "l"(src + i)
+                     : "memory");
+    }
     asm volatile("cp.async.commit_group;\ncp.async.wait_all;" ::: "memory");
   };
-  // adjacent numerators of a staged tile: warp w takes rows w, w + 8, ...
+  // adjacent numerators of a staged tile: for B <= 64 a thread per row
+  // (row_dist), else warp w takes rows w, w + 8, ... (a warp reduction each)
   auto adjacent = [&](uint32_t tile) {
     const uint32_t j0 = tile * rows_per_tile, m = min(rows_per_tile, n - j0);
     const uint32_t* buf = tiles + (tile & 1) * kLazyTileWords;
+    if (B <= 64) {
+      for (uint32_t f = tid; f < m; f += kLazyThreads) {
+        const uint32_t* c = buf + f * B;
+        const uint32_t d = row_dist(c, f ? c - B : sprev, B, lane, a.dist_kind);
+        if (COFIE_BOUND(f < kLazyMaxRows)) sadj[f] = d;
+      }
+      return;
+    }
     for (uint32_t f = warp; f < m; f += kLazyThreads / 32) {
       const uint32_t* c = buf + f * B;
       const uint32_t* p = f ? c - B : sprev;
@@ -116,15 +191,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     } else if (windowed) {
       for (uint32_t f = 0; f < m;) {
         const uint32_t fl = f + lane;
-        uint32_t dref = 0;
-        if (fl < m) {
-          const uint32_t* row = buf + fl * B;
-          uint32_t b = lane % B;
-          for (uint32_t i = 0; i < B; ++i) {
-            dref += word_dist(row[b], sref[b], a.dist_kind);
-            b = (b + 1 == B) ? 0u : b + 1;
-          }
-        }
+        const uint32_t dref = fl < m ? row_dist(buf + fl * B, sref, B, lane, a.dist_kind) : 0u;
         const uint32_t d = fl < m ? max(sadj[fl], dref) : 0u;
         const bool first = t0 + j0 + fl == 0;
         const bool keep = fl < m && (first || d >= a.x_tau);
