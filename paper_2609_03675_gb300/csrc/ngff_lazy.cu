@@ -7,16 +7,17 @@
 // rows in shared memory while the other warps stage the next tile from the
 // (L2-resident) feature rows into the other buffer with asynchronous copies.
 // Two walks:
-//   windowed (B <= 64, no scene changes): the reference stays fixed until
+//   windowed (no scene changes): the reference stays fixed until
 //     the next keep, so lane l scores frame f + l against it (the whole row,
 //     read from a per-lane rotated word so the lanes hit distinct banks);
 //     one ballot finds the first keep in the window, the frames up to it
 //     stand, it becomes the reference, and the next window starts after it.
 //     With a keep every few frames this replaces a warp reduction per frame
 //     by a fraction of one;
-//   serial (otherwise): warp 0 holds c_{r(t)} in registers (lane l: feature
-//     words l, l + 32, ...), one warp reduction per frame, the twin
-//     comparison of scene changes inline.
+//   serial (scene changes): warp 0 holds c_{r(t)} in registers (lane l:
+//     feature words l, l + 32, ...), one warp reduction per frame, the twin
+//     comparison of scene changes inline (its open run depends on every
+//     frame's adjacent difference in order).
 // The stream's state between pushes is {t, the open scene-change run} and
 // two ring rows: slot 0 holds c_{t-1}, slot 1 holds c_{r(t)}.
 #include "ngff_common.cuh"
@@ -165,7 +166,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     }
   };
 
-  const bool windowed = !a.scd && B <= 64;  // uniform
+  const bool windowed = !a.scd;  // uniform
   uint32_t ref[kP];  // warp 0: the reference frame's row (serial walk)
   unsigned long long acc = 0;
   if (windowed)
