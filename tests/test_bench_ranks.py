@@ -8,6 +8,8 @@ import socket
 import pytest
 import torch.multiprocessing as mp
 
+REPO = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
 
 def _free_port():
     with socket.socket() as s:
@@ -51,3 +53,36 @@ def test_single_process_needs_no_group():
     import bench
     assert bench.max_over_ranks(3.5, device="cpu") == 3.5
     assert bench.whole_job_rate(100, 1, 0.5) == 200.0
+
+
+def _bench(args, env=None):
+    import json
+    import subprocess
+    import sys
+    e = dict(os.environ)
+    e.update(env or {})
+    r = subprocess.run([sys.executable, os.path.join(REPO, "bench.py"), *args], capture_output=True, text=True,
+                       timeout=600, env=e, cwd=REPO)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    return [json.loads(ln) for ln in lines]
+
+
+def test_reference_arm_prints_the_contract_line():
+    """`bench.py --impl reference` (the oracle on host cores) prints one JSON
+    line with the benchmark's keys, a cpu_baseline describing the run, and an
+    e2e object with no host-device bytes."""
+    (d,) = _bench(["--impl", "reference", "--steps", "1", "--warmup", "0"])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["unit"] == "frames/s"
+    for key in ("metric", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling", "dtype", "data"):
+        assert key in d, key
+    assert d["vs_baseline"] is None and d["higher_is_better"] is True and d["steps"] == 1
+    assert "workload" in d["config"]
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_reference_arm_other_ranks_do_no_work():
+    """Under torchrun only rank 0 runs the reference arm; the others exit 0 silently."""
+    assert _bench(["--impl", "reference", "--steps", "1", "--warmup", "0"], {"RANK": "1", "WORLD_SIZE": "2"}) == []
