@@ -6,18 +6,15 @@
 // One CTA per stream segment. Warp 0 walks the frames of a tile of feature
 // rows in shared memory while the other warps stage the next tile from the
 // (L2-resident) feature rows into the other buffer with asynchronous copies.
-// Two walks:
-//   windowed (no scene changes): the reference stays fixed until
-//     the next keep, so lane l scores frame f + l against it (the whole row,
-//     read from a per-lane rotated word so the lanes hit distinct banks);
-//     one ballot finds the first keep in the window, the frames up to it
-//     stand, it becomes the reference, and the next window starts after it.
-//     With a keep every few frames this replaces a warp reduction per frame
-//     by a fraction of one;
-//   serial (scene changes): warp 0 holds c_{r(t)} in registers (lane l:
-//     feature words l, l + 32, ...), one warp reduction per frame, the twin
-//     comparison of scene changes inline (its open run depends on every
-//     frame's adjacent difference in order).
+// The walk goes by windows: the reference stays fixed until the next keep,
+// so lane l scores frame f + l against it (the whole row, read from a
+// per-lane rotated word so the lanes hit distinct banks); one ballot finds
+// the first keep in the window, the frames up to it stand, it becomes the
+// reference, and the next window starts after it. With a keep every few
+// frames this replaces a warp reduction per frame by a fraction of one.
+// Scene changes (twin comparison) depend only on the adjacent differences,
+// not on the reference, so a tile's scene flags are found first, by a scan,
+// and enter the walk as keeps.
 // The stream's state between pushes is {t, the open scene-change run} and
 // two ring rows: slot 0 holds c_{t-1}, slot 1 holds c_{r(t)}.
 #include "ngff_common.cuh"
@@ -86,19 +83,31 @@ __device__ __forceinline__ uint32_t row_dist(const uint32_t* x, const uint32_t* 
   return sum;
 }
 
+// The twin comparison's run as a monoid: a frame ends the open run (reset,
+// the run restarts at sum 0 after it) or adds its adjacent numerator to it.
+struct LzRun {
+  uint32_t reset;
+  unsigned long long sum;
+};
+__device__ __forceinline__ LzRun lz_cat(LzRun x, LzRun y) { return y.reset ? y : LzRun{x.reset, x.sum + y.sum}; }
+__device__ __forceinline__ LzRun lz_shfl_up(LzRun v, uint32_t off) {
+  return LzRun{__shfl_up_sync(0xffffffffu, v.reset, off), __shfl_up_sync(0xffffffffu, v.sum, off)};
+}
+
 // Per tile of feature rows (shared memory, double-buffered):
 //   all warps  adjacent distances d_adj[f] = |c_f - c_{f-1}| of the tile (a
 //              thread per row for B <= 64, else a warp per row);
-//   warp 0     the walk (windowed as above, or serial): d_ref = |c_f - c_r|, the
-//              decision as an integer compare against the host-computed
+//   warp 0     with scene changes, the tile's scene flags first (a scan of
+//              the run monoid: a lane takes a run of consecutive frames, the
+//              runs are scanned across the warp, each lane replays its run
+//              from its prefix), then the windowed walk: d_ref = |c_f - c_r|,
+//              the decision as an integer compare against the host-computed
 //              thresholds (the smallest numerators whose fp32 quotient by 2N
 //              reaches tau_h, T_b, T_s; exact since that quotient never
-//              decreases as the numerator grows), the scene-change run, and
-//              the reference update; meanwhile the other warps stage the
-//              next tile with asynchronous copies;
+//              decreases as the numerator grows), and the reference update;
+//              meanwhile the other warps stage the next tile with
+//              asynchronous copies;
 //   all warps  the tile's fp32 scores and keep codes to global memory.
-// kP feature words per lane in the walk (B <= 32 kP).
-template <int kP>
 __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs, SelectArgs a,
                                                                    const uint32_t* __restrict__ feat,
                                                                    uint32_t* __restrict__ ring,
@@ -108,8 +117,9 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   uint32_t* sadj = tiles + 2 * kLazyTileWords;       // [rows_per_tile] adjacent numerators
   uint32_t* sd = sadj + kLazyMaxRows;                // [rows_per_tile] max(d_adj, d_ref)
   uint8_t* scode = reinterpret_cast<uint8_t*>(sd + kLazyMaxRows);  // [rows_per_tile]
-  uint32_t* sprev = reinterpret_cast<uint32_t*>(scode + kLazyMaxRows);  // [B] the row before the tile
-  uint32_t* sref = sprev + kMaxBins;                                    // [B] the reference row (windowed walk)
+  uint8_t* sscene = scode + kLazyMaxRows;                          // [rows_per_tile] scene-change flags
+  uint32_t* sprev = reinterpret_cast<uint32_t*>(sscene + kLazyMaxRows);  // [B] the row before the tile
+  uint32_t* sref = sprev + kMaxBins;                                     // [B] the reference row
   const Segment sg = segs.s[blockIdx.x];
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t B = a.bins, n = sg.n;
@@ -166,20 +176,11 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     }
   };
 
-  const bool windowed = !a.scd;  // uniform
-  uint32_t ref[kP];  // warp 0: the reference frame's row (serial walk)
-  unsigned long long acc = 0;
-  if (windowed)
-    for (uint32_t b = tid; b < B; b += kLazyThreads) sref[b] = t0 > 0 ? sring[B + b] : 0u;
-  if (warp == 0) {
-#pragma unroll
-    for (int q = 0; q < kP; ++q) {
-      const uint32_t b = lane + 32 * q;
-      ref[q] = (t0 > 0 && b < B) ? sring[B + b] : 0u;
-    }
-    acc = t0 > 0 ? state[sg.stream].acc : 0ull;
+  unsigned long long acc = t0 > 0 ? state[sg.stream].acc : 0ull;  // warp 0: the scene-change run open so far
+  for (uint32_t b = tid; b < B; b += kLazyThreads) {
+    sref[b] = t0 > 0 ? sring[B + b] : 0u;
+    sprev[b] = t0 > 0 ? sring[b] : 0u;
   }
-  for (uint32_t b = tid; b < B; b += kLazyThreads) sprev[b] = t0 > 0 ? sring[b] : 0u;
   stage(0, 0, kLazyThreads);
   __syncthreads();
   adjacent(0);
@@ -189,18 +190,53 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     const uint32_t* buf = tiles + (tile & 1) * kLazyTileWords;
     if (warp != 0) {
       if (tile + 1 < n_tiles) stage(tile + 1, 32, kLazyThreads - 32);
-    } else if (windowed) {
+    } else {
+      if (a.scd) {
+        // scene flags: frame f cuts (d_adj >= T_b: a scene change that ends
+        // the run), joins the run (T_s <= d_adj < T_b: a scene change when
+        // the run's sum first reaches T_b) or ends it; the stream's first
+        // frame is neither (the identity)
+        const uint32_t per = (m + 31) / 32, f0 = min(lane * per, m), f1 = min(f0 + per, m);
+        auto elem = [&](uint32_t f) {
+          const uint32_t d = sadj[f];
+          if (t0 + j0 + f == 0) return LzRun{0u, 0ull};
+          return (d >= a.x_cut || d < a.x_grad) ? LzRun{1u, 0ull} : LzRun{0u, d};
+        };
+        LzRun run{0u, 0ull};
+        for (uint32_t f = f0; f < f1; ++f) run = lz_cat(run, elem(f));
+        LzRun incl = run;
+#pragma unroll
+        for (uint32_t off = 1; off < 32; off <<= 1) {
+          const LzRun o = lz_shfl_up(incl, off);
+          if (lane >= off) incl = lz_cat(o, incl);
+        }
+        LzRun pre = lz_shfl_up(incl, 1);
+        if (lane == 0) pre = LzRun{0u, 0ull};
+        for (uint32_t f = f0; f < f1; ++f) {
+          const uint32_t d = sadj[f];
+          pre = lz_cat(pre, elem(f));
+          const unsigned long long r = pre.reset ? pre.sum : acc + pre.sum;  // the run's sum at f
+          const bool first = t0 + j0 + f == 0;
+          const bool scene = !first && (d >= a.x_cut || (d >= a.x_grad && r >= a.x_cut && r - d < a.x_cut));
+          if (COFIE_BOUND(f < kLazyMaxRows)) sscene[f] = scene ? 1 : 0;
+        }
+        const LzRun total{__shfl_sync(0xffffffffu, incl.reset, 31), __shfl_sync(0xffffffffu, incl.sum, 31)};
+        acc = total.reset ? total.sum : acc + total.sum;
+        __syncwarp();
+      }
+      // the windowed walk
       for (uint32_t f = 0; f < m;) {
         const uint32_t fl = f + lane;
         const uint32_t dref = fl < m ? row_dist(buf + fl * B, sref, B, lane, a.dist_kind) : 0u;
         const uint32_t d = fl < m ? max(sadj[fl], dref) : 0u;
         const bool first = t0 + j0 + fl == 0;
-        const bool keep = fl < m && (first || d >= a.x_tau);
+        const bool nov = d >= a.x_tau, scene = a.scd && fl < m && sscene[fl];
+        const bool keep = fl < m && (first || nov || scene);
         const uint32_t bal = __ballot_sync(0xffffffffu, keep);
         const uint32_t upto = bal ? static_cast<uint32_t>(__ffs(bal)) - 1 : 31u;  // the last lane whose result stands
         if (lane <= upto && fl < m && COFIE_BOUND(fl < kLazyMaxRows)) {
           sd[fl] = d;
-          scode[fl] = first ? 3 : (keep ? 1 : 0);
+          scode[fl] = first ? 3 : (nov ? 1 : (scene ? 4 : 0));
         }
         if (bal) {  // frame f + upto is kept: it becomes the reference
           __syncwarp();
@@ -209,47 +245,6 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
           __syncwarp();
         }
         f += upto + 1;
-      }
-    } else {
-      uint32_t nxt[kP];
-#pragma unroll
-      for (int q = 0; q < kP; ++q) nxt[q] = (lane + 32 * q < B) ? buf[lane + 32 * q] : 0u;
-      for (uint32_t f = 0; f < m; ++f) {
-        uint32_t cur[kP];
-        uint32_t pr = 0;
-#pragma unroll
-        for (int q = 0; q < kP; ++q) {
-          cur[q] = nxt[q];
-          const uint32_t b = lane + 32 * q;
-          nxt[q] = (f + 1 < m && b < B) ? buf[(f + 1) * B + b] : 0u;  // the next row, off the chain
-          pr += word_dist(cur[q], ref[q], a.dist_kind);
-        }
-        const uint32_t d_adj = sadj[f];
-        const uint32_t d = max(d_adj, __reduce_add_sync(0xffffffffu, pr));
-        uint8_t code;
-        if (t0 + j0 + f == 0) {
-          code = 3;  // the stream's first frame
-        } else {
-          bool scene = false;
-          if (a.scd) {  // twin comparison on the adjacent difference
-            if (d_adj >= a.x_cut) {
-              scene = true;
-              acc = 0;
-            } else if (d_adj >= a.x_grad) {
-              scene = acc < a.x_cut && acc + d_adj >= a.x_cut;  // the run's sum first reaches T_b
-              acc += d_adj;
-            } else {
-              acc = 0;
-            }
-          }
-          code = d >= a.x_tau ? 1 : (scene ? 4 : 0);
-        }
-        if (lane == 0 && COFIE_BOUND(f < kLazyMaxRows && (f + 1) * B <= kLazyTileWords)) {
-          sd[f] = d;
-          scode[f] = code;
-        }
-#pragma unroll
-        for (int q = 0; q < kP; ++q) ref[q] = code ? cur[q] : ref[q];
       }
     }
     __syncthreads();
@@ -268,41 +263,27 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   // the ring: slot 0 the last frame's row, slot 1 the reference's
   const uint32_t last = (n - 1) - (n_tiles - 1) * rows_per_tile;
   const uint32_t* lbuf = tiles + ((n_tiles - 1) & 1) * kLazyTileWords;
-  for (uint32_t b = tid; b < B; b += kLazyThreads) sring[b] = lbuf[last * B + b];
-  if (warp == 0) {
-#pragma unroll
-    for (int q = 0; q < kP; ++q) {
-      const uint32_t b = lane + 32 * q;
-      if (b < B) sring[B + b] = windowed ? sref[b] : ref[q];
-    }
-    if (lane == 0) {
-      state[sg.stream].t = t0 + n;
-      state[sg.stream].g = 1;
-      state[sg.stream].acc = acc;
-    }
+  for (uint32_t b = tid; b < B; b += kLazyThreads) {
+    sring[b] = lbuf[last * B + b];
+    sring[B + b] = sref[b];
   }
-}
-
-template <int kP>
-cudaError_t launch_p(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
-                     StreamState* state, cudaStream_t st) {
-  const size_t smem = 2 * kLazyTileWords * 4 + kLazyMaxRows * (4 + 4 + 1) + 2 * kMaxBins * 4;
-  cudaError_t e = cudaFuncSetAttribute(lazy_select_kernel<kP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
-  if (e != cudaSuccess) return e;
-  lazy_select_kernel<kP><<<segs.count, kLazyThreads, smem, st>>>(segs, a, feat, ring, state);
-  return cudaGetLastError();
+  if (tid == 0) {
+    state[sg.stream].t = t0 + n;
+    state[sg.stream].g = 1;
+    state[sg.stream].acc = acc;
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_lazy_select(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
                                StreamState* state, cudaStream_t st) {
-  const uint32_t per = (a.bins + 31) / 32;
-  if (per <= 1) return launch_p<1>(segs, a, feat, ring, state, st);
-  if (per <= 2) return launch_p<2>(segs, a, feat, ring, state, st);
-  if (per <= 4) return launch_p<4>(segs, a, feat, ring, state, st);
-  return launch_p<8>(segs, a, feat, ring, state, st);
+  const size_t smem = 2 * kLazyTileWords * 4 + kLazyMaxRows * (4 + 4 + 1 + 1) + 2 * kMaxBins * 4;
+  cudaError_t e = cudaFuncSetAttribute(lazy_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  lazy_select_kernel<<<segs.count, kLazyThreads, smem, st>>>(segs, a, feat, ring, state);
+  return cudaGetLastError();
 }
 
 uint32_t take_bounds_errors_lazy() { return take_local_bounds_errors(); }

@@ -97,6 +97,13 @@ def test_hd1080_without_gap_and_with_scene_changes():
              max_frames_per_push=spec.frames)
     assert_parity(run_stream(f, dev, [spec.frames]), (hist_o, so, ko), 0.30, "1080p scene changes")
     f.close()
+    # scene changes without forced retention (the walk with scanned scene flags)
+    so, ko = SC.select(hist_o, O.Params(spec.width, spec.height, tau=0.30, l_max=0), t_cut, t_grad)
+    assert (ko == SC.KEEP_SCENE).any() and not (ko == O.KEEP_GAP).any()
+    f = NGFF(spec.width, spec.height, tau=0.30, l_max=0, signal=_abi.SIGNAL_SCD, scd_cut=t_cut, scd_gradual=t_grad,
+             max_frames_per_push=spec.frames)
+    assert_parity(run_stream(f, dev, [spec.frames]), (hist_o, so, ko), 0.30, "1080p scene changes, L_max=0")
+    f.close()
 
 
 def test_rare_event_720p():
