@@ -42,7 +42,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=600)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=7)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards",
@@ -304,7 +304,8 @@ def bench_gb300(args):
             fe.reset()
             fe.push(host, scores=hs, keep=hk)
 
-        estep()
+        for _ in range(2):  # untimed: the first passes over the pinned buffer are the slowest
+            estep()
         torch.cuda.synchronize()
         # the raw host->device link over the same bytes (one plain copy of the
         # whole pinned stream into the device frame tensor), measured right
