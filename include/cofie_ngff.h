@@ -59,7 +59,8 @@ extern "C" {
 #define COFIE_ENOMEM 2   /* a device or pinned-host allocation failed */
 #define COFIE_ECUDA 3    /* a CUDA runtime call failed */
 #define COFIE_ETIMEOUT 4 /* a device-side bounded wait ran out (cofie_ngff_status) */
-#define COFIE_EDEVICE 5  /* a device-side check failed: a gather index outside the frames (cofie_ngff_status) */
+#define COFIE_EDEVICE 5  /* a device-side check failed: a gather index outside the frames, or in a build with
+                            -DCOFIE_DEBUG_CHECKS=1 an index or layout check (cofie_ngff_status, cofie_qer_status) */
 
 /* Keep codes written to keep_out. Nonzero means retained (a candidate). */
 #define COFIE_KEEP_DROP 0
@@ -88,8 +89,9 @@ typedef struct cofie_ngff cofie_ngff_t;
  *   l_max             L_max in sampled-frame indices, 0..256; default 30 (App. B.2).
  *                     0 turns the forced retention (Eq. 5's second term) off:
  *                     frames are then kept only as first, novelty or scene
- *                     change, the rule is walked in frame order by one warp
- *                     per stream, and the stream cannot be sharded.
+ *                     change, the rule is walked in frame order (by windows
+ *                     of 32 frames between keeps, one warp per stream), and
+ *                     the stream cannot be sharded.
  *   m_min             M_min, used by cofie_ngff_candidates only; default 4 (App. B.2).
  *   tau               tau_h, any non-NaN float; default 0.30f (App. B.2).
  *   luma_w, luma_den  grayscale weights (wR, wG, wB) / den; each weight <= 65535,
@@ -241,7 +243,8 @@ int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames,
  * "NGFS", version 2, width, height, bins, l_max, signal, frames seen t,
  * current gap g, the scene-change signal's open run sum) followed by the ring
  * of the last l_max feature rows (l_max * cofie_ngff_feature_words uint32,
- * slot i holds the frame t' with t' mod l_max == i).
+ * slot i holds the frame t' with t' mod l_max == i; for l_max == 0 two rows,
+ * the previous frame's and the current reference frame's).
  *   cofie_ngff_state_bytes   the size of that buffer.
  *   cofie_ngff_state_save    writes stream `stream`'s state to buf (device or
  *                            host memory; host memory synchronises cuda_stream).
