@@ -1,0 +1,72 @@
+/* A plain C client of libcofie_ngff.so (no CUDA runtime, no Python): reads
+ * frames from a file, pushes them from pageable host memory in pieces of the
+ * given sizes, and writes every frame's score and keep code (host outputs)
+ * to an output file.
+ * Usage: ngff_client IN OUT WIDTH HEIGHT FRAMES TAU L_MAX PIECE...
+ * IN holds FRAMES * WIDTH * HEIGHT * 3 bytes; OUT receives FRAMES floats and
+ * FRAMES keep bytes. Exit status 0 on success; a failing call prints the
+ * library's message. */
+#include <stdint.h>
+#include <stdio.h>
+#include <stdlib.h>
+
+#include "cofie_ngff.h"
+
+static int check(int rc, cofie_ngff_t* h, const char* what) {
+  if (rc != COFIE_OK) {
+    fprintf(stderr, "%s failed (%d): %s\n", what, rc, h ? cofie_ngff_last_error(h) : cofie_ngff_global_error());
+    return 1;
+  }
+  return 0;
+}
+
+int main(int argc, char** argv) {
+  if (argc < 9) {
+    fprintf(stderr, "usage: %s IN OUT WIDTH HEIGHT FRAMES TAU L_MAX PIECE...\n", argv[0]);
+    return 2;
+  }
+  const uint32_t W = (uint32_t)strtoul(argv[3], NULL, 10), H = (uint32_t)strtoul(argv[4], NULL, 10);
+  const uint32_t T = (uint32_t)strtoul(argv[5], NULL, 10);
+  const size_t frame_bytes = (size_t)W * H * 3;
+  uint8_t* frames = malloc(frame_bytes * T);
+  float* scores = malloc(sizeof(float) * T);
+  uint8_t* keep = malloc(T);
+  if (!frames || !scores || !keep) return 3;
+  FILE* in = fopen(argv[1], "rb");
+  if (!in || fread(frames, 1, frame_bytes * T, in) != frame_bytes * T) return 4;
+  fclose(in);
+
+  cofie_ngff_params p;
+  cofie_ngff_default_params(&p, W, H);
+  p.tau = strtof(argv[6], NULL);
+  p.l_max = (uint32_t)strtoul(argv[7], NULL, 10);
+  p.max_frames_per_push = T ? T : 1;
+  cofie_ngff_t* h = NULL;
+  if (check(cofie_ngff_create(&p, &h), NULL, "cofie_ngff_create")) return 1;
+
+  uint32_t off = 0;
+  for (int a = 8; a < argc && off < T; ++a) {
+    uint32_t n = (uint32_t)strtoul(argv[a], NULL, 10);
+    if (n > T - off) n = T - off;
+    if (check(cofie_ngff_push(h, 0, frames + (size_t)off * frame_bytes, n, scores + off, keep + off, NULL), h,
+              "cofie_ngff_push"))
+      return 1;
+    off += n;
+  }
+  if (off != T) {
+    fprintf(stderr, "pieces cover %u of %u frames\n", off, T);
+    return 2;
+  }
+  if (check(cofie_ngff_status(h, NULL), h, "cofie_ngff_status")) return 1;
+  cofie_ngff_destroy(h);
+
+  FILE* out = fopen(argv[2], "wb");
+  if (!out) return 5;
+  fwrite(scores, sizeof(float), T, out);
+  fwrite(keep, 1, T, out);
+  fclose(out);
+  free(frames);
+  free(scores);
+  free(keep);
+  return 0;
+}

@@ -121,3 +121,19 @@ def test_qer_create_rejects_bad_params_without_gpu(lib, field, value, msg):
     assert lib.cofie_qer_create(ctypes.byref(p), ctypes.byref(h)) == _abi.EINVAL
     assert msg in lib.cofie_qer_last_error(None).decode()
     assert not h.value
+
+
+def test_header_is_c99_and_a_c_client_links(tmp_path):
+    """include/cofie_ngff.h compiles as C99 (warnings are errors) and a C
+    client links against the library alone."""
+    import shutil
+    import subprocess
+    from paper_2609_03675_gb300 import _abi
+    if shutil.which("gcc") is None:
+        pytest.skip("no gcc")
+    lib_dir = os.path.dirname(_abi.LIB_PATH)
+    exe = tmp_path / "ngff_client"
+    r = subprocess.run(["gcc", "-std=c99", "-O2", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(REPO, "include"),
+                        os.path.join(REPO, "tests", "c", "ngff_client.c"), "-o", str(exe), "-L", lib_dir,
+                        "-lcofie_ngff", f"-Wl,-rpath,{lib_dir}"], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
