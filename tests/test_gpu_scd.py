@@ -167,3 +167,25 @@ def test_state_carries_an_open_run_and_sharding_is_refused():
     assert e.value.code == _abi.EINVAL
     with pytest.raises(NGFFError):  # a histogram-signal state does not load into a scene-change handle
         NGFF(W, H, **kw).state_load(NGFF(W, H, tau=1.5, l_max=256).state_save())
+
+
+@pytest.mark.parametrize("t_cut,t_grad", [(0.02, 0.05), (0.03, 0.03)])
+@pytest.mark.parametrize("l_max", [30, 0])
+def test_gradual_threshold_at_or_above_the_cut(t_cut, t_grad, l_max):
+    """T_s >= T_b: no difference lies between them, so no run ever opens and
+    every scene change is a cut; both selection kernels (scan tiles for
+    L_max > 0, the walk with scanned scene flags for L_max = 0) must agree
+    with the oracle."""
+    from paper_2609_03675_gb300 import NGFF, _abi
+    T = 3000
+    pos = _walk(T, seed=900 + l_max)
+    fr = _frames_from_positions(pos)
+    p = O.Params(W, H, tau=1.5, l_max=l_max)
+    so, ko = _oracle(fr, p, t_cut, t_grad)
+    assert (ko == SC.KEEP_SCENE).sum() > 10
+    dev = torch.from_numpy(fr).cuda()
+    for chunks in ([T], [1, 999, 2000]):
+        f = NGFF(W, H, tau=1.5, l_max=l_max, signal=_abi.SIGNAL_SCD, scd_cut=t_cut, scd_gradual=t_grad,
+                 max_frames_per_push=T)
+        sg, kg = _run(f, dev, chunks)
+        _assert_same(sg, kg, so, ko, f"T_b {t_cut} T_s {t_grad} L_max {l_max} {chunks[:2]}")
