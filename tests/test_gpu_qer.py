@@ -183,3 +183,15 @@ def test_qer_long_query_integer_inputs_exact():
         q, k, _, w_gpu, _ = _run_gpu(spec, 0.5, kernel)
         w_o = Q.frame_relevance(Q.token_scores(q, k), spec.tokens_per_frame)
         assert np.allclose(w_gpu, w_o, rtol=2.0 ** -21, atol=0), kernel
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_qer_at_its_limits(kernel):
+    """The largest key width (H_kv * d_h = 16384: 256 K chunks per tile) and
+    the longest query (4096 text tokens: 16 passes over the keys)."""
+    wide = S.QerSpec(n_text=64, n_heads=128, n_kv_heads=128, head_dim=128, n_frames=4, tokens_per_frame=32,
+                     n_evidence=1, seed=51)
+    check(wide, 0.5, kernel=kernel)
+    long_q = S.QerSpec(n_text=4096, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=5, tokens_per_frame=40,
+                       n_evidence=1, seed=52)
+    check(long_q, 0.4, kernel=kernel)
