@@ -32,7 +32,8 @@ METRIC = "NGFF frames/s and pixel GB/s (fraction of HBM peak) at 1 GB300 vs CPU 
 UNIT = "frames/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-K1_SOURCES = [os.path.join(REPO, "paper_2609_03675_gb300", "csrc", f) for f in ("ngff_hist.cu", "ngff_device.cuh")]
+K1_SOURCES = [os.path.join(REPO, "paper_2609_03675_gb300", "csrc", f)
+              for f in ("ngff_hist.cu", "ngff_device.cuh", "ngff_common.cuh")]
 K1_TRAFFIC = os.path.join(REPO, "profiles", "k1_hist_1080p_traffic.json")
 
 
@@ -98,7 +99,7 @@ def peaks():
 
 
 def k1_source_hash() -> str:
-    """sha256 over K1's sources (the kernel file and its device helpers)."""
+    """sha256 over K1's sources (the kernel file, its device helpers and the common header)."""
     h = hashlib.sha256()
     for path in K1_SOURCES:
         h.update(open(path, "rb").read())

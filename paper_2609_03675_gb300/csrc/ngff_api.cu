@@ -245,7 +245,7 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
     const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->cells_grid) ? chunks : h->cells_grid);
     const bool dhash = h->p.signal == COFIE_SIGNAL_DHASH;
     cudaError_t e = launch_cells_fast(segs, ha, h->lc, dhash ? h->d_cells : h->d_hist, h->d_err, grid, st);
-    if (e == cudaSuccess && dhash) e = launch_dhash_finish(h->d_cells, segs.rows, h->fa, h->d_hist, st);
+    if (e == cudaSuccess && dhash) e = launch_dhash_finish(h->d_cells, segs.rows, h->fa, h->d_hist, st, true);
     return e;
   }
   if (fast) {
@@ -324,17 +324,17 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
   cudaEvent_t es0 = nullptr, es1 = nullptr;
   if (h->time_kernels && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
   if (h->p.l_max == 0) {  // no forced retention: the rule walked in frame order
-    e = launch_lazy_select(segs, sa, h->d_hist, h->d_ring, h->d_state, st);
+    e = launch_lazy_select(segs, sa, h->d_hist, h->d_ring, h->d_state, st, !ev0);
     if (e != cudaSuccess) return h->cuda_fail(e, "lazy selection kernel launch");
     h->n_select += 1;
   } else if (fused) {  // distances and scan in one launch
-    e = launch_select_small(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
+    e = launch_select_small(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st, !ev0);
     if (e != cudaSuccess) return h->cuda_fail(e, "selection kernel launch");
     h->n_select += 1;
   } else {
-    e = launch_window(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st);
+    e = launch_window(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st, !ev0);
     if (e != cudaSuccess) return h->cuda_fail(e, "window kernel launch");
-    e = launch_scan(segs, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st);
+    e = launch_scan(segs, sa, h->d_l1, h->d_mask, h->d_hist, h->d_ring, h->d_state, st, !es0);
     if (e != cudaSuccess) return h->cuda_fail(e, "scan kernel launch");
     h->n_select += 2;
   }

@@ -67,6 +67,34 @@ struct StreamState {
   unsigned long long acc;  // scene-change signal: L1 numerator summed over the open gradual run (0: none)
 };
 
+// Programmatic dependent launch inside one push: the first-stage kernel lets
+// the selection kernels that follow it be scheduled early (pdl_trigger), and
+// those wait for it (pdl_wait) before their first read of its output, so
+// their launch and set-up overlap its tail. Only launches whose predecessor
+// in the stream is the library's own kernel of the same push use it (the
+// first-stage kernel itself is an ordinary launch: a caller's kernel writing
+// the frames may precede it). Both instructions are no-ops for a kernel
+// launched without the attribute.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// A launch that is a programmatic dependent of the kernel before it when pdl.
+template <typename... Params, typename... Args>
+inline cudaError_t launch_dependent(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                                    cudaStream_t st, Args... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Index checks of the checked build (-DCOFIE_DEBUG_CHECKS=1), which stands in
 // for a memory checker: COFIE_BOUND(c) is true in normal builds (and
 // compiles away); in checked builds a false c sets this translation unit's
@@ -178,21 +206,22 @@ cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const Luma
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* hist,
                                 cudaStream_t st);
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
-                          const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st);
+                          const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl = false);
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
-                        uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st);
+                        uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st, bool pdl = false);
 uint32_t select_small_max();
 cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
-                                StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st);
+                                StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl = false);
 cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const LumaConsts& lc, uint32_t* feat, uint32_t fw,
                             cudaStream_t st);
 int cells_blocks_per_sm();
 cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* cells,
                               uint32_t* err, int grid, cudaStream_t st);
-cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st);
+cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st,
+                                bool pdl = false);
 cudaError_t launch_wait_probe(uint64_t timeout_ns, uint32_t* err, cudaStream_t st);
 cudaError_t launch_lazy_select(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
-                               StreamState* state, cudaStream_t st);
+                               StreamState* state, cudaStream_t st, bool pdl = false);
 cudaError_t launch_debug_bins(const uint8_t* px, uint64_t n_groups, const LumaConsts& lc, int bin_path,
                               uint8_t* bins_out, cudaStream_t st);
 cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max);

@@ -21,6 +21,7 @@ constexpr int kFeatThreads = 512;
 __global__ void __launch_bounds__(kFeatThreads) features_kernel(SegTable segs, FeatArgs fa, LumaConsts L,
                                                                 uint32_t* __restrict__ feat, uint32_t fw) {
   __shared__ uint32_t cell[256];
+  pdl_trigger();
   const uint32_t row = blockIdx.x, tid = threadIdx.x;
   uint32_t seg = 0;
   while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
@@ -86,6 +87,8 @@ __global__ void __launch_bounds__(kFeatThreads) features_kernel(SegTable segs, F
 // for the next push once read.
 __global__ void __launch_bounds__(96) dhash_finish_kernel(uint32_t* __restrict__ cells, FeatArgs fa,
                                                           uint32_t* __restrict__ bits) {
+  pdl_trigger();
+  pdl_wait();  // the cell sums of the streaming kernel before it
   const uint32_t row = blockIdx.x, tid = threadIdx.x;
   uint32_t* c = cells + static_cast<uint64_t>(row) * 72;
   if (tid < 64) {
@@ -135,9 +138,10 @@ __global__ void debug_bins_kernel(const uint8_t* __restrict__ px, uint64_t n_gro
 
 }  // namespace
 
-cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st) {
-  dhash_finish_kernel<<<rows, 96, 0, st>>>(cells, fa, bits);
-  return cudaGetLastError();
+cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st,
+                                bool pdl) {
+  const cudaError_t e = launch_dependent(pdl, dhash_finish_kernel, dim3(rows), dim3(96), 0, st, cells, fa, bits);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const LumaConsts& lc, uint32_t* feat, uint32_t fw,

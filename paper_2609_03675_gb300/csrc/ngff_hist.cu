@@ -221,6 +221,7 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
   const uint32_t n_cnt = kBin == kCells ? a.grid_h * a.grid_w : L.bins * 32;
   uint64_t* bars = reinterpret_cast<uint64_t*>(cnt + (kBin == kCells ? kMaxBins : L.bins * 32));
 
+  pdl_trigger();  // the push's selection kernels may be scheduled; they wait for this grid before reading it
   const uint64_t total = static_cast<uint64_t>(segs.rows) * a.chunks_per_frame;
   const uint64_t c0 = total * blockIdx.x / gridDim.x;
   const uint64_t c1 = total * (blockIdx.x + 1) / gridDim.x;
@@ -348,6 +349,7 @@ constexpr uint32_t kGenericPixels = 16384;
 __global__ void __launch_bounds__(kGenericThreads) hist_generic_kernel(SegTable segs, HistArgs a, LumaConsts L,
                                                                       uint32_t* __restrict__ hist) {
   __shared__ uint32_t cnt[kMaxBins];
+  pdl_trigger();
   const uint32_t row = blockIdx.y;
   uint32_t seg = 0;
   while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;

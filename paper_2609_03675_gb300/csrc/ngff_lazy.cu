@@ -181,6 +181,7 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     sref[b] = t0 > 0 ? sring[B + b] : 0u;
     sprev[b] = t0 > 0 ? sring[b] : 0u;
   }
+  pdl_wait();  // the feature rows of the first-stage kernel before it (state and ring are older)
   stage(0, 0, kLazyThreads);
   __syncthreads();
   adjacent(0);
@@ -277,13 +278,14 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
 }  // namespace
 
 cudaError_t launch_lazy_select(const SegTable& segs, const SelectArgs& a, const uint32_t* feat, uint32_t* ring,
-                               StreamState* state, cudaStream_t st) {
+                               StreamState* state, cudaStream_t st, bool pdl) {
   const size_t smem = 2 * kLazyTileWords * 4 + kLazyMaxRows * (4 + 4 + 1 + 1) + 2 * kMaxBins * 4;
   cudaError_t e = cudaFuncSetAttribute(lazy_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  lazy_select_kernel<<<segs.count, kLazyThreads, smem, st>>>(segs, a, feat, ring, state);
-  return cudaGetLastError();
+  e = launch_dependent(pdl, lazy_select_kernel, dim3(segs.count), dim3(kLazyThreads), smem, st, segs, a, feat, ring,
+                       state);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 uint32_t take_bounds_errors_lazy() { return take_local_bounds_errors(); }

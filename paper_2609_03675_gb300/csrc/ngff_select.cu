@@ -95,6 +95,8 @@ __global__ void __launch_bounds__(kWinWarps * 32) window_kernel(SegTable segs, S
                                                                 const uint32_t* __restrict__ ring,
                                                                 const StreamState* __restrict__ state,
                                                                 uint32_t* __restrict__ l1, uint32_t* __restrict__ mask) {
+  pdl_trigger();
+  pdl_wait();  // the histograms of the first-stage kernel before it
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t row = blockIdx.x * kWinWarps + warp;
   if (row >= segs.rows) return;
@@ -318,6 +320,7 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(SegTable segs, Selec
   __shared__ uint32_t entry[kScanWarps + 1];
   __shared__ unsigned long long s_t0, s_acc;
   __shared__ uint32_t s_g;
+  pdl_wait();  // the distance and mask rows of the window kernel before it
   if (threadIdx.x == 0) {
     sseg = segs.s[blockIdx.x];
     s_t0 = state[sseg.stream].t;
@@ -349,6 +352,7 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
     s_acc = state[sseg.stream].acc;
   }
   __syncthreads();
+  pdl_wait();  // the histograms of the first-stage kernel before it (the stream state is older)
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (uint32_t j = warp; j < sseg.n; j += kScanWarps)
     window_row<kVec4>(sseg.row0 + j, lane, sseg, a, hist, ring, s_t0, l1, mask);
@@ -462,38 +466,38 @@ cudaError_t scan_prepare(uint32_t mask_words, uint32_t l_max) {
 }
 
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
-                          const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
+                          const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl) {
   const uint32_t grid = (segs.rows + kWinWarps - 1) / kWinWarps;
-  if (a.bins % 4 == 0 && a.dist_kind == 0)
-    window_kernel<true><<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
-  else
-    window_kernel<false><<<grid, kWinWarps * 32, 0, st>>>(segs, a, hist, ring, state, l1, mask);
-  return cudaGetLastError();
+  const cudaError_t e =
+      (a.bins % 4 == 0 && a.dist_kind == 0)
+          ? launch_dependent(pdl, window_kernel<true>, dim3(grid), dim3(kWinWarps * 32), 0, st, segs, a, hist, ring,
+                             state, l1, mask)
+          : launch_dependent(pdl, window_kernel<false>, dim3(grid), dim3(kWinWarps * 32), 0, st, segs, a, hist, ring,
+                             state, l1, mask);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
-                        uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st) {
+                        uint32_t* hist, uint32_t* ring, StreamState* state, cudaStream_t st, bool pdl) {
   const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
-  if (a.mask_words == 1)
-    scan_kernel<true><<<segs.count, kScanThreads, smem, st>>>(segs, a, l1, mask, hist, ring, state);
-  else
-    scan_kernel<false><<<segs.count, kScanThreads, smem, st>>>(segs, a, l1, mask, hist, ring, state);
-  return cudaGetLastError();
+  const cudaError_t e =
+      a.mask_words == 1
+          ? launch_dependent(pdl, scan_kernel<true>, dim3(segs.count), dim3(kScanThreads), smem, st, segs, a, l1, mask,
+                             hist, ring, state)
+          : launch_dependent(pdl, scan_kernel<false>, dim3(segs.count), dim3(kScanThreads), smem, st, segs, a, l1,
+                             mask, hist, ring, state);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
-                                StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st) {
+                                StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl) {
   const size_t smem = scan_smem_bytes(a.mask_words, a.l_max);
   const bool vec = a.bins % 4 == 0 && a.dist_kind == 0, one = a.mask_words == 1;
-  if (vec && one)
-    select_small_kernel<true, true><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
-  else if (vec)
-    select_small_kernel<true, false><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
-  else if (one)
-    select_small_kernel<false, true><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
-  else
-    select_small_kernel<false, false><<<segs.count, kScanThreads, smem, st>>>(segs, a, hist, ring, state, l1, mask);
-  return cudaGetLastError();
+  const auto kernel = vec ? (one ? select_small_kernel<true, true> : select_small_kernel<true, false>)
+                          : (one ? select_small_kernel<false, true> : select_small_kernel<false, false>);
+  const cudaError_t e =
+      launch_dependent(pdl, kernel, dim3(segs.count), dim3(kScanThreads), smem, st, segs, a, hist, ring, state, l1, mask);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 uint32_t take_bounds_errors_select() { return take_local_bounds_errors(); }
