@@ -68,6 +68,7 @@ constexpr uint32_t kQerPairQSlots = 3;                // q~ slots: enough to cov
 constexpr uint32_t kQerMaxN = 256;      // text tokens (MMA N) per scoring pass
 constexpr uint32_t kQerMaxText = 4096;  // text tokens per query: up to 16 passes
 constexpr int kRankThreads = 256;  // 8 frames per CTA (a warp each): the O(m^2) ranking spreads over many SMs
+constexpr uint32_t kRankTile = 2048;  // scores staged per pass of the ranking (8 KiB of shared memory)
 
 constexpr uint32_t kQerErrProducer = 16u, kQerErrMma = 32u, kQerErrEpilogue = 64u, kQerErrDrain = 128u;
 
@@ -784,8 +785,10 @@ __global__ void __launch_bounds__(256) qer_mean(const float* __restrict__ colmax
 }
 
 // Eq. 8: flag[f] = 1 when fewer than k frames rank above frame f (higher w,
-// or equal w and lower index). A warp per frame: its lanes split the m scores
-// (coalesced reads of the L2-resident w) and one warp reduction counts them.
+// or equal w and lower index). A warp per frame: the CTA stages the m scores
+// in shared memory, kRankTile at a time (one coalesced pass over the
+// L2-resident w instead of a chain of dependent loads per lane), its lanes
+// split each tile and one warp reduction counts them.
 // The last CTA to finish (a ticket taken after a fence) then writes the flagged frames
 // in time order (ballot, popcount and a scan of the warp totals per pass of
 // kRankThreads frames), the count to k_out, and returns the ticket counter
@@ -798,17 +801,25 @@ __global__ void __launch_bounds__(kRankThreads) qer_rank(const float* __restrict
   constexpr uint32_t kWarps = kRankThreads / 32;
   __shared__ uint32_t wsum[kWarps];
   __shared__ uint32_t s_total, s_last;
+  __shared__ float sw[kRankTile];
   grid_dependency_wait();
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t f = blockIdx.x * kWarps + warp;
-  if (f < n_frames) {  // uniform across the warp
-    const float wf = w[f];
-    uint32_t above = 0;
-#pragma unroll 4
-    for (uint32_t g = lane; g < n_frames; g += 32) {
-      const float wg = __ldg(w + g);
-      above += (wg > wf) | ((wg == wf) & (g < f));
-    }
+  const bool mine = f < n_frames;  // uniform across the warp
+  const float wf = mine ? w[f] : 0.f;
+  uint32_t above = 0;
+  for (uint32_t c0 = 0; c0 < n_frames; c0 += kRankTile) {
+    const uint32_t cn = min(kRankTile, n_frames - c0);
+    for (uint32_t i = tid; i < cn; i += kRankThreads) sw[i] = w[c0 + i];
+    __syncthreads();
+    if (mine)
+      for (uint32_t j = lane; j < cn; j += 32) {
+        const float wg = sw[j];
+        above += (wg > wf) | ((wg == wf) & (c0 + j < f));
+      }
+    __syncthreads();  // the tile is read before the next one overwrites it
+  }
+  if (mine) {
     above = __reduce_add_sync(0xffffffffu, above);
     if (lane == 0) flag[f] = above < k;
   }
