@@ -431,6 +431,26 @@ def _pct(xs, q):
     return float(np.percentile(np.asarray(xs), q))
 
 
+def _graph_seconds(capture, reset, reps=5):
+    """Wall seconds of one launch of a CUDA graph holding a whole sequence of
+    pushes (captured once by `capture`), best of `reps` after one untimed
+    launch; `reset` restarts the streams before each launch, outside the graph."""
+    import torch
+    g = torch.cuda.CUDAGraph()
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g):
+        capture()
+    times = []
+    for _ in range(reps + 1):
+        reset()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        g.replay()
+        torch.cuda.synchronize()
+        times.append(time.perf_counter() - t0)
+    return min(times[1:])
+
+
 def bench_serving(args):
     """32 concurrent 640x360 streams, each call pushing U{1..8} new frames per
     stream in one batched launch sequence: per-call latency (synchronised
@@ -490,9 +510,17 @@ def bench_serving(args):
     el_pipe, _ = run(False)
     el_sync, lat = run(True)
     f.status()
+
+    def reset_all():
+        for s in range(S):
+            f.reset(s)
+
+    el_graph = _graph_seconds(lambda: [f.push_batch_raw(arr, nd) for arr, nd in plan], reset_all)
+    f.status()
     line = {"workload": "serving: 32 streams x 1800 frames of 640x360, U{1..8} frames per stream per batched call",
             "calls": len(plan), "frames": frames_total,
             "pipelined_frames_per_s": frames_total / el_pipe, "pipelined_ms_per_call": el_pipe / len(plan) * 1e3,
+            "graph_frames_per_s": frames_total / el_graph, "graph_ms_per_call": el_graph / len(plan) * 1e3,
             "sync_frames_per_s": frames_total / el_sync,
             "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99), "latency_ms_max": max(lat),
             "latency": "host wall time of one push_batch call plus a device synchronise",
@@ -534,8 +562,11 @@ def bench_medium(args):
     el_pipe, _ = run(False)
     el_sync, lat = run(True)
     f.status()
+    el_graph = _graph_seconds(lambda: [f.push_raw(0, fp, 8, sp, kp) for fp, sp, kp in ptrs], f.reset)
+    f.status()
     print(json.dumps({"workload": "medium: 600 frames of 448x448 pushed in chunks of 8", "pushes": len(lat),
                       "pipelined_frames_per_s": spec.frames / el_pipe, "sync_frames_per_s": spec.frames / el_sync,
+                      "graph_frames_per_s": spec.frames / el_graph, "graph_ms_per_push": el_graph / len(ptrs) * 1e3,
                       "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99),
                       "latency": "host wall time of one push plus a device synchronise",
                       "kept": int((keep != 0).sum().item())}), flush=True)

@@ -184,6 +184,17 @@ void cofie_ngff_destroy(cofie_ngff_t* h);
  * n == 0 is a no-op. Splitting a stream into pushes of any sizes gives the
  * same results as one push. Errors: COFIE_EINVAL (null handle or frames with
  * n > 0, stream out of range), COFIE_ECUDA.
+ *
+ * CUDA graphs: a push whose frames and outputs are all device memory (or
+ * NULL outputs) may be enqueued on a stream that is capturing into a CUDA
+ * graph; each launch of the graph then decides the next n frames of the
+ * stream, reading the frames and writing the outputs at the addresses given
+ * at capture, exactly as an ordinary push at that point would. Every push
+ * leaves the library's scratch as it found it, so captured and ordinary
+ * pushes may be interleaved on one handle. Host memory while capturing is
+ * COFIE_EINVAL. Frames decided by graph launches are not counted by
+ * cofie_ngff_frames_seen, and kernel timing (cofie_ngff_profile_reset) skips
+ * captured pushes.
  */
 int cofie_ngff_push(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, uint32_t n,
                     float* scores_out, uint8_t* keep_out, void* cuda_stream);
@@ -201,8 +212,8 @@ int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, 
  * concurrent streams). desc[i] is as in cofie_ngff_push for stream
  * desc[i].stream; device memory only; streams distinct within the call;
  * nd <= COFIE_NGFF_MAX_BATCH and the total frame count <= max_frames_per_push.
- * Equivalent to one cofie_ngff_push per descriptor. Errors: COFIE_EINVAL,
- * COFIE_ECUDA.
+ * Equivalent to one cofie_ngff_push per descriptor, and capturable into a
+ * CUDA graph as cofie_ngff_push is. Errors: COFIE_EINVAL, COFIE_ECUDA.
  */
 int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream);
 
@@ -299,7 +310,8 @@ int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream);
 
 /*
  * Number of frames stream `stream` has been pushed since creation or its
- * last reset, as enqueued (host-side count, no synchronisation).
+ * last reset, as enqueued (host-side count, no synchronisation; launches of
+ * a CUDA graph that holds captured pushes are not counted).
  */
 int cofie_ngff_frames_seen(const cofie_ngff_t* h, uint32_t stream, uint64_t* t_out);
 

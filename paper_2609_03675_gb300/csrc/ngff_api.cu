@@ -294,21 +294,29 @@ SelectArgs select_args(const cofie_ngff* h) {
   return sa;
 }
 
+// Zeroes histogram rows [0, rows) (dHash rows are written whole and need it not).
+cudaError_t clear_rows(cofie_ngff* h, uint64_t rows, cudaStream_t st) {
+  if (rows == 0 || h->p.signal == COFIE_SIGNAL_DHASH) return cudaSuccess;
+  return cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(rows) * h->fw * 4, st);
+}
+
 // Runs K1-K3 over the rows described by segs (device frames). Histogram rows
-// must be zero when K1 starts: the fused small-push kernel clears its rows
-// after use (unless keep_hist: the caller copies them out afterwards);
-// otherwise the rows are marked dirty and the next push clears them first.
-int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep_hist = false) {
+// are zero between calls, so that a push enqueues the same work whatever came
+// before it (which is what lets a push be captured into a CUDA graph and
+// replayed): the fused small-push kernel clears its rows after use, and
+// otherwise one memset after the selection does, or, with keep_hist, the
+// caller after copying them out. Rows that an earlier call left nonzero (a
+// prepared shard, a push that failed part way) are cleared first.
+// While `capturing`, nothing here runs until the graph is launched, so the
+// host's record of dirty rows is left as it was and no timing events are taken.
+int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep_hist, bool capturing) {
   if (segs.rows == 0) return COFIE_OK;
-  cudaError_t e = cudaSuccess;
-  if (h->dirty_rows && h->p.signal != COFIE_SIGNAL_DHASH) {  // dHash rows are written whole
-    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->fw * 4, st);
-    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
-    h->dirty_rows = 0;
-  }
-  h->dirty_rows = h->p.max_frames_per_push;  // until the whole sequence is enqueued
+  cudaError_t e = clear_rows(h, h->dirty_rows, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+  if (!capturing) h->dirty_rows = h->p.max_frames_per_push;  // until the clean-up is enqueued
   cudaEvent_t ev0 = nullptr, ev1 = nullptr;
-  if (h->time_kernels && take_pair(h->ev_pool, h->ev_used, &ev0, &ev1)) cudaEventRecord(ev0, st);
+  const bool timed = h->time_kernels && !capturing;
+  if (timed && take_pair(h->ev_pool, h->ev_used, &ev0, &ev1)) cudaEventRecord(ev0, st);
   e = launch_first_stage(h, segs, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
   if (ev1) cudaEventRecord(ev1, st);
@@ -318,11 +326,11 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
   uint32_t longest = 0;
   for (uint32_t i = 0; i < segs.count; ++i) longest = segs.s[i].n > longest ? segs.s[i].n : longest;
   // small pushes clear their rows inside the fused kernel (saving a launch);
-  // large ones leave that to one device-wide memset before the next push
+  // large ones with one device-wide memset after the selection
   const bool fused = longest <= select_small_max();
   sa.zero_hist = (fused && !keep_hist && h->p.l_max > 0) ? 1u : 0u;
   cudaEvent_t es0 = nullptr, es1 = nullptr;
-  if (h->time_kernels && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
+  if (timed && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
   if (h->p.l_max == 0) {  // no forced retention: the rule walked in frame order
     e = launch_lazy_select(segs, sa, h->d_hist, h->d_ring, h->d_state, st, !ev0);
     if (e != cudaSuccess) return h->cuda_fail(e, "lazy selection kernel launch");
@@ -339,13 +347,21 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
     h->n_select += 2;
   }
   if (es1) cudaEventRecord(es1, st);
-  h->dirty_rows = sa.zero_hist ? 0 : segs.rows;
+  if (keep_hist) {  // the caller clears the rows once it has copied them
+    if (!capturing) h->dirty_rows = segs.rows;
+    return COFIE_OK;
+  }
+  if (!sa.zero_hist) {
+    e = clear_rows(h, segs.rows, st);
+    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
+  }
+  if (!capturing) h->dirty_rows = 0;
   return COFIE_OK;
 }
 
 // One piece of a single-stream push: n <= max_frames_per_push device frames.
 int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n, float* scores, MemKind ks,
-              uint8_t* keep, MemKind kk, uint32_t* hist_out, MemKind kh, cudaStream_t st) {
+              uint8_t* keep, MemKind kk, uint32_t* hist_out, MemKind kh, cudaStream_t st, bool capturing) {
   SegTable segs;
   memset(&segs, 0, sizeof segs);
   segs.count = 1;
@@ -357,7 +373,7 @@ int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n
   s.stream = stream;
   s.scores = ks == kDevice ? scores : (ks == kNull ? nullptr : h->d_scores);
   s.keep = kk == kDevice ? keep : (kk == kNull ? nullptr : h->d_keep);
-  int rc = run_segments(h, segs, st, kh != kNull);
+  int rc = run_segments(h, segs, st, kh != kNull, capturing);
   if (rc != COFIE_OK) return rc;
   cudaError_t e = cudaSuccess;
   if (ks == kHostPinned || ks == kHostPageable)
@@ -366,8 +382,21 @@ int run_piece(cofie_ngff* h, uint32_t stream, const uint8_t* dframes, uint32_t n
     e = cudaMemcpyAsync(keep, h->d_keep, n, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess && kh != kNull)
     e = cudaMemcpyAsync(hist_out, h->d_hist, static_cast<size_t>(n) * h->fw * 4, cudaMemcpyDefault, st);
+  if (e == cudaSuccess && kh != kNull) e = clear_rows(h, n, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "output copy");
+  if (kh != kNull && !capturing) h->dirty_rows = 0;
   return COFIE_OK;
+}
+
+// 1 while st is capturing into a CUDA graph, 0 when it is not, -1 when the
+// state cannot be read or the capture has been invalidated.
+int capture_state(cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    return -1;
+  }
+  return cs == cudaStreamCaptureStatusActive ? 1 : (cs == cudaStreamCaptureStatusNone ? 0 : -1);
 }
 
 int ensure_staging(cofie_ngff* h) {
@@ -401,6 +430,12 @@ int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n,
   const MemKind kf = classify(frames, &fdev);
   const MemKind ks = classify(scores), kk = classify(keep), kh = classify(hist_out);
   if (kf == kDevice && fdev != h->device) return h->fail(COFIE_EINVAL, "frames live on another device");
+  const int cap = capture_state(st);
+  if (cap < 0) return h->fail(COFIE_ECUDA, "cannot read the CUDA stream's capture state");
+  const auto dev_or_null = [](MemKind k) { return k == kDevice || k == kNull; };
+  if (cap && !(kf == kDevice && dev_or_null(ks) && dev_or_null(kk) && dev_or_null(kh)))
+    return h->fail(COFIE_EINVAL, "a push captured into a CUDA graph takes device frames and outputs only");
+  h->shard.ready = false;  // a push between shard_prepare and shard_commit reuses the shard's rows
   const uint32_t B = h->fw;
   if (kf == kDevice) {
     const uint32_t step = h->p.max_frames_per_push;
@@ -408,7 +443,7 @@ int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n,
       const uint32_t m = n - off < step ? n - off : step;
       int rc = run_piece(h, stream, frames + off * h->frame_bytes, m, scores ? scores + off : nullptr, ks,
                          keep ? keep + off : nullptr, kk, hist_out ? hist_out + static_cast<size_t>(off) * B : nullptr,
-                         kh, st);
+                         kh, st, cap == 1);
       if (rc != COFIE_OK) return rc;
     }
   } else {
@@ -427,13 +462,13 @@ int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n,
       if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_copied[slot], 0);
       if (e != cudaSuccess) return h->cuda_fail(e, "host frame staging");
       rc = run_piece(h, stream, h->d_stage[slot], m, scores ? scores + off : nullptr, ks, keep ? keep + off : nullptr,
-                     kk, hist_out ? hist_out + static_cast<size_t>(off) * B : nullptr, kh, st);
+                     kk, hist_out ? hist_out + static_cast<size_t>(off) * B : nullptr, kh, st, false);
       if (rc != COFIE_OK) return rc;
       e = cudaEventRecord(h->ev_free[slot], st);
       if (e != cudaSuccess) return h->cuda_fail(e, "staging event");
     }
   }
-  h->seen[stream] += n;
+  if (!cap) h->seen[stream] += n;
   h->err.clear();
   return COFIE_OK;
 }
@@ -697,9 +732,14 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
   }
   if (rows > h->p.max_frames_per_push) return h->fail(COFIE_EINVAL, "batch exceeds max_frames_per_push frames");
   segs.rows = static_cast<uint32_t>(rows);
-  int rc = run_segments(h, segs, static_cast<cudaStream_t>(cuda_stream));
+  const cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const int cap = capture_state(st);
+  if (cap < 0) return h->fail(COFIE_ECUDA, "cannot read the CUDA stream's capture state");
+  h->shard.ready = false;
+  int rc = run_segments(h, segs, st, false, cap == 1);
   if (rc != COFIE_OK) return rc;
-  for (uint32_t i = 0; i < nd; ++i) h->seen[desc[i].stream] += desc[i].n;
+  if (!cap)
+    for (uint32_t i = 0; i < nd; ++i) h->seen[desc[i].stream] += desc[i].n;
   h->err.clear();
   return COFIE_OK;
 }
@@ -823,10 +863,8 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   cudaError_t e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "shard state");
   // the first stage only (histograms or features): the selection runs later
-  if (h->dirty_rows && h->p.signal != COFIE_SIGNAL_DHASH) {
-    e = cudaMemsetAsync(h->d_hist, 0, static_cast<size_t>(h->dirty_rows) * h->fw * 4, st);
-    if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
-  }
+  e = clear_rows(h, h->dirty_rows, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "memset histograms");
   h->dirty_rows = h->p.max_frames_per_push;
   e = launch_first_stage(h, all, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
@@ -892,7 +930,9 @@ int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap
     e = cudaMemcpyAsync(scores_out, h->d_scores, n * sizeof(float), cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess && (kk == kHostPinned || kk == kHostPageable))
     e = cudaMemcpyAsync(keep_out, h->d_keep, n, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = clear_rows(h, static_cast<uint64_t>(n_halo) + n, st);  // rows are zero between calls
   if (e != cudaSuccess) return h->cuda_fail(e, "shard commit");
+  h->dirty_rows = 0;
   h->n_select += 1;
   h->shard.ready = false;
   h->seen[stream] = h->shard.t0 + n;
