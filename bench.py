@@ -714,6 +714,18 @@ def bench_qer(args):
         f.run_async(qd, kd, w, sel_all, k_dev)
     e1.record()
     torch.cuda.synchronize()
+    # the same call captured once into a CUDA graph, its launches back to back
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        f.run_async(qd, kd, w, sel_all, k_dev)
+    for _ in range(3):
+        g.replay()
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0.record()
+    for _ in range(reps):
+        g.replay()
+    g1.record()
+    torch.cuda.synchronize()
     # the scoring kernel alone, bracketed by events on the launching stream
     # (which also serialise it against the kernel before it)
     f.profile_reset(time_kernels=True)
@@ -733,6 +745,7 @@ def bench_qer(args):
                     f"{spec.n_heads}/{spec.n_kv_heads} heads of {spec.head_dim}, rho 0.3",
         "call_us": e0.elapsed_time(e1) / reps * 1e3, "score_kernel_us": k_ms * 1e3,
         "frames_per_s": spec.n_frames / (e0.elapsed_time(e1) / reps / 1e3),
+        "graph_call_us": g0.elapsed_time(g1) / reps * 1e3,
         "tensor": {"achieved": tflops, "peak": tc_peak, "unit": "TFLOP/s", "frac": tflops / tc_peak,
                    "peak_kind": f"{tc_kind} bf16 dense (burst)",
                    "flops_per_launch": pr["flops"] / pr["launches"]},

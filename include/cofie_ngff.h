@@ -471,8 +471,11 @@ uint32_t cofie_qer_kernel_in_use(const cofie_qer_t* h);
  *   w_out    n_frames floats (w_f), device memory, or NULL.
  *   sel_out  room for n_frames uint32 frame indices (S_e, ascending), device memory.
  *   k_out    |S_e|: device memory (asynchronous) or host memory (synchronises).
- * Errors: COFIE_EINVAL, COFIE_ECUDA; device-side waits are reported by
- * cofie_qer_status.
+ * With k_out in device memory the call may be captured into a CUDA graph;
+ * each launch of the graph ranks the q and k then at the captured addresses
+ * (kernel timing skips captured calls; a host k_out while capturing is
+ * COFIE_EINVAL). Errors: COFIE_EINVAL, COFIE_ECUDA; device-side waits are
+ * reported by cofie_qer_status.
  */
 int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t n_frames, float* w_out,
                   uint32_t* sel_out, uint32_t* k_out, void* cuda_stream);

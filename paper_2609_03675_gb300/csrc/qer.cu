@@ -1123,6 +1123,19 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   if (reinterpret_cast<uintptr_t>(k) % 16 != 0) return h->fail(COFIE_EINVAL, "k must be 16-byte aligned");
   const cofie_qer_params& p = h->p;
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  // Captured into a CUDA graph, the call's work is recorded, not run: every
+  // buffer it writes is rewritten by each launch (the ranking kernel returns
+  // its ticket to zero), so the graph can be launched again and again; a host
+  // k_out would need a synchronisation and is refused, and timing is skipped.
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    return h->fail(COFIE_ECUDA, "cannot read the CUDA stream's capture state");
+  }
+  if (cs == cudaStreamCaptureStatusInvalidated) return h->fail(COFIE_ECUDA, "the stream's capture was invalidated");
+  const bool capturing = cs == cudaStreamCaptureStatusActive;
+  if (capturing && !is_device(k_out, h->device))
+    return h->fail(COFIE_EINVAL, "k_out must be device memory while the stream captures a CUDA graph");
   const uint64_t nv = static_cast<uint64_t>(n_frames) * p.tokens_per_frame;
   CUtensorMap map_k, map_q;
   const uint32_t tiles = static_cast<uint32_t>((nv + kQerTile - 1) / kQerTile);
@@ -1150,7 +1163,7 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
   float* w = w_out ? w_out : h->d_w;
   uint32_t* kdev = is_device(k_out, h->device) ? k_out : h->d_k;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
-  if (h->time_on && h->ev_used + 2 <= (1u << 16)) {
+  if (h->time_on && !capturing && h->ev_used + 2 <= (1u << 16)) {
     while (h->ev.size() < h->ev_used + 2) {
       cudaEvent_t x;
       if (cudaEventCreate(&x) != cudaSuccess) break;
@@ -1210,9 +1223,11 @@ int cofie_qer_run(cofie_qer_t* h, const uint16_t* q, const uint16_t* k, uint32_t
     }
   }
   if (e1) cudaEventRecord(e1, st);
-  h->launches += 1;
-  h->flops += 2.0 * n_rows * static_cast<double>(nv) * h->D;
-  h->key_bytes += 2.0 * static_cast<double>(nv) * h->D * h->n_blk;  // each pass reads the keys
+  if (!capturing) {
+    h->launches += 1;
+    h->flops += 2.0 * n_rows * static_cast<double>(nv) * h->D;
+    h->key_bytes += 2.0 * static_cast<double>(nv) * h->D * h->n_blk;  // each pass reads the keys
+  }
   cfg.gridDim = dim3((n_frames + 7) / 8, 1, 1);
   cfg.blockDim = dim3(256, 1, 1);
   cfg.dynamicSmemBytes = 0;

@@ -195,3 +195,36 @@ def test_qer_at_its_limits(kernel):
     long_q = S.QerSpec(n_text=4096, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=5, tokens_per_frame=40,
                        n_evidence=1, seed=52)
     check(long_q, 0.4, kernel=kernel)
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_captured_call_replays_on_new_inputs(kernel):
+    """A QER call captured into a CUDA graph, launched on fresh q and k copied
+    into the captured buffers, gives the ordinary call's results bit for bit
+    (the text spans two 256-token blocks, so the folding passes are captured too)."""
+    from paper_2609_03675_gb300 import QER
+    base = dict(n_text=300, n_heads=8, n_kv_heads=2, head_dim=64, n_frames=40, tokens_per_frame=64)
+    f = QER(base["n_text"], base["n_heads"], base["n_kv_heads"], base["head_dim"], base["n_frames"],
+            base["tokens_per_frame"], 0.25, kernel=kernel)
+    inputs = []
+    for seed in (71, 72, 73):
+        q, k, _ = S.generate(S.QerSpec(**base, seed=seed))
+        inputs.append((torch.from_numpy(q.view(np.int16)).cuda(), torch.from_numpy(k.view(np.int16)).cuda()))
+    qd, kd = torch.empty_like(inputs[0][0]), torch.empty_like(inputs[0][1])
+    w = torch.empty(base["n_frames"], dtype=torch.float32, device="cuda")
+    sel = torch.empty(base["n_frames"], dtype=torch.int32, device="cuda")
+    kdev = torch.zeros(1, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        f.run_async(qd, kd, w, sel, kdev)
+    for q, k in inputs:
+        w_ref, sel_ref = f.run(q, k)
+        qd.copy_(q)
+        kd.copy_(k)
+        g.replay()
+        torch.cuda.synchronize()
+        f.status()
+        assert torch.equal(w, w_ref)
+        assert int(kdev.item()) == sel_ref.numel()
+        assert torch.equal(sel[: sel_ref.numel()], sel_ref)
