@@ -47,7 +47,7 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards",
-                                           "signals"],
+                                           "signals", "pipeline"],
                     default="hd1080",
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
@@ -675,6 +675,84 @@ def bench_gather(args):
                       "frac": gbs / peak, "peak_kind": f"{kind} copy bandwidth (read + write)"}), flush=True)
 
 
+def bench_pipeline(args):
+    """The coarse-to-fine path of one 1080p prefix on the device, per step:
+    NGFF over the 3600 frames (Sec. 3.2), the candidate set S_c, the gather
+    of S_c into the encoder's input buffer, and QER over S_c (Sec. 3.3) on
+    synthetic visual keys standing in for the encoder's output (the encoder
+    and the LLM are not part of this library). Time per phase from CUDA events."""
+    import numpy as np
+    import torch
+
+    import synth
+    from paper_2609_03675_gb300 import NGFF, QER
+    from synth import qer as SQ
+    spec = synth.hd1080()
+    spec = spec.with_(frames=min(spec.frames, max(1, args.frames)))
+    host = torch.empty((spec.frames, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.cuda()
+    del host
+    f = NGFF(spec.width, spec.height, max_frames_per_push=spec.frames)
+    scores = torch.empty(spec.frames, dtype=torch.float32, device="cuda")
+    keep = torch.empty(spec.frames, dtype=torch.uint8, device="cuda")
+    f.push(dev, scores=scores, keep=keep)
+    m = f.candidates(keep).numel()  # the same every step (the stream restarts)
+    f.reset()
+    qs = SQ.QerSpec(n_frames=m)
+    q, k, _ = SQ.generate(qs)
+    qd = torch.from_numpy(q.view(np.int16)).cuda()
+    kd = torch.from_numpy(k.view(np.int16)).cuda()
+    fq = QER(qs.n_text, qs.n_heads, qs.n_kv_heads, qs.head_dim, m, qs.tokens_per_frame, 0.3)
+    idx = torch.empty(spec.frames, dtype=torch.int32, device="cuda")
+    m_dev = torch.empty(1, dtype=torch.int32, device="cuda")
+    out = torch.empty((m, spec.height, spec.width, 3), dtype=torch.uint8, device="cuda")
+    w = torch.empty(m, dtype=torch.float32, device="cuda")
+    sel = torch.empty(m, dtype=torch.int32, device="cuda")
+    k_dev = torch.zeros(1, dtype=torch.int32, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    steps = max(1, min(args.steps, 50))
+    acc = np.zeros(4)
+
+    def step(timed):
+        f.reset()
+        if timed:
+            ev[0].record()
+        f.push(dev, scores=scores, keep=keep)
+        if timed:
+            ev[1].record()
+        f._check(f._lib.cofie_ngff_candidates(f._h, keep.data_ptr(), spec.frames, idx.data_ptr(),
+                                              m_dev.data_ptr(), st))
+        if timed:
+            ev[2].record()
+        f.gather(dev, idx[:m], out=out)
+        if timed:
+            ev[3].record()
+        fq.run_async(qd, kd, w, sel, k_dev)
+        if timed:
+            ev[4].record()
+
+    for _ in range(max(3, args.warmup)):
+        step(False)
+    torch.cuda.synchronize()
+    for _ in range(steps):
+        step(True)
+        torch.cuda.synchronize()
+        acc += [ev[i].elapsed_time(ev[i + 1]) for i in range(4)]
+    f.status()
+    fq.status()
+    assert int(m_dev.item()) == m
+    ms = acc / steps
+    print(json.dumps({
+        "workload": f"pipeline: 1080p prefix of {spec.frames} frames -> NGFF -> S_c -> gather -> QER "
+                    f"({qs.n_text} text tokens, {qs.tokens_per_frame} synthetic keys per frame)",
+        "steps": steps, "ms_per_step": float(ms.sum()), "frames_per_s": spec.frames / (ms.sum() / 1e3),
+        "candidates": m, "qer_selected": int(k_dev.item()),
+        "phase_ms": {"ngff_push": ms[0], "candidates": ms[1], "gather": ms[2], "qer": ms[3]},
+        "timing": "CUDA events between phases on one stream, device synchronised after each step"}), flush=True)
+
+
 def peaks_bf16():
     try:
         with open(os.path.join(REPO, "MEASURED_PEAKS.json")) as fh:
@@ -974,6 +1052,8 @@ def main():
         bench_serving(args)
     elif args.workload == "medium":
         bench_medium(args)
+    elif args.workload == "pipeline":
+        bench_pipeline(args)
     elif args.workload == "rare_event":
         bench_rare_event(args)
     elif args.workload == "gather":
