@@ -218,8 +218,10 @@ double sum_pairs(const std::vector<cudaEvent_t>& pool, size_t used, cudaError_t*
 }
 
 // The first stage over the rows of segs: grayscale histograms (K1), or the
-// spatial signal's per-frame features.
-cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t st) {
+// spatial signal's per-frame features. With pdl the bulk-copy kernels are
+// programmatic dependents of the kernel before them (they wait for it before
+// reading a frame).
+cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool pdl = false) {
   const bool cells = h->p.signal == COFIE_SIGNAL_LOWRES || h->p.signal == COFIE_SIGNAL_DHASH;
   bool fast = cells ? h->cells_grid > 0 : h->size_fast && h->bin_path >= 0;
   for (uint32_t i = 0; i < segs.count && fast; ++i)
@@ -244,14 +246,14 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
     const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
     const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->cells_grid) ? chunks : h->cells_grid);
     const bool dhash = h->p.signal == COFIE_SIGNAL_DHASH;
-    cudaError_t e = launch_cells_fast(segs, ha, h->lc, dhash ? h->d_cells : h->d_hist, h->d_err, grid, st);
+    cudaError_t e = launch_cells_fast(segs, ha, h->lc, dhash ? h->d_cells : h->d_hist, h->d_err, grid, st, pdl);
     if (e == cudaSuccess && dhash) e = launch_dhash_finish(h->d_cells, segs.rows, h->fa, h->d_hist, st, true);
     return e;
   }
   if (fast) {
     const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
     const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid);
-    return launch_hist_fast(segs, ha, h->lc, h->bin_path, h->d_hist, h->d_err, grid, st);
+    return launch_hist_fast(segs, ha, h->lc, h->bin_path, h->d_hist, h->d_err, grid, st, pdl);
   }
   return launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
 }
@@ -317,7 +319,7 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
   cudaEvent_t ev0 = nullptr, ev1 = nullptr;
   const bool timed = h->time_kernels && !capturing;
   if (timed && take_pair(h->ev_pool, h->ev_used, &ev0, &ev1)) cudaEventRecord(ev0, st);
-  e = launch_first_stage(h, segs, st);
+  e = launch_first_stage(h, segs, st, !ev0);
   if (e != cudaSuccess) return h->cuda_fail(e, "histogram kernel launch");
   if (ev1) cudaEventRecord(ev1, st);
   h->n_hist += 1;

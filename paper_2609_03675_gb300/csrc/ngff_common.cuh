@@ -67,14 +67,14 @@ struct StreamState {
   unsigned long long acc;  // scene-change signal: L1 numerator summed over the open gradual run (0: none)
 };
 
-// Programmatic dependent launch inside one push: the first-stage kernel lets
-// the selection kernels that follow it be scheduled early (pdl_trigger), and
-// those wait for it (pdl_wait) before their first read of its output, so
-// their launch and set-up overlap its tail. Only launches whose predecessor
-// in the stream is the library's own kernel of the same push use it (the
-// first-stage kernel itself is an ordinary launch: a caller's kernel writing
-// the frames may precede it). Both instructions are no-ops for a kernel
-// launched without the attribute.
+// Programmatic dependent launch: the first-stage kernel lets the selection
+// kernels that follow it be scheduled early (pdl_trigger), and those wait
+// for it (pdl_wait) before their first read of its output, so their launch
+// and set-up overlap its tail. The small-push selection kernel does the same
+// for the next push's first-stage kernel, whose producer waits before it
+// reads a frame (a caller's kernel writing those frames may be the kernel
+// before it instead: the wait then covers that kernel). Both instructions are
+// no-ops for a kernel launched without the attribute.
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
@@ -202,7 +202,7 @@ int hist_blocks_per_sm(int bin_path, uint32_t bins);
 uint32_t hist_chunk_groups();
 size_t hist_smem_bytes(uint32_t bins);
 cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
-                             uint32_t* hist, uint32_t* err, int grid, cudaStream_t st);
+                             uint32_t* hist, uint32_t* err, int grid, cudaStream_t st, bool pdl = false);
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* hist,
                                 cudaStream_t st);
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
@@ -216,7 +216,7 @@ cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const Luma
                             cudaStream_t st);
 int cells_blocks_per_sm();
 cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* cells,
-                              uint32_t* err, int grid, cudaStream_t st);
+                              uint32_t* err, int grid, cudaStream_t st, bool pdl = false);
 cudaError_t launch_dhash_finish(uint32_t* cells, uint32_t rows, const FeatArgs& fa, uint32_t* bits, cudaStream_t st,
                                 bool pdl = false);
 cudaError_t launch_wait_probe(uint64_t timeout_ns, uint32_t* err, cudaStream_t st);

@@ -249,6 +249,10 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
   if (warp == kCW) {
     // ---------------------------------------------------------- producer --
     if (lane != 0) return;
+    // Launched as a programmatic dependent of the kernel before it, this CTA
+    // has set up while that kernel ran; no frame is read and no row written
+    // until that kernel has completed and its memory is visible.
+    pdl_wait();
     const uint64_t pol = l2_read_policy();
     const uint32_t ring0 = smem_u32(ring);
     ChunkCursor cur;
@@ -415,19 +419,22 @@ int cells_blocks_per_sm() {
 }
 
 cudaError_t launch_cells_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* cells,
-                              uint32_t* err, int grid, cudaStream_t st) {
-  hist_fast_kernel<kCells><<<grid, Shape<kCells>::threads, cells_smem_bytes(), st>>>(segs, a, lc, cells, err);
-  return cudaGetLastError();
+                              uint32_t* err, int grid, cudaStream_t st, bool pdl) {
+  const cudaError_t e = launch_dependent(pdl, hist_fast_kernel<kCells>, dim3(grid), dim3(Shape<kCells>::threads),
+                                         cells_smem_bytes(), st, segs, a, lc, cells, err);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
-                             uint32_t* hist, uint32_t* err, int grid, cudaStream_t st) {
+                             uint32_t* hist, uint32_t* err, int grid, cudaStream_t st, bool pdl) {
   const size_t smem = hist_smem_bytes(lc.bins);
-  if (bin_path == kBinFast)
-    hist_fast_kernel<kBinFast><<<grid, kThreads, smem, st>>>(segs, a, lc, hist, err);
-  else
-    hist_fast_kernel<kBinTwoStep><<<grid, kThreads, smem, st>>>(segs, a, lc, hist, err);
-  return cudaGetLastError();
+  const cudaError_t e =
+      bin_path == kBinFast
+          ? launch_dependent(pdl, hist_fast_kernel<kBinFast>, dim3(grid), dim3(kThreads), smem, st, segs, a, lc, hist,
+                             err)
+          : launch_dependent(pdl, hist_fast_kernel<kBinTwoStep>, dim3(grid), dim3(kThreads), smem, st, segs, a, lc,
+                             hist, err);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* hist,

@@ -125,6 +125,10 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
   const uint32_t B = a.bins, n = sg.n;
   const uint32_t rows_per_tile = kLazyTileWords / B;
   const uint32_t n_tiles = (n + rows_per_tile - 1) / rows_per_tile;
+  // Every read of device memory follows the wait: the first-stage kernel
+  // before this one may itself have been scheduled before the previous
+  // push's selection finished writing the stream's state and ring.
+  pdl_wait();
   const unsigned long long t0 = state[sg.stream].t;
   uint32_t* sring = ring + static_cast<uint64_t>(sg.stream) * 2 * B;
   if (n == 0) return;
@@ -181,7 +185,6 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
     sref[b] = t0 > 0 ? sring[B + b] : 0u;
     sprev[b] = t0 > 0 ? sring[b] : 0u;
   }
-  pdl_wait();  // the feature rows of the first-stage kernel before it (state and ring are older)
   stage(0, 0, kLazyThreads);
   __syncthreads();
   adjacent(0);

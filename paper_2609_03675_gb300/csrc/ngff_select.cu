@@ -345,6 +345,12 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
   __shared__ uint32_t entry[kScanWarps + 1];
   __shared__ unsigned long long s_t0, s_acc;
   __shared__ uint32_t s_g;
+  pdl_trigger();  // the next push's first-stage kernel may be scheduled; it waits for this grid before its work
+  // Every read of device memory follows the wait: the histograms of the
+  // first-stage kernel before this one, and the stream's state, which the
+  // previous push's selection may still have been writing when that kernel
+  // was scheduled.
+  pdl_wait();
   if (threadIdx.x == 0) {
     sseg = segs.s[blockIdx.x];
     s_t0 = state[sseg.stream].t;
@@ -352,7 +358,6 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
     s_acc = state[sseg.stream].acc;
   }
   __syncthreads();
-  pdl_wait();  // the histograms of the first-stage kernel before it (the stream state is older)
   const uint32_t warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (uint32_t j = warp; j < sseg.n; j += kScanWarps)
     window_row<kVec4>(sseg.row0 + j, lane, sseg, a, hist, ring, s_t0, l1, mask);
