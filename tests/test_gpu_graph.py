@@ -6,7 +6,8 @@ the stream. The decisions of a stream replayed that way, chunk by chunk
 from one input buffer, must be the oracle's single-pass result (Sec. 3.2,
 Eqs. 2-5), on every selection path (the fused small push, the windowed
 distances and scan of larger pushes, batches, L_max = 0) and with ordinary
-pushes between the launches."""
+pushes between the launches. Also the launch chaining those pushes rely on:
+frames written by a caller's kernel just before a push."""
 import numpy as np
 import pytest
 import torch
@@ -193,3 +194,33 @@ def test_capture_refuses_host_memory():
     f.status()
     _check(fr, O.Params(spec.width, spec.height, tau=0.05), torch.cat(s_all).cpu().numpy(),
            torch.cat(k_all).cpu().numpy())
+
+
+@pytest.mark.parametrize("chunk", [8, 100])
+def test_frames_written_by_a_kernel_just_before_each_push(chunk):
+    """The first-stage kernel is a programmatic dependent of the kernel before
+    it; when that kernel is the caller's and writes the frames, the push must
+    still read them complete. Each chunk is decoded (an elementwise XOR
+    kernel) into the input buffer immediately before its push, with no other
+    work between."""
+    from paper_2609_03675_gb300 import NGFF
+    T = 400
+    spec, fr = _stream(T, seed=68)
+    p = O.Params(spec.width, spec.height, tau=0.05, l_max=9)
+    f = NGFF(spec.width, spec.height, tau=0.05, l_max=9)
+    dev = torch.from_numpy(fr).cuda()
+    gen = torch.Generator(device="cuda").manual_seed(5)
+    noise = torch.randint(0, 256, dev.shape, dtype=torch.uint8, device="cuda", generator=gen)
+    enc = torch.bitwise_xor(dev, noise)
+    del dev
+    buf = torch.empty_like(enc[:chunk])
+    scores, keep = [], []
+    for i in range(0, T, chunk):
+        n = min(chunk, T - i)
+        torch.bitwise_xor(enc[i:i + n], noise[i:i + n], out=buf[:n])
+        s, k = f.push(buf[:n])
+        scores.append(s)
+        keep.append(k)
+    torch.cuda.synchronize()
+    f.status()
+    _check(fr, p, torch.cat(scores).cpu().numpy(), torch.cat(keep).cpu().numpy())
