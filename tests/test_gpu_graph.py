@@ -224,3 +224,42 @@ def test_frames_written_by_a_kernel_just_before_each_push(chunk):
     torch.cuda.synchronize()
     f.status()
     _check(fr, p, torch.cat(scores).cpu().numpy(), torch.cat(keep).cpu().numpy())
+
+
+@pytest.mark.parametrize("signal", ["lowres", "dhash"])
+@pytest.mark.parametrize("chunk", [8, 100])
+def test_captured_push_spatial_signals(signal, chunk):
+    """The ablation's signals under capture: low-res cell sums (rows cleared
+    after use like histograms) and dHash (cell sums cleared by the hash
+    kernel, hash rows written whole), replayed chunk by chunk."""
+    from oracle import signals_oracle as SO
+    from paper_2609_03675_gb300 import NGFF, _abi
+    from tests.test_gpu_signals import _tau_for
+    kind = SO.LOWRES if signal == "lowres" else SO.DHASH
+    T, W, H = 3 * chunk if chunk > 64 else 12 * chunk, 160, 90
+    spec, fr = _stream(T, w=W, h=H, seed=69)
+    feats = np.stack([SO.features(x, O.Params(W, H), kind) for x in fr])
+    tau = _tau_for(feats, O.Params(W, H), kind, l_max=6)
+    p = O.Params(W, H, tau=tau, l_max=6)
+    so, ko = SO.select(feats, p, kind)
+    assert (ko == O.KEEP_NOVELTY).any() and (ko == O.KEEP_DROP).any()
+    sig = _abi.SIGNAL_LOWRES if signal == "lowres" else _abi.SIGNAL_DHASH
+    f = NGFF(W, H, tau=tau, l_max=6, signal=sig)
+    dev = torch.from_numpy(fr).cuda()
+    buf = torch.empty_like(dev[:chunk])
+    sc = torch.empty(chunk, dtype=torch.float32, device="cuda")
+    kp = torch.empty(chunk, dtype=torch.uint8, device="cuda")
+    torch.cuda.synchronize()
+    g = _capture(lambda: f.push(buf, scores=sc, keep=kp))
+    s_all, k_all = [], []
+    for i in range(0, T, chunk):
+        buf.copy_(dev[i:i + chunk])
+        g.replay()
+        s_all.append(sc.clone())
+        k_all.append(kp.clone())
+    torch.cuda.synchronize()
+    f.status()
+    kg = torch.cat(k_all).cpu().numpy()
+    sg = torch.cat(s_all).cpu().numpy().astype(np.float64)
+    assert np.array_equal(kg, ko)
+    assert np.all(np.abs(sg - so) <= 1e-6 * so)
