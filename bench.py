@@ -60,6 +60,15 @@ def parse():
                     help="NGFF's novelty signal for the hd1080 workload (histogram is the paper's)")
     ap.add_argument("--frames", type=int, default=3600,
                     help="use the first FRAMES frames of the stream (small cases for profiling; default all 3600)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="hd1080 line without the figures of the tiny, medium, serving and rare-event streams")
+    ap.add_argument("--configs-budget", type=float, default=240.0,
+                    help="seconds the other streams' figures may take after the headline (a config that would start "
+                         "past the budget is skipped and says so)")
+    ap.add_argument("--no-parity", action="store_true", help="hd1080 line without the oracle parity block")
+    ap.add_argument("--size", default="1920x1080",
+                    help="frame size WxH of the hd1080 workload's stream (same recipe); a pixel count that is not a "
+                         "multiple of 16 runs the generic histogram kernel")
     return ap.parse_args()
 
 
@@ -99,7 +108,7 @@ def peaks():
 
 
 def k1_source_hash() -> str:
-    """sha256 over K1's sources (the kernel file, its device helpers and the common header)."""
+    """sha256 over K1's sources (the kernel file, its device helpers, and the common header)."""
     h = hashlib.sha256()
     for path in K1_SOURCES:
         h.update(open(path, "rb").read())
@@ -226,6 +235,174 @@ def oracle_parallel_sample(frames_u8_ptr, spec, target_s: float, l_max: int = 30
     return k, run(k), cores
 
 
+SCORE_RTOL = 1e-6  # the fp32 score against the oracle's double-precision distance
+
+
+def parity_block(tau, scores, keep, want_scores, want_keep, hist=None, want_hist=None, idx=None, want_idx=None):
+    """Oracle parity of one run: histograms bit-exact, keep codes identical,
+    the largest relative score error, and the frames whose oracle score lies
+    within the score tolerance of tau_h (the band where the keep decision
+    could legitimately differ; listed even when every decision agrees)."""
+    import numpy as np
+    sg = np.asarray(scores, dtype=np.float64)
+    so = np.asarray(want_scores, dtype=np.float64)
+    rel = np.abs(sg - so) / np.maximum(np.abs(so), 1e-300)
+    rel[(so == 0) & (sg == 0)] = 0.0
+    band = np.flatnonzero(np.abs(so - tau) <= SCORE_RTOL * max(abs(tau), 1e-30))
+    diff = np.flatnonzero(np.asarray(keep) != np.asarray(want_keep))
+    out = {"frames": int(so.size), "keep_equal": bool(diff.size == 0),
+           "keep_mismatch_outside_band": int(np.setdiff1d(diff, band).size),
+           "max_rel_score_err": float(rel.max()) if rel.size else 0.0, "score_rtol": SCORE_RTOL,
+           "band_frames": [int(x) for x in band[:64]], "band_count": int(band.size)}
+    if want_hist is not None:
+        out["hist_equal"] = bool(hist is not None and np.array_equal(np.asarray(hist), np.asarray(want_hist)))
+    if want_idx is not None:
+        out["candidates_equal"] = bool(idx is not None and np.array_equal(np.asarray(idx, dtype=np.uint32),
+                                                                           np.asarray(want_idx, dtype=np.uint32)))
+    return out
+
+
+def _event_runs(ev):
+    runs, t = [], 0
+    while t < ev.size:
+        if ev[t]:
+            u = t
+            while u < ev.size and ev[u]:
+                u += 1
+            runs.append((t, u))
+            t = u
+        else:
+            t += 1
+    return runs
+
+
+def tiny_figures(args):
+    """The tiny stream (64 uint8 RGB frames of 224x224, one whole-stream push):
+    device-resident frames/s from CUDA events over repeated steps, per-push
+    latency (host call + synchronise), end to end from pinned host frames to
+    host outputs through the same C entry point, and oracle parity."""
+    import numpy as np
+    import torch
+
+    import oracle as O
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    spec = synth.tiny()
+    T = spec.frames
+    host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+    synth.generate(spec, out=host.data_ptr())
+    dev = host.cuda()
+    f = NGFF(spec.width, spec.height)
+    scores = torch.empty(T, dtype=torch.float32, device="cuda")
+    keep = torch.empty(T, dtype=torch.uint8, device="cuda")
+
+    def step():
+        f.reset()
+        f.push(dev, scores=scores, keep=keep)
+
+    for _ in range(20):
+        step()
+    torch.cuda.synchronize()
+    reps = 300
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    dev_s = e0.elapsed_time(e1) / 1e3
+    lat = []
+    for _ in range(200):
+        c0 = time.perf_counter()
+        step()
+        torch.cuda.synchronize()
+        lat.append((time.perf_counter() - c0) * 1e3)
+    hs = torch.empty(T, dtype=torch.float32, pin_memory=True)
+    hk = torch.empty(T, dtype=torch.uint8, pin_memory=True)
+    e2e = []
+    for i in range(60):
+        torch.cuda.synchronize()
+        c0 = time.perf_counter()
+        f.reset()
+        f.push(host, scores=hs, keep=hk)
+        torch.cuda.synchronize()
+        if i >= 10:
+            e2e.append(time.perf_counter() - c0)
+    f.reset()
+    s, k, h = f.push(dev, return_hist=True)
+    idx = f.candidates(0)
+    f.status()
+    o = O.load()
+    ho, so, ko = o.run(host.numpy(), O.Params(spec.width, spec.height))
+    par = parity_block(0.30, s.cpu().numpy(), k.cpu().numpy(), so, ko, h.cpu().numpy().view(np.uint32), ho,
+                       idx.cpu().numpy(), o.candidates(ko, 4))
+    assert torch.equal(hk, k.cpu()), "end-to-end keep codes differ from the device-resident run"
+    f.close()
+    e2e_s = statistics.median(e2e)
+    return {"workload": "tiny: 64 uint8 RGB frames of 224x224, one whole-stream push per step, B=32, L_max=30, "
+                        "tau_h=0.30",
+            "frames_per_s": reps * T / dev_s, "ms_per_step": dev_s / reps * 1e3,
+            "pixel_gbs": reps * T * spec.frame_bytes / dev_s / 1e9,
+            "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99),
+            "e2e": {"frames_per_s": T / e2e_s, "ms_per_step": e2e_s * 1e3, "h2d_bytes_per_step": T * spec.frame_bytes,
+                    "d2h_bytes_per_step": T * 5, "statistic": "median of 50 steps"},
+            "kept": int((k != 0).sum().item()), "parity": par,
+            "timing": f"CUDA events over {reps} steps (reset + push); latency: host call + synchronise, 200 steps"}
+
+
+def hd1080_parity(f, dev, host, spec, signal, l_max):
+    """Parity of the benchmark's own configuration (same handle, same frames
+    as the timed steps): GPU histograms, scores, keep codes and the stream's
+    candidate set against the oracle. For the spatial signals, whose oracle
+    is numpy per frame, this is left to the tests."""
+    import numpy as np
+
+    import oracle as O
+    from oracle import scd_oracle as SC
+    if signal in (1, 2):
+        return {"skipped": "the spatial signals' oracle is numpy per frame; their parity is in the GPU tests"}
+    t0 = time.perf_counter()
+    T = spec.frames
+    f.reset()
+    s, k, h = f.push(dev, return_hist=True)
+    idx = f.candidates(0)
+    f.status()
+    o = O.load()
+    p = O.Params(spec.width, spec.height, l_max=l_max)
+    cores = max(1, len(os.sched_getaffinity(0)))
+    hist_o = o.histograms_parallel(host.data_ptr(), T, p, nthreads=cores)
+    so, ko = SC.select(hist_o, p, 0.30, 0.10) if signal == 3 else o.select(hist_o, p)
+    out = parity_block(0.30, s.cpu().numpy(), k.cpu().numpy(), so, ko, h.cpu().numpy().view(np.uint32), hist_o,
+                       idx.cpu().numpy(), o.candidates(ko, 4))
+    out["oracle"] = (f"C oracle histograms on {cores} host threads (frames in parallel), then its selection "
+                     "rule and candidate set, single-threaded")
+    out["seconds"] = time.perf_counter() - t0
+    return out
+
+
+def other_configs(args):
+    """Figures of the benchmark's other streams, each at its full size, in one
+    run after the headline: tiny (64 x 224x224), medium (600 x 448x448 in
+    pushes of 8), rare-event (3600 x 1280x720) and serving (32 x 1800 x
+    640x360). A config that would start after args.configs_budget seconds is
+    skipped and says so."""
+    import torch
+    t_start = time.perf_counter()
+    out = {}
+    for name, fn in (("tiny", tiny_figures), ("medium", medium_figures), ("rare_event", rare_event_figures),
+                     ("serving", serving_figures)):
+        el = time.perf_counter() - t_start
+        if el > args.configs_budget:
+            out[name] = {"skipped": f"the {args.configs_budget:.0f} s budget was spent ({el:.0f} s)"}
+            continue
+        t0 = time.perf_counter()
+        out[name] = fn(args)
+        out[name]["seconds"] = time.perf_counter() - t0
+        torch.cuda.empty_cache()
+    out["seconds"] = time.perf_counter() - t_start
+    return out
+
+
 def bench_gb300(args):
     import numpy as np  # noqa: F401
     import torch
@@ -239,7 +416,8 @@ def bench_gb300(args):
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     spec = synth.hd1080(seed=stream_seed(rank))
-    spec = spec.with_(frames=min(spec.frames, max(1, args.frames)))
+    sw, sh = (int(x) for x in args.size.lower().split("x"))
+    spec = spec.with_(frames=min(spec.frames, max(1, args.frames)), width=sw, height=sh)
     T = spec.frames
     # inputs: generated on the host (pinned, kept for the end-to-end leg), resident in HBM for the timed region
     host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
@@ -291,7 +469,7 @@ def bench_gb300(args):
     k1_ms = prof["hist_ms"] / max(prof["hist_timed"], 1)
     k1_bytes = prof["hist_bytes"] / max(prof["hist_launches"], 1)
     achieved = k1_bytes / (k1_ms / 1e3) / 1e9
-    traffic = k1_traffic_per_launch() if signal == 0 else None
+    traffic = k1_traffic_per_launch() if signal == 0 and (spec.width, spec.height) == (1920, 1080) else None
 
     # end to end through the same C entry point with host buffers: H2D of the
     # step's frames and D2H of its scores and keep codes inside the timed region
@@ -342,6 +520,12 @@ def bench_gb300(args):
                "h2d_achieved_gbs": T * spec.frame_bytes / el / 1e9}
         fe.close()
 
+    # oracle parity of the timed configuration: one more step with the
+    # histograms out, against the oracle's histograms (its routine on all host
+    # cores) and its selection on them
+    parity = None
+    if rank == 0 and not args.no_parity:
+        parity = hd1080_parity(f, dev, host, spec, signal, args.l_max)
     cpu = None
     if rank == 0 and world == 1 and args.cpu_seconds > 0:
         k, dt = oracle_sample(host.data_ptr(), spec, args.cpu_seconds, signal, args.l_max)
@@ -358,13 +542,21 @@ def bench_gb300(args):
                                 "sample": f"first {kp} frames, the oracle's histogram routine on {cores} threads "
                                           "(frames in parallel), then its selection"}
 
+    # the other streams of the benchmark, after everything above (rank 0 at N=1)
+    configs = None
+    if rank == 0 and world == 1 and not args.no_configs:
+        f.close()
+        del dev, host
+        torch.cuda.empty_cache()
+        configs = other_configs(args)
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u8", "data": "synthetic",
-            "config": {"workload": f"1080p stream: {T} uint8 RGB frames of 1920x1080 (HWC), one whole-stream push "
-                                   f"per step, B=32, L_max={args.l_max}, tau_h=0.30"
+            "config": {"workload": f"1080p stream: {T} uint8 RGB frames of {spec.width}x{spec.height} (HWC), one "
+                                   f"whole-stream push per step, B=32, L_max={args.l_max}, tau_h=0.30"
                                    + ("" if signal == 0 else f", signal {args.signal} in place of the histogram"),
                        "signal": args.signal, "frames_per_step": T, "width": spec.width, "height": spec.height,
                        "bins": 32, "l_max": args.l_max,
@@ -374,7 +566,9 @@ def bench_gb300(args):
             "frac_of_nominal_8tbs": pixel_gbs / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                          "peak_kind": f"{peak_kind} copy bandwidth", "traffic": traffic,
-                         "kernel": "ngff histogram (K1)" if signal == 0 else f"ngff {args.signal} cell sums (K1 cells)",
+                         "kernel": ("ngff histogram (K1)" if (spec.width * spec.height) % 16 == 0
+                                    else "ngff histogram, generic kernel (pixel count not a multiple of 16)")
+                         if signal == 0 else f"ngff {args.signal} cell sums (K1 cells)",
                          "launch_ms": k1_ms, "bytes_per_launch": k1_bytes,
                          "select_ms_per_step": prof["select_ms"] / max(prof["select_timed"], 1)},
             "e2e": e2e,
@@ -382,6 +576,8 @@ def bench_gb300(args):
             "gpu_launches": int(prof["hist_launches"] + prof["select_launches"]),
             "clocks": clocks,
             "kept_frames_last_step": kept,
+            "parity": parity,
+            "configs": configs,
         }
         print(json.dumps(line), flush=True)
     f.close()
@@ -390,39 +586,50 @@ def bench_gb300(args):
 
 
 def bench_reference(args):
-    """The oracle (single-threaded C, host cores) on the same workload and metric."""
+    """The oracle (single-threaded C, host cores) on the same workload and
+    metric: the timed steps cover the 3600-frame 1080p stream in consecutive
+    slices of about T / K frames (at most 200 per step, so K >= 18 covers the
+    whole stream), each
+    slice a stream the oracle filters from its first frame; the warm-up steps
+    run an 8-frame sample."""
     rank, world, _ = dist_env()
     if rank != 0:
         return
-    import numpy as np
-
     import oracle as O
     import synth
     spec = synth.hd1080()
     o = O.load()
     p = O.Params(spec.width, spec.height)
-    # each step: a bounded sample of frames so that the whole run stays within about two minutes
-    t_frame = 0.012
-    per_step = int(max(2, min(64, 120.0 / max(args.steps + args.warmup, 1) / t_frame)))
-    frames = synth.generate(spec, 0, per_step)
+    T = spec.frames
+    steps = max(1, args.steps)
+    per_step = min(200, -(-T // steps))
+    import numpy as np
+    buf = np.empty((per_step, spec.height, spec.width, 3), dtype=np.uint8)
+    warm = synth.generate(spec, 0, 8)
     for _ in range(args.warmup):
-        o.run(frames, p)
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        o.run(frames, p)
-    el = time.perf_counter() - t0
-    value = args.steps * per_step / el
-    sample = f"first {per_step} frames of the 1080p stream per step, single-threaded C oracle"
+        o.run(warm, p)
+    el, done = 0.0, 0
+    for i in range(steps):
+        a = (i * per_step) % T
+        b = min(a + per_step, T)
+        synth.generate(spec, a, b, out=buf)
+        t0 = time.perf_counter()
+        o.run(buf[: b - a], p)
+        el += time.perf_counter() - t0
+        done += b - a
+    value = done / el
+    sample = (f"{steps} consecutive slices of up to {per_step} frames of the 1080p stream ({done} frames"
+              f"{', the whole stream' if done >= T else ''}), single-threaded C oracle (histograms + selection)")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": el / steps * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "u8", "data": "synthetic",
         "config": {"workload": "1080p stream: 3600 uint8 RGB frames of 1920x1080 (HWC), B=32, L_max=30, tau_h=0.30",
-                   "frames_per_step": per_step, "width": spec.width, "height": spec.height},
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+                   "frames_per_step": per_step, "frames_timed": done, "width": spec.width, "height": spec.height},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample,
+                         "wall_s": el},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
-    del np
     print(json.dumps(line), flush=True)
 
 
@@ -452,21 +659,33 @@ def _graph_seconds(capture, reset, reps=5):
 
 
 def bench_serving(args):
+    print(json.dumps(serving_figures(args)), flush=True)
+
+
+def serving_figures(args, parity: bool = True):
     """32 concurrent 640x360 streams, each call pushing U{1..8} new frames per
     stream in one batched launch sequence: per-call latency (synchronised
-    calls) and pipelined aggregate frames/s."""
+    calls) and pipelined aggregate frames/s; the pipelined run's keep codes
+    and scores against the oracle (its histogram routine on all host cores)."""
+    import numpy as np
     import torch
 
+    import oracle as O
     import synth
     from paper_2609_03675_gb300 import NGFF
     S = synth.SERVING_STREAMS
     specs = [synth.serving_stream(s) for s in range(S)]
     T, W, H = specs[0].frames, specs[0].width, specs[0].height
     host = torch.empty((T, H, W, 3), dtype=torch.uint8, pin_memory=True)
-    dev = []
+    dev, want = [], []
+    o = O.load()
+    p = O.Params(W, H)
     for sp in specs:
         synth.generate(sp, out=host.data_ptr())
         dev.append(host.cuda())
+        if parity:
+            want.append(o.select(o.histograms_parallel(host.data_ptr(), T, p), p))
+    del host
     sizes = [synth.push_sizes(synth.SEED_BASE + 4, s, T) for s in range(S)]
     scores = torch.empty((S, T), dtype=torch.float32, device="cuda")
     keep = torch.empty((S, T), dtype=torch.uint8, device="cuda")
@@ -508,6 +727,16 @@ def bench_serving(args):
     for _ in range(max(1, args.warmup // 3)):
         run(False)
     el_pipe, _ = run(False)
+    f.status()
+    par = None
+    if parity:
+        sc, kc = scores.cpu().numpy(), keep.cpu().numpy()
+        par = parity_block(0.30, sc.reshape(-1), kc.reshape(-1), np.concatenate([w[0] for w in want]),
+                           np.concatenate([w[1] for w in want]))
+        par["candidates_equal"] = all(
+            np.array_equal(f.candidates(s).cpu().numpy().astype(np.uint32), o.candidates(want[s][1], 4))
+            for s in range(S))
+        par["streams"] = S
     el_sync, lat = run(True)
     f.status()
 
@@ -517,25 +746,35 @@ def bench_serving(args):
 
     el_graph = _graph_seconds(lambda: [f.push_batch_raw(arr, nd) for arr, nd in plan], reset_all)
     f.status()
-    line = {"workload": "serving: 32 streams x 1800 frames of 640x360, U{1..8} frames per stream per batched call",
+    line = {"workload": "serving: 32 streams x 1800 uint8 RGB frames of 640x360, U{1..8} frames per stream per "
+                        "batched call, B=32, L_max=30, tau_h=0.30",
             "calls": len(plan), "frames": frames_total,
             "pipelined_frames_per_s": frames_total / el_pipe, "pipelined_ms_per_call": el_pipe / len(plan) * 1e3,
             "graph_frames_per_s": frames_total / el_graph, "graph_ms_per_call": el_graph / len(plan) * 1e3,
             "sync_frames_per_s": frames_total / el_sync,
             "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99), "latency_ms_max": max(lat),
             "latency": "host wall time of one push_batch call plus a device synchronise",
-            "keep_ratio": float((keep != 0).float().mean().item())}
-    print(json.dumps(line), flush=True)
+            "keep_ratio": float((keep != 0).float().mean().item()), "parity": par}
+    f.close()
+    return line
 
 
 def bench_medium(args):
-    """600 frames of 448x448 pushed 8 at a time: per-push latency and frames/s."""
+    print(json.dumps(medium_figures(args)), flush=True)
+
+
+def medium_figures(args):
+    """600 frames of 448x448 pushed 8 at a time: per-push latency and frames/s,
+    and the keep codes and scores of the pipelined run against the oracle."""
+    import numpy as np
     import torch
 
+    import oracle as O
     import synth
     from paper_2609_03675_gb300 import NGFF
     spec = synth.medium()
-    dev = torch.from_numpy(synth.generate(spec)).cuda()
+    frames_np = synth.generate(spec)
+    dev = torch.from_numpy(frames_np).cuda()
     scores = torch.empty(spec.frames, dtype=torch.float32, device="cuda")
     keep = torch.empty(spec.frames, dtype=torch.uint8, device="cuda")
     f = NGFF(spec.width, spec.height)
@@ -560,6 +799,12 @@ def bench_medium(args):
     for _ in range(max(1, args.warmup)):
         run(False)
     el_pipe, _ = run(False)
+    f.status()
+    o = O.load()
+    _, so, ko = o.run(frames_np, O.Params(spec.width, spec.height))
+    idx = f.candidates(0)
+    par = parity_block(0.30, scores.cpu().numpy(), keep.cpu().numpy(), so, ko, idx=idx.cpu().numpy(),
+                       want_idx=o.candidates(ko, 4))
     el_sync, lat = run(True)
     f.status()
     el_graph = _graph_seconds(lambda: [f.push_raw(0, fp, 8, sp, kp) for fp, sp, kp in ptrs], f.reset)
@@ -583,29 +828,45 @@ def bench_medium(args):
         torch.cuda.synchronize()
         glat.append((time.perf_counter() - c0) * 1e3)
     f.status()
-    print(json.dumps({"workload": "medium: 600 frames of 448x448 pushed in chunks of 8", "pushes": len(lat),
-                      "pipelined_frames_per_s": spec.frames / el_pipe, "sync_frames_per_s": spec.frames / el_sync,
-                      "graph_frames_per_s": spec.frames / el_graph, "graph_ms_per_push": el_graph / len(ptrs) * 1e3,
-                      "graph_latency_ms_p50": _pct(glat, 50), "graph_latency_ms_p99": _pct(glat, 99),
-                      "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99),
-                      "latency": "host wall time of one push plus a device synchronise",
-                      "kept": int((keep != 0).sum().item())}), flush=True)
+    prof = f.profile_read()
+    f.close()
+    return {"workload": "medium: 600 uint8 RGB frames of 448x448 pushed in chunks of 8, B=32, L_max=30, tau_h=0.30",
+            "pushes": len(lat), "pipelined_frames_per_s": spec.frames / el_pipe,
+            "sync_frames_per_s": spec.frames / el_sync,
+            "graph_frames_per_s": spec.frames / el_graph, "graph_ms_per_push": el_graph / len(ptrs) * 1e3,
+            "graph_latency_ms_p50": _pct(glat, 50), "graph_latency_ms_p99": _pct(glat, 99),
+            "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99),
+            "latency": "host wall time of one push plus a device synchronise",
+            "kernels_per_push": (prof["hist_launches"] + prof["select_launches"]) / max(1, prof["hist_launches"]),
+            "kept": int((keep != 0).sum().item()), "parity": par}
 
 
 def bench_rare_event(args):
+    print(json.dumps(rare_event_figures(args)), flush=True)
+
+
+def rare_event_figures(args):
     """3600 frames of 1280x720 with 40 injected events: frames/s, keep ratio
-    and event-frame recall across tau_h."""
+    and event-frame recall across tau_h; every tau's keep codes and scores
+    against the oracle (one histogram pass on all host cores, its selection
+    per tau)."""
+    import numpy as np
     import torch
 
+    import oracle as O
     import synth
     from paper_2609_03675_gb300 import NGFF
     spec = synth.rare_event()
     host = torch.empty((spec.frames, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
     synth.generate(spec, out=host.data_ptr())
     dev = host.cuda()
+    o = O.load()
+    hist_o = o.histograms_parallel(host.data_ptr(), spec.frames, O.Params(spec.width, spec.height))
+    del host
     events = torch.from_numpy(synth.event_mask(spec).astype(bool)).cuda()
     starts = synth.event_mask(spec)
-    out = {"workload": "rare-event: 3600 frames of 1280x720, 40 events of 1-3 frames", "taus": {}}
+    out = {"workload": "rare-event: 3600 uint8 RGB frames of 1280x720, 40 events of 1-3 frames, one whole-stream "
+                       "push per step, B=32, L_max=30", "taus": {}}
     for tau in (0.30, 0.15, 0.10, 0.05, 0.02):
         f = NGFF(spec.width, spec.height, tau=tau)
         scores = torch.empty(spec.frames, dtype=torch.float32, device="cuda")
@@ -626,25 +887,24 @@ def bench_rare_event(args):
         f.status()
         kept = keep != 0
         # per-event recall: an event counts as caught if any of its frames is kept
-        ev = starts.astype(bool)
-        runs, t = [], 0
-        while t < spec.frames:
-            if ev[t]:
-                u = t
-                while u < spec.frames and ev[u]:
-                    u += 1
-                runs.append((t, u))
-                t = u
-            else:
-                t += 1
+        runs = _event_runs(starts.astype(bool))
         kc = kept.cpu().numpy()
         caught = sum(1 for a, b in runs if kc[a:b].any())
+        so, ko = o.select(hist_o, O.Params(spec.width, spec.height, tau=tau))
+        par = parity_block(tau, scores.cpu().numpy(), keep.cpu().numpy(), so, ko)
         out["taus"][str(tau)] = {"frames_per_s": 20 * spec.frames / (e0.elapsed_time(e1) / 1e3),
                                  "keep_ratio": float(kept.float().mean().item()),
                                  "event_frame_recall": float(kept[events].float().mean().item()),
-                                 "event_recall": caught / max(1, len(runs))}
+                                 "event_recall": caught / max(1, len(runs)),
+                                 "parity": {"keep_equal": par["keep_equal"],
+                                            "max_rel_score_err": par["max_rel_score_err"],
+                                            "band_frames": par["band_frames"]}}
         f.close()
-    print(json.dumps(out), flush=True)
+    t30 = out["taus"]["0.3"]
+    out["frames_per_s"] = t30["frames_per_s"]
+    out["pixel_gbs"] = t30["frames_per_s"] * spec.frame_bytes / 1e9
+    out["events"] = len(_event_runs(starts.astype(bool)))
+    return out
 
 
 def bench_gather(args):
@@ -662,8 +922,8 @@ def bench_gather(args):
     dev = host.cuda()
     del host
     f = NGFF(spec.width, spec.height, max_frames_per_push=spec.frames)
-    _, keep = f.push(dev)
-    idx = f.candidates(keep)
+    f.push(dev)
+    idx = f.candidates(0)
     m = idx.numel()
     out = torch.empty((m, spec.height, spec.width, 3), dtype=torch.uint8, device="cuda")
     m_dev = torch.empty(1, dtype=torch.int32, device="cuda")
@@ -677,8 +937,7 @@ def bench_gather(args):
     e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
     e0.record()
     for _ in range(reps):
-        f._check(f._lib.cofie_ngff_candidates(f._h, keep.data_ptr(), spec.frames, idx_buf.data_ptr(),
-                                              m_dev.data_ptr(), st))
+        f.candidates_raw(0, idx_buf.data_ptr(), spec.frames, m_dev.data_ptr(), st)
     e1.record()
     for _ in range(reps):
         f.gather(dev, idx, out=out)
@@ -717,7 +976,7 @@ def bench_pipeline(args):
     scores = torch.empty(spec.frames, dtype=torch.float32, device="cuda")
     keep = torch.empty(spec.frames, dtype=torch.uint8, device="cuda")
     f.push(dev, scores=scores, keep=keep)
-    m = f.candidates(keep).numel()  # the same every step (the stream restarts)
+    m = f.candidates(0).numel()  # the same every step (the stream restarts)
     f.reset()
     qs = SQ.QerSpec(n_frames=m)
     q, k, _ = SQ.generate(qs)
@@ -742,8 +1001,7 @@ def bench_pipeline(args):
         f.push(dev, scores=scores, keep=keep)
         if timed:
             ev[1].record()
-        f._check(f._lib.cofie_ngff_candidates(f._h, keep.data_ptr(), spec.frames, idx.data_ptr(),
-                                              m_dev.data_ptr(), st))
+        f.candidates_raw(0, idx.data_ptr(), spec.frames, m_dev.data_ptr(), st)
         if timed:
             ev[2].record()
         f.gather(dev, idx[:m], out=out)
@@ -877,9 +1135,7 @@ def bench_shards_ranks(args):
 
     def step():
         f.reset()
-        m = f.shard_prepare(dev, n_halo=halo, t0=a)
-        maps = shards.exchange_maps(m, world)
-        return f.shard_commit(shards.entry_gaps([x.tolist() for x in maps])[rank], b - a)
+        return shards.sharded_push(f, dev, T, rank, world)
 
     for _ in range(max(3, args.warmup)):
         step()

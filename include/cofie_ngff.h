@@ -18,7 +18,9 @@
  *      t - r(t) >= L_max.
  * Decisions are causal and final when a push completes; the closing
  * safeguards of Sec. 3.2 that need the end of the prefix (the last frame, the
- * M_min uniform fill) are applied by cofie_ngff_candidates.
+ * M_min uniform fill) are applied by cofie_ngff_candidates, which reads the
+ * stream's retention record (the library notes every retained frame of every
+ * stream on the device as it decides it).
  *
  * Conventions for every entry point:
  *   - All calls are asynchronous on `cuda_stream` (a cudaStream_t passed as
@@ -51,7 +53,7 @@
 extern "C" {
 #endif
 
-#define COFIE_NGFF_ABI_VERSION 3
+#define COFIE_NGFF_ABI_VERSION 4
 
 /* Return codes. */
 #define COFIE_OK 0
@@ -59,7 +61,8 @@ extern "C" {
 #define COFIE_ENOMEM 2   /* a device or pinned-host allocation failed */
 #define COFIE_ECUDA 3    /* a CUDA runtime call failed */
 #define COFIE_ETIMEOUT 4 /* a device-side bounded wait ran out (cofie_ngff_status) */
-#define COFIE_EDEVICE 5  /* a device-side check failed: a gather index outside the frames, or in a build with
+#define COFIE_EDEVICE 5  /* a device-side check failed: a gather index outside the frames, candidates of a
+                            stream that ran past its retention record, or in a build with
                             -DCOFIE_DEBUG_CHECKS=1 an index or layout check (cofie_ngff_status, cofie_qer_status) */
 
 /* Keep codes written to keep_out. Nonzero means retained (a candidate). */
@@ -128,6 +131,11 @@ typedef struct cofie_ngff cofie_ngff_t;
  *   scd_cut, scd_gradual
  *                     the twin-comparison thresholds T_b, T_s of the scene
  *                     change signal (non-NaN); defaults 0.30f and 0.10f.
+ *   max_stream_frames frames per stream that the retention record covers
+ *                     (cofie_ngff_candidates); 0 picks the default, 1048576
+ *                     (9.7 h at 30 frames/s). The record takes
+ *                     ceil(max_stream_frames / 32) * 4 bytes of device memory
+ *                     per stream (128 KiB at the default).
  */
 typedef struct {
   uint32_t width, height;
@@ -144,7 +152,7 @@ typedef struct {
   uint32_t signal;
   float scd_cut;
   float scd_gradual;
-  uint32_t reserved;
+  uint32_t max_stream_frames;
 } cofie_ngff_params;
 
 /* One stream's frames in a batched push (see cofie_ngff_push_batch). */
@@ -218,28 +226,60 @@ int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, 
 int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream);
 
 /*
- * Closes a prefix of T frames (Sec. 3.2, the safeguards that need the end of
- * the prefix) and writes its candidate set S_c as ascending frame indices:
- * every frame with a nonzero keep code, the last frame T-1, and -- when that
- * leaves fewer than M_min frames -- the uniformly spaced frames
+ * Closes stream `stream` at the frames pushed so far (Sec. 3.2, "Gap-aware
+ * frame retention": the safeguards that need the end of the prefix) and
+ * writes its candidate set S_c as ascending frame indices. With T the number
+ * of frames the stream has been pushed when the call runs on cuda_stream
+ * (read on the device, so the call may be captured into a CUDA graph after
+ * the pushes it closes), S_c holds every frame t < T-1 that was retained
+ * (nonzero keep code), the last frame T-1, and -- when that leaves fewer
+ * than M_min frames -- the uniformly spaced frames
  * round(i (T-1) / (M_min - 1)), i = 0..M_min-1, rounded half up.
- *   keep     T keep codes of frames 0..T-1 (the concatenated keep_out of the
- *            stream's pushes), device memory.
+ * The frames come from the stream's retention record: one bit per frame,
+ * set on the device by every push (and shard commit) as it decides the
+ * frame, so the caller needs to keep no keep codes. The stream is not
+ * changed: pushes may continue and a later call closes a longer prefix.
+ *   idx_out  room for `cap` uint32 indices (NULL when cap == 0): device
+ *            memory, or host memory together with a host m_out (the first
+ *            such call allocates a device buffer of max_stream_frames
+ *            indices, kept until cofie_ngff_destroy). Only the first
+ *            min(|S_c|, cap) indices are written.
+ *   m_out    |S_c| (also when it exceeds cap): device memory (asynchronous)
+ *            or host memory (the call then synchronises cuda_stream; not
+ *            while capturing).
+ * T == 0 gives |S_c| = 0. A stream that has been pushed more than
+ * max_stream_frames frames has no complete record: COFIE_EINVAL when the
+ * handle knows it on the host, otherwise m_out = 0 and cofie_ngff_status
+ * reports COFIE_EDEVICE. After cofie_ngff_reset the record starts empty;
+ * cofie_ngff_state_save/load carry it; after cofie_ngff_shard_commit it holds
+ * the committed shard's frames only (close a sharded stream with
+ * cofie_ngff_candidates_from_keep over the shards' keep codes). M_min is the
+ * handle's m_min. Errors: COFIE_EINVAL, COFIE_ENOMEM, COFIE_ECUDA.
+ */
+int cofie_ngff_candidates(cofie_ngff_t* h, uint32_t stream, uint32_t* idx_out, uint32_t cap, uint32_t* m_out,
+                          void* cuda_stream);
+
+/*
+ * The same candidate set S_c for a prefix of T frames given as keep codes
+ * (Sec. 3.2): every frame t < T-1 with a nonzero keep code, the last frame
+ * T-1, and the M_min uniform fill as above.
+ *   keep     T keep codes of frames 0..T-1 (for example the concatenated
+ *            keep_out of a stream's pushes, or of a sharded stream's
+ *            shards), device memory.
  *   idx_out  room for T uint32 indices, device memory.
  *   m_out    |S_c|, device memory (asynchronous) or host memory (the call then
  *            synchronises cuda_stream).
- * M_min is the handle's m_min. T == 0 gives |S_c| = 0. Errors: COFIE_EINVAL,
- * COFIE_ECUDA.
+ * T == 0 gives |S_c| = 0. Errors: COFIE_EINVAL, COFIE_ECUDA.
  */
-int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out, uint32_t* m_out,
-                          void* cuda_stream);
+int cofie_ngff_candidates_from_keep(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out,
+                                    uint32_t* m_out, void* cuda_stream);
 
 /*
  * Copies the m frames idx[0..m) of `frames` back to back into `out`: the
  * frames S_c that go on to the vision encoder (Sec. 3.2, "only these m frames
  * are sent to the encoder").
  *   frames   n_frames frames of 3 W H bytes, device memory.
- *   idx      m frame indices, device memory (for example cofie_ngff_candidates' idx_out).
+ *   idx      m frame indices, device memory (for example the idx_out of cofie_ngff_candidates).
  *   out      m * 3 W H bytes, device memory, not overlapping frames.
  * An index >= n_frames is skipped and reported as COFIE_EDEVICE by
  * cofie_ngff_status. Errors: COFIE_EINVAL, COFIE_ECUDA.
@@ -250,19 +290,23 @@ int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames,
 /*
  * Checkpoint and resume of one stream. The saved state is everything a later
  * push depends on (Sec. 3.2: r(t) enters only through the gap t - r(t), and
- * distances reach back at most L_max frames): a 64-byte header (format tag
- * "NGFS", version 2, width, height, bins, l_max, signal, frames seen t,
- * current gap g, the scene-change signal's open run sum) followed by the ring
- * of the last l_max feature rows (l_max * cofie_ngff_feature_words uint32,
- * slot i holds the frame t' with t' mod l_max == i; for l_max == 0 two rows,
- * the previous frame's and the current reference frame's).
+ * distances reach back at most L_max frames), and the retention record that
+ * cofie_ngff_candidates reads: a 64-byte header (format tag "NGFS", version 3,
+ * width, height, bins, l_max, signal, frames seen t, current gap g, the
+ * scene-change signal's open run sum, the record's word count) followed by
+ * the ring of the last l_max feature rows (l_max * cofie_ngff_feature_words
+ * uint32, slot i holds the frame t' with t' mod l_max == i; for l_max == 0
+ * two rows, the previous frame's and the current reference frame's), then
+ * the record (ceil(max_stream_frames / 32) uint32, bit t of word t / 32 set
+ * when frame t was retained).
  *   cofie_ngff_state_bytes   the size of that buffer.
  *   cofie_ngff_state_save    writes stream `stream`'s state to buf (device or
  *                            host memory; host memory synchronises cuda_stream).
  *   cofie_ngff_state_load    restores a saved state into stream `stream` of a
- *                            handle with the same width, height, bins, l_max and
- *                            signal (COFIE_EINVAL otherwise); pushes that follow behave
- *                            exactly as if the saved stream had continued.
+ *                            handle with the same width, height, bins, l_max,
+ *                            signal and max_stream_frames (COFIE_EINVAL otherwise);
+ *                            pushes and candidate sets that follow behave exactly
+ *                            as if the saved stream had continued.
  */
 size_t cofie_ngff_state_bytes(const cofie_ngff_t* h);
 int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream);
@@ -296,14 +340,17 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
 int cofie_ngff_shard_commit(cofie_ngff_t* h, uint32_t stream, uint32_t entry_gap, float* scores_out, uint8_t* keep_out,
                             void* cuda_stream);
 
-/* Restarts stream `stream` at t = 0 (its next frame is a first frame). */
+/* Restarts stream `stream` at t = 0 (its next frame is a first frame) and
+ * empties its retention record (one small kernel on cuda_stream). */
 int cofie_ngff_reset(cofie_ngff_t* h, uint32_t stream, void* cuda_stream);
 
 /*
  * Synchronises cuda_stream and reports device-side failures of earlier
  * calls on the handle: COFIE_ETIMEOUT if a bounded wait inside a kernel ran
  * out (the affected results are invalid), COFIE_EDEVICE if a gather index
- * was outside its frames, COFIE_ECUDA on a CUDA error, COFIE_OK otherwise.
+ * was outside its frames or a candidate set was asked of a stream that had
+ * run past its retention record, COFIE_ECUDA on a CUDA error, COFIE_OK
+ * otherwise.
  * Clears the device error word.
  */
 int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream);
@@ -370,6 +417,7 @@ typedef struct {
   double hist_ms;           /* summed event-timed histogram-kernel durations, milliseconds */
   uint64_t select_timed;    /* distance + scan launch pairs that were event-timed */
   double select_ms;         /* summed event-timed durations of those pairs, milliseconds */
+  uint64_t other_launches;  /* launches of the stream-reset, candidate and gather kernels */
 } cofie_ngff_profile;
 
 /* Zeroes the counters; time_kernels != 0 turns event timing on, 0 off. */
@@ -388,10 +436,13 @@ int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out);
  *
  * Decides the first n frames of a fresh stream from their integer histograms
  * and writes the same scores and keep codes cofie_ngff_push_ex gives on a new
- * stream. Needs no handle and allocates nothing: its working tables live in a
- * static device array of 1048576 32-bit words (4 MiB) that every GPU loading
- * the library holds until the process exits.
- *   p           width, height, bins, l_max and tau are used (the rest ignored).
+ * stream of the histogram signal (no scene changes). Needs no handle and
+ * allocates nothing: its working tables live in a static device array of
+ * 1048576 32-bit words (4 MiB) that every GPU loading the library holds until
+ * the process exits. One CTA does the work: at the largest n it takes
+ * milliseconds, not microseconds.
+ *   p           width, height, bins, l_max and tau are used; signal must be
+ *               COFIE_SIGNAL_HISTOGRAM (else COFIE_EINVAL); the rest is ignored.
  *   hist        n * bins uint32 counts, row-major, device memory on the
  *               current device (for example hist_out of cofie_ngff_push_ex).
  *   n           frames; n * (l_max + ceil(l_max / 32)) must not exceed

@@ -40,7 +40,8 @@ class NGFF:
     def __init__(self, width: int, height: int, *, bins: int = 32, l_max: int = 30, m_min: int = 4,
                  tau: float = 0.30, luma_weights=(299, 587, 114), luma_den: int = 1000, max_streams: int = 1,
                  max_frames_per_push: int = 4096, device: int | None = None, host_stage_bytes: int = 0,
-                 signal: int = 0, scd_cut: float | None = None, scd_gradual: float | None = None):
+                 signal: int = 0, scd_cut: float | None = None, scd_gradual: float | None = None,
+                 max_stream_frames: int = 0):
         lib = _abi.load()
         p = _abi.Params()
         lib.cofie_ngff_default_params(ctypes.byref(p), width, height)
@@ -57,6 +58,7 @@ class NGFF:
             p.scd_cut = scd_cut
         if scd_gradual is not None:
             p.scd_gradual = scd_gradual
+        p.max_stream_frames = max_stream_frames
         h = ctypes.c_void_p()
         rc = lib.cofie_ngff_create(ctypes.byref(p), ctypes.byref(h))
         if rc != _abi.OK:
@@ -142,15 +144,33 @@ class NGFF:
         """The batched C entry point on a prebuilt descriptor array."""
         self._check(self._lib.cofie_ngff_push_batch(self._h, arr, nd, self._stream(cuda_stream)))
 
-    def candidates(self, keep: torch.Tensor, cuda_stream=None) -> torch.Tensor:
-        """S_c of a closed prefix: ascending indices of the retained frames, the
-        last frame, and the M_min uniform fill (cuda uint8 keep codes in, cuda
-        int32 indices out; synchronises to read the count)."""
+    def candidates(self, stream: int = 0, cap: int | None = None, cuda_stream=None) -> torch.Tensor:
+        """S_c of ``stream`` closed at the frames pushed so far, from the
+        library's retention record: ascending indices (cuda int32) of the
+        retained frames, the last frame and the M_min uniform fill.
+        Synchronises to read the count. ``cap`` defaults to the frames seen."""
+        if cap is None:
+            cap = max(1, self.frames_seen(stream))
+        idx = torch.empty(max(cap, 1), dtype=torch.int32, device=self.device)
+        m = ctypes.c_uint32(0)
+        self._check(self._lib.cofie_ngff_candidates(self._h, stream, _ptr(idx), cap, ctypes.addressof(m),
+                                                    self._stream(cuda_stream)))
+        if m.value > cap:
+            raise ValueError(f"S_c has {m.value} frames, more than cap={cap}")
+        return idx[: m.value]
+
+    def candidates_raw(self, stream: int, idx_ptr: int, cap: int, m_ptr: int, cuda_stream=None):
+        """The per-stream C entry point with plain device addresses (asynchronous)."""
+        self._check(self._lib.cofie_ngff_candidates(self._h, stream, idx_ptr, cap, m_ptr, self._stream(cuda_stream)))
+
+    def candidates_from_keep(self, keep: torch.Tensor, cuda_stream=None) -> torch.Tensor:
+        """S_c of a prefix given by its keep codes (cuda uint8 in, cuda int32
+        indices out; synchronises to read the count)."""
         T = keep.numel()
         idx = torch.empty(max(T, 1), dtype=torch.int32, device=self.device)
         m = ctypes.c_uint32(0)
-        self._check(self._lib.cofie_ngff_candidates(self._h, _ptr(keep), T, _ptr(idx), ctypes.addressof(m),
-                                                    self._stream(cuda_stream)))
+        self._check(self._lib.cofie_ngff_candidates_from_keep(self._h, _ptr(keep), T, _ptr(idx), ctypes.addressof(m),
+                                                              self._stream(cuda_stream)))
         return idx[: m.value]
 
     def gather(self, frames: torch.Tensor, idx: torch.Tensor, out: torch.Tensor | None = None, cuda_stream=None):

@@ -27,6 +27,7 @@ EXPORTS = (
     "cofie_ngff_push_ex",
     "cofie_ngff_push_batch",
     "cofie_ngff_candidates",
+    "cofie_ngff_candidates_from_keep",
     "cofie_ngff_gather",
     "cofie_ngff_reset",
     "cofie_ngff_state_bytes",
@@ -73,7 +74,7 @@ class Params(ctypes.Structure):
         ("signal", ctypes.c_uint32),
         ("scd_cut", ctypes.c_float),
         ("scd_gradual", ctypes.c_float),
-        ("reserved", ctypes.c_uint32),
+        ("max_stream_frames", ctypes.c_uint32),
     ]
 
 
@@ -96,6 +97,7 @@ class Profile(ctypes.Structure):
         ("hist_ms", ctypes.c_double),
         ("select_timed", ctypes.c_uint64),
         ("select_ms", ctypes.c_double),
+        ("other_launches", ctypes.c_uint64),
     ]
 
 
@@ -151,8 +153,10 @@ def load():
     lib.cofie_ngff_push_ex.restype = ctypes.c_int
     lib.cofie_ngff_push_batch.argtypes = [H, ctypes.POINTER(PushDesc), u32, vp]
     lib.cofie_ngff_push_batch.restype = ctypes.c_int
-    lib.cofie_ngff_candidates.argtypes = [H, vp, u32, vp, vp, vp]
+    lib.cofie_ngff_candidates.argtypes = [H, u32, vp, u32, vp, vp]
     lib.cofie_ngff_candidates.restype = ctypes.c_int
+    lib.cofie_ngff_candidates_from_keep.argtypes = [H, vp, u32, vp, vp, vp]
+    lib.cofie_ngff_candidates_from_keep.restype = ctypes.c_int
     lib.cofie_ngff_gather.argtypes = [H, vp, u32, vp, u32, vp, vp]
     lib.cofie_ngff_gather.restype = ctypes.c_int
     lib.cofie_ngff_state_bytes.argtypes = [H]

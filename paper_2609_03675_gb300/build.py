@@ -36,9 +36,9 @@ def _flags(extra=()):
 
 
 def _inputs():
-    files = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, "ngff_common.cuh"),
-                                                        os.path.join(CSRC, "ngff_device.cuh"),
-                                                        os.path.join(INCLUDE, "cofie_ngff.h"), __file__]
+    headers = ["ngff_common.cuh", "ngff_device.cuh"]
+    files = ([os.path.join(CSRC, s) for s in SOURCES + headers]
+             + [os.path.join(INCLUDE, "cofie_ngff.h"), __file__])
     return files
 
 

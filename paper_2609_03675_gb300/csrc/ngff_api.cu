@@ -33,6 +33,7 @@ thread_local std::string g_global_error;
 enum MemKind { kNull = 0, kDevice = 1, kHostPinned = 2, kHostPageable = 3 };
 
 constexpr uint64_t kDefaultStageBytes = 256ull << 20;
+constexpr uint32_t kDefaultRecordFrames = 1u << 20;  // frames per stream the retention record covers
 constexpr uint64_t kTimeoutNs = 2000000000ull;  // bounded device waits: 2 s
 constexpr size_t kMaxTimedEvents = 1u << 16;
 
@@ -74,10 +75,13 @@ struct cofie_ngff {
   uint32_t* d_mask = nullptr;
   uint32_t* d_ring = nullptr;
   StreamState* d_state = nullptr;
+  uint32_t* d_record = nullptr;  // [S][rec_words] retention record (bit t: frame t retained)
+  uint32_t rec_words = 0;
   float* d_scores = nullptr;
   uint8_t* d_keep = nullptr;
   uint32_t* d_err = nullptr;
   uint32_t* d_count = nullptr;  // candidate count when the caller's m_out is host memory
+  uint32_t* d_idx = nullptr;    // candidate indices when the caller's idx_out is host memory (allocated on first use)
   uint64_t dirty_rows = 0;      // histogram rows [0, dirty_rows) may be nonzero
   uint16_t* d_map = nullptr;    // a shard's gap map
   struct {                      // the shard prepared and not yet committed
@@ -95,7 +99,7 @@ struct cofie_ngff {
   std::vector<uint64_t> seen;
   std::string err;
   // launch counters and optional event timing of the histogram kernel
-  uint64_t n_hist = 0, n_select = 0, hist_bytes = 0;
+  uint64_t n_hist = 0, n_select = 0, n_other = 0, hist_bytes = 0;
   bool time_kernels = false;
   std::vector<cudaEvent_t> ev_pool;  // pairs: [2i] start, [2i+1] end
   size_t ev_used = 0;
@@ -217,15 +221,24 @@ double sum_pairs(const std::vector<cudaEvent_t>& pool, size_t used, cudaError_t*
   return ms;
 }
 
+// Whether the first stage over segs runs on the bulk-copy kernel (K1 or its
+// cells mode): frames of a multiple of 16 pixels, 16-byte aligned, and a bin
+// or grid path the host has verified.
+bool first_stage_fast(const cofie_ngff* h, const SegTable& segs) {
+  const bool cells = h->p.signal == COFIE_SIGNAL_LOWRES || h->p.signal == COFIE_SIGNAL_DHASH;
+  bool fast = cells ? h->cells_grid > 0 : h->size_fast && h->bin_path >= 0;
+  for (uint32_t i = 0; i < segs.count && fast; ++i)
+    if (reinterpret_cast<uintptr_t>(segs.s[i].frames) % 16 != 0) fast = false;
+  return fast;
+}
+
 // The first stage over the rows of segs: grayscale histograms (K1), or the
 // spatial signal's per-frame features. With pdl the bulk-copy kernels are
 // programmatic dependents of the kernel before them (they wait for it before
 // reading a frame).
 cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool pdl = false) {
   const bool cells = h->p.signal == COFIE_SIGNAL_LOWRES || h->p.signal == COFIE_SIGNAL_DHASH;
-  bool fast = cells ? h->cells_grid > 0 : h->size_fast && h->bin_path >= 0;
-  for (uint32_t i = 0; i < segs.count && fast; ++i)
-    if (reinterpret_cast<uintptr_t>(segs.s[i].frames) % 16 != 0) fast = false;
+  const bool fast = first_stage_fast(h, segs);
   HistArgs ha{};
   ha.frame_bytes = h->frame_bytes;
   ha.npix = h->npix;
@@ -255,7 +268,7 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
     const int grid = static_cast<int>(chunks < static_cast<uint64_t>(h->hist_grid) ? chunks : h->hist_grid);
     return launch_hist_fast(segs, ha, h->lc, h->bin_path, h->d_hist, h->d_err, grid, st, pdl);
   }
-  return launch_hist_generic(segs, ha, h->lc, h->d_hist, st);
+  return launch_hist_generic(segs, ha, h->lc, h->bin_path, h->d_hist, st);
 }
 
 // The smallest numerator x with fp32(x) / den >= thr, or 2^64 - 1 if none.
@@ -293,6 +306,8 @@ SelectArgs select_args(const cofie_ngff* h) {
   sa.x_tau = h->x_tau;
   sa.x_cut = h->x_cut;
   sa.x_grad = h->x_grad;
+  sa.record = h->d_record;
+  sa.rec_words = h->rec_words;
   return sa;
 }
 
@@ -327,15 +342,20 @@ int run_segments(cofie_ngff* h, const SegTable& segs, cudaStream_t st, bool keep
   SelectArgs sa = select_args(h);
   uint32_t longest = 0;
   for (uint32_t i = 0; i < segs.count; ++i) longest = segs.s[i].n > longest ? segs.s[i].n : longest;
-  // small pushes clear their rows inside the fused kernel (saving a launch);
-  // large ones with one device-wide memset after the selection
+  // small pushes clear their rows inside the selection kernel (saving a
+  // launch); large ones with one device-wide memset after the selection
+  const bool walk = h->p.l_max > 0 && h->p.l_max <= select_walk_max_lmax() && longest <= select_walk_max_frames();
   const bool fused = longest <= select_small_max();
-  sa.zero_hist = (fused && !keep_hist && h->p.l_max > 0) ? 1u : 0u;
+  sa.zero_hist = ((walk || fused) && !keep_hist && h->p.l_max > 0) ? 1u : 0u;
   cudaEvent_t es0 = nullptr, es1 = nullptr;
   if (timed && take_pair(h->ev_sel, h->ev_sel_used, &es0, &es1)) cudaEventRecord(es0, st);
   if (h->p.l_max == 0) {  // no forced retention: the rule walked in frame order
     e = launch_lazy_select(segs, sa, h->d_hist, h->d_ring, h->d_state, st, !ev0);
     if (e != cudaSuccess) return h->cuda_fail(e, "lazy selection kernel launch");
+    h->n_select += 1;
+  } else if (walk) {  // distances and the rule walked in frame order, in one small launch per stream
+    e = launch_select_walk(segs, sa, h->d_hist, h->d_ring, h->d_state, st, !ev0);
+    if (e != cudaSuccess) return h->cuda_fail(e, "selection kernel launch");
     h->n_select += 1;
   } else if (fused) {  // distances and scan in one launch
     e = launch_select_small(segs, sa, h->d_hist, h->d_ring, h->d_state, h->d_l1, h->d_mask, st, !ev0);
@@ -479,8 +499,8 @@ void free_handle(cofie_ngff* h) {
   if (!h) return;
   DeviceGuard guard(h->device);
   cudaDeviceSynchronize();
-  void* bufs[] = {h->d_hist, h->d_l1, h->d_mask, h->d_ring, h->d_state, h->d_scores, h->d_keep,
-                  h->d_err,  h->d_stage[0], h->d_stage[1], h->d_count, h->d_map, h->d_cells};
+  void* bufs[] = {h->d_hist,     h->d_l1,       h->d_mask,  h->d_ring, h->d_state, h->d_scores, h->d_keep,
+                  h->d_err,      h->d_stage[0], h->d_stage[1], h->d_count, h->d_map, h->d_cells, h->d_record, h->d_idx};
   for (void* b : bufs)
     if (b) cudaFree(b);
   for (cudaEvent_t ev : h->ev_pool) cudaEventDestroy(ev);
@@ -519,7 +539,7 @@ void cofie_ngff_default_params(cofie_ngff_params* p, uint32_t width, uint32_t he
   p->signal = COFIE_SIGNAL_HISTOGRAM;
   p->scd_cut = 0.30f;     // twin-comparison thresholds of the scene-change signal
   p->scd_gradual = 0.10f;
-  p->reserved = 0;
+  p->max_stream_frames = kDefaultRecordFrames;
 }
 
 int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
@@ -588,6 +608,9 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   }
   h->size_fast = (h->npix % 16) == 0;
   h->seen.assign(p->max_streams, 0);
+  const uint32_t rec_frames = p->max_stream_frames ? p->max_stream_frames : kDefaultRecordFrames;
+  h->rec_words = (rec_frames + 31) / 32;
+  h->p.max_stream_frames = rec_frames;
 
   LumaConsts& lc = h->lc;
   const uint32_t wr = p->luma_w[0], wg = p->luma_w[1], wb = p->luma_w[2], den = p->luma_den;
@@ -634,6 +657,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   if (e == cudaSuccess) e = dalloc(&h->d_err, 1);
   if (e == cudaSuccess) e = dalloc(&h->d_count, 1);
   if (e == cudaSuccess) e = dalloc(&h->d_map, COFIE_NGFF_MAX_LMAX);
+  if (e == cudaSuccess) e = dalloc(&h->d_record, S * h->rec_words);
   if (e == cudaSuccess && p->signal == COFIE_SIGNAL_DHASH) {
     e = dalloc(&h->d_cells, F * 72);
     if (e == cudaSuccess) e = cudaMemset(h->d_cells, 0, F * 72 * sizeof(uint32_t));
@@ -645,6 +669,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     return COFIE_ENOMEM;
   }
   if (e == cudaSuccess) e = cudaMemset(h->d_state, 0, S * sizeof(StreamState));
+  if (e == cudaSuccess) e = cudaMemset(h->d_record, 0, S * h->rec_words * sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(h->d_hist, 0, F * h->fw * sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaMemset(h->d_err, 0, sizeof(uint32_t));
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
@@ -749,21 +774,22 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
 namespace {
 
 constexpr uint32_t kStateMagic = 0x5346474Eu;  // "NGFS" little-endian
-constexpr uint32_t kStateVersion = 2;
+constexpr uint32_t kStateVersion = 3;
 constexpr size_t kStateHeader = 64;
 
 struct StateHeader {  // the first 64 bytes of a saved state
   uint32_t magic, version, width, height, bins, l_max;
   uint32_t pad0, pad1;
   StreamState st;  // frames seen, current gap, open scene-change run (24 bytes)
-  uint32_t reserved[2];
+  uint32_t rec_words;  // words of the retention record that follows the ring
+  uint32_t reserved;
 };
 static_assert(sizeof(StateHeader) == kStateHeader, "state header layout");
 
 }  // namespace
 
 size_t cofie_ngff_state_bytes(const cofie_ngff_t* h) {
-  return h ? kStateHeader + static_cast<size_t>(ring_rows(h)) * h->fw * sizeof(uint32_t) : 0;
+  return h ? kStateHeader + (static_cast<size_t>(ring_rows(h)) * h->fw + h->rec_words) * sizeof(uint32_t) : 0;
 }
 
 int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cuda_stream) {
@@ -782,6 +808,7 @@ int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cud
   hdr.bins = h->p.bins;
   hdr.l_max = h->p.l_max;
   hdr.pad0 = h->p.signal;
+  hdr.rec_words = h->rec_words;
   uint8_t* b = static_cast<uint8_t*>(buf);
   const size_t ring_bytes = static_cast<size_t>(ring_rows(h)) * h->fw * sizeof(uint32_t);
   const uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * ring_rows(h) * h->fw;
@@ -790,6 +817,8 @@ int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cud
     // the header's fixed part travels through the handle's pinned-free path: a
     // synchronous copy of 32 host bytes, then the device-resident parts
     e = cudaMemcpyAsync(b, &hdr, offsetof(StateHeader, st), cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(b + offsetof(StateHeader, rec_words), &hdr.rec_words, 8, cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   } else {
     memcpy(b, &hdr, kStateHeader);
@@ -798,6 +827,9 @@ int cofie_ngff_state_save(cofie_ngff_t* h, uint32_t stream, void* buf, void* cud
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(b + offsetof(StateHeader, st), h->d_state + stream, sizeof(StreamState), cudaMemcpyDefault, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(b + kStateHeader, ring, ring_bytes, cudaMemcpyDefault, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(b + kStateHeader + ring_bytes, h->d_record + static_cast<size_t>(stream) * h->rec_words,
+                        h->rec_words * sizeof(uint32_t), cudaMemcpyDefault, st);
   if (e == cudaSuccess && kb != kDevice) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return h->cuda_fail(e, "state save");
   return COFIE_OK;
@@ -819,12 +851,17 @@ int cofie_ngff_state_load(cofie_ngff_t* h, uint32_t stream, const void* buf, voi
   if (hdr.width != h->p.width || hdr.height != h->p.height || hdr.bins != h->p.bins || hdr.l_max != h->p.l_max ||
       hdr.pad0 != h->p.signal)
     return h->fail(COFIE_EINVAL, "saved state has another width, height, bins, l_max or signal");
+  if (hdr.rec_words != h->rec_words)
+    return h->fail(COFIE_EINVAL, "saved state has another retention record size (max_stream_frames)");
   if (hdr.st.t > 0 && h->p.l_max > 0 && (hdr.st.g < 1 || hdr.st.g > h->p.l_max))
     return h->fail(COFIE_EINVAL, "saved state has a gap outside [1, l_max]");
   const uint8_t* b = static_cast<const uint8_t*>(buf);
   const size_t ring_bytes = static_cast<size_t>(ring_rows(h)) * h->fw * sizeof(uint32_t);
   uint32_t* ring = h->d_ring + static_cast<size_t>(stream) * ring_rows(h) * h->fw;
   e = cudaMemcpyAsync(ring, b + kStateHeader, ring_bytes, cudaMemcpyDefault, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->d_record + static_cast<size_t>(stream) * h->rec_words, b + kStateHeader + ring_bytes,
+                        h->rec_words * sizeof(uint32_t), cudaMemcpyDefault, st);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(h->d_state + stream, b + offsetof(StateHeader, st), sizeof(StreamState), cudaMemcpyDefault, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // buf may be released when this returns
@@ -863,6 +900,10 @@ int cofie_ngff_shard_prepare(cofie_ngff_t* h, uint32_t stream, const uint8_t* fr
   all.s[0].stream = stream;
   StreamState ss{t0, 1u, 0u, 0ull};
   cudaError_t e = cudaMemcpyAsync(h->d_state + stream, &ss, sizeof ss, cudaMemcpyHostToDevice, st);
+  // the record of a sharded stream holds the committed shard's frames only
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(h->d_record + static_cast<size_t>(stream) * h->rec_words, 0, h->rec_words * sizeof(uint32_t),
+                        st);
   if (e != cudaSuccess) return h->cuda_fail(e, "shard state");
   // the first stage only (histograms or features): the selection runs later
   e = clear_rows(h, h->dirty_rows, st);
@@ -945,9 +986,10 @@ int cofie_ngff_reset(cofie_ngff_t* h, uint32_t stream, void* cuda_stream) {
   if (!h) return COFIE_EINVAL;
   if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
   DeviceGuard guard(h->device);
-  cudaError_t e =
-      cudaMemsetAsync(h->d_state + stream, 0, sizeof(StreamState), static_cast<cudaStream_t>(cuda_stream));
+  const cudaError_t e = launch_stream_reset(h->d_state + stream, h->d_record + static_cast<size_t>(stream) * h->rec_words,
+                                            h->rec_words, static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return h->cuda_fail(e, "reset");
+  h->n_other += 1;
   h->seen[stream] = 0;
   return COFIE_OK;
 }
@@ -970,7 +1012,7 @@ int cofie_ngff_status(cofie_ngff_t* h, void* cuda_stream) {
     char buf[128];
     snprintf(buf, sizeof buf,
              "device-side failure (error bits 0x%x: 1/2/4 a wait ran out, 8 a bad gather index, 16 an index check "
-             "of the checked build)",
+             "of the checked build, 32 candidates of a stream past its retention record)",
              word);
     return h->fail((word & (kErrConsumerTimeout | kErrProducerTimeout | kErrDrainTimeout)) ? COFIE_ETIMEOUT
                                                                                           : COFIE_EDEVICE,
@@ -1012,9 +1054,58 @@ int cofie_ngff_debug_bins(cofie_ngff_t* h, const uint8_t* pixels, uint64_t n_pix
   return COFIE_OK;
 }
 
-int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out, uint32_t* m_out,
+int cofie_ngff_candidates(cofie_ngff_t* h, uint32_t stream, uint32_t* idx_out, uint32_t cap, uint32_t* m_out,
                           void* cuda_stream) {
   NvtxRange nvtx("ngff.candidates");
+  if (!h) return COFIE_EINVAL;
+  if (stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
+  if (!m_out) return h->fail(COFIE_EINVAL, "m_out is NULL");
+  DeviceGuard guard(h->device);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  int di = -1;
+  const MemKind ki = cap > 0 ? classify(idx_out, &di) : kNull;
+  if (cap > 0 && (ki == kNull || (ki == kDevice && di != h->device)))
+    return h->fail(COFIE_EINVAL, "idx_out must be device memory on the handle's device, or host memory");
+  const MemKind km = classify(m_out);
+  const int capturing = capture_state(st);
+  if (capturing < 0) return h->fail(COFIE_ECUDA, "cannot read the CUDA stream's capture state");
+  if (capturing && (km != kDevice || (ki != kDevice && ki != kNull)))
+    return h->fail(COFIE_EINVAL, "a captured call takes device idx_out and m_out");
+  if (ki != kDevice && ki != kNull && km == kDevice)
+    return h->fail(COFIE_EINVAL, "a host idx_out needs a host m_out");
+  if (!capturing && h->seen[stream] > h->p.max_stream_frames)
+    return h->fail(COFIE_EINVAL, "the stream has run past its retention record (max_stream_frames)");
+  uint32_t* idx = idx_out;
+  if (ki != kDevice && ki != kNull) {  // host indices: through a device buffer of the record's size
+    if (!h->d_idx) {
+      if (dalloc(&h->d_idx, static_cast<size_t>(h->rec_words) * 32) != cudaSuccess) {
+        cudaGetLastError();
+        h->d_idx = nullptr;
+        return h->fail(COFIE_ENOMEM, "index buffer allocation failed");
+      }
+    }
+    idx = h->d_idx;
+    if (cap > h->p.max_stream_frames) cap = h->p.max_stream_frames;  // |S_c| <= T <= the record's frames
+  }
+  uint32_t* count = km == kDevice ? m_out : h->d_count;
+  cudaError_t e = launch_stream_candidates(h->d_record + static_cast<size_t>(stream) * h->rec_words, h->rec_words,
+                                           h->d_state + stream, h->p.m_min, idx, cap, count, h->d_err, st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "candidates kernel launch");
+  h->n_other += 1;
+  if (km != kDevice) {
+    e = cudaMemcpyAsync(m_out, count, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess && idx != idx_out && *m_out > 0)
+      e = cudaMemcpy(idx_out, idx, static_cast<size_t>(std::min(*m_out, cap)) * sizeof(uint32_t),
+                     cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return h->cuda_fail(e, "candidates count");
+  }
+  return COFIE_OK;
+}
+
+int cofie_ngff_candidates_from_keep(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint32_t* idx_out,
+                                    uint32_t* m_out, void* cuda_stream) {
+  NvtxRange nvtx("ngff.candidates_from_keep");
   if (!h) return COFIE_EINVAL;
   if (!m_out) return h->fail(COFIE_EINVAL, "m_out is NULL");
   DeviceGuard guard(h->device);
@@ -1035,6 +1126,7 @@ int cofie_ngff_candidates(cofie_ngff_t* h, const uint8_t* keep, uint32_t T, uint
   uint32_t* count = km == kDevice ? m_out : h->d_count;
   cudaError_t e = launch_candidates(keep, T, h->p.m_min, idx_out, count, st);
   if (e != cudaSuccess) return h->cuda_fail(e, "candidates kernel launch");
+  h->n_other += 1;
   if (km != kDevice) {
     e = cudaMemcpyAsync(m_out, count, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
@@ -1056,12 +1148,13 @@ int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames,
   cudaError_t e = launch_gather(frames, n_frames, h->frame_bytes, idx, m, out, h->d_err,
                                 static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return h->cuda_fail(e, "gather kernel launch");
+  h->n_other += 1;
   return COFIE_OK;
 }
 
 int cofie_ngff_profile_reset(cofie_ngff_t* h, int time_kernels) {
   if (!h) return COFIE_EINVAL;
-  h->n_hist = h->n_select = h->hist_bytes = 0;
+  h->n_hist = h->n_select = h->n_other = h->hist_bytes = 0;
   h->ev_used = h->ev_sel_used = 0;
   h->time_kernels = time_kernels != 0;
   return COFIE_OK;
@@ -1082,6 +1175,7 @@ int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out) {
   out->hist_ms = hist_ms;
   out->select_timed = h->ev_sel_used / 2;
   out->select_ms = sel_ms;
+  out->other_launches = h->n_other;
   return COFIE_OK;
 }
 

@@ -11,6 +11,9 @@
 //                                     (L_max = 0: [streams][2][B], the previous
 //                                     frame's and the reference frame's rows)
 //   state    StreamState [streams]    frames seen and current gap
+//   record   uint32 [streams][R]      retention record: bit t of stream s is set
+//                                     when frame t was retained (any nonzero keep
+//                                     code), for t < 32 R (cofie_ngff_candidates)
 #pragma once
 
 #include <atomic>
@@ -138,6 +141,7 @@ constexpr uint32_t kErrProducerTimeout = 2u;
 constexpr uint32_t kErrDrainTimeout = 4u;
 constexpr uint32_t kErrBadIndex = 8u;  // a gather index outside the frame buffer
 constexpr uint32_t kErrBounds = 16u;   // checked build: an index check failed
+constexpr uint32_t kErrRecord = 32u;   // candidates of a stream that has run past its retention record
 
 struct HistArgs {
   uint64_t frame_bytes;      // 3 W H
@@ -166,7 +170,24 @@ struct SelectArgs {
   // the same three decisions as integer thresholds on the L1 numerator: the
   // smallest x with fp32(x) / two_n >= tau, T_b, T_s (2^64 - 1: never)
   unsigned long long x_tau, x_cut, x_grad;
+  // the streams' retention records ([streams][rec_words]; nullptr: none)
+  uint32_t* record;
+  uint32_t rec_words;
 };
+
+// Sets the record bits of retained frames: bit i of `bits` stands for frame
+// t_first + i of the stream whose record is `rec` (rec_words words). Frames
+// at or past the record's end are not recorded. One thread per call.
+__device__ __forceinline__ void record_bits(uint32_t* rec, uint32_t rec_words, unsigned long long t_first,
+                                            uint32_t bits) {
+  const unsigned long long cap = 32ull * rec_words;
+  if (!rec || !bits || t_first >= cap) return;
+  if (cap - t_first < 32) bits &= (1u << (cap - t_first)) - 1u;
+  const unsigned long long w = t_first >> 5;
+  const uint32_t sh = static_cast<uint32_t>(t_first & 31);
+  if (bits << sh) atomicOr(rec + w, bits << sh);
+  if (sh && (bits >> (32 - sh))) atomicOr(rec + w + 1, bits >> (32 - sh));
+}
 
 // The spatial signals: per-frame grayscale sums on a grid of cells.
 struct FeatArgs {
@@ -203,8 +224,8 @@ uint32_t hist_chunk_groups();
 size_t hist_smem_bytes(uint32_t bins);
 cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
                              uint32_t* hist, uint32_t* err, int grid, cudaStream_t st, bool pdl = false);
-cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* hist,
-                                cudaStream_t st);
+cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
+                                uint32_t* hist, cudaStream_t st);
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
                           const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl = false);
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,
@@ -212,6 +233,11 @@ cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_
 uint32_t select_small_max();
 cudaError_t launch_select_small(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
                                 StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl = false);
+// pushes of at most select_walk_max_frames() frames per stream with L_max <= select_walk_max_lmax()
+uint32_t select_walk_max_frames();
+uint32_t select_walk_max_lmax();
+cudaError_t launch_select_walk(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
+                               StreamState* state, cudaStream_t st, bool pdl = false);
 cudaError_t launch_features(const SegTable& segs, const FeatArgs& fa, const LumaConsts& lc, uint32_t* feat, uint32_t fw,
                             cudaStream_t st);
 int cells_blocks_per_sm();
@@ -231,6 +257,10 @@ cudaError_t launch_ring_store(const uint32_t* hist, uint32_t rows, unsigned long
                               const SelectArgs& a, uint32_t* ring, cudaStream_t st);
 cudaError_t launch_candidates(const uint8_t* keep, uint32_t T, uint32_t m_min, uint32_t* idx, uint32_t* m_out,
                               cudaStream_t st);
+cudaError_t launch_stream_candidates(const uint32_t* rec, uint32_t rec_words, const StreamState* state,
+                                     uint32_t m_min, uint32_t* idx, uint32_t cap, uint32_t* m_out, uint32_t* err,
+                                     cudaStream_t st);
+cudaError_t launch_stream_reset(StreamState* state, uint32_t* rec, uint32_t rec_words, cudaStream_t st);
 cudaError_t launch_gather(const uint8_t* frames, uint32_t n_frames, uint64_t frame_bytes, const uint32_t* idx, uint32_t m,
                           uint8_t* out, uint32_t* err, cudaStream_t st);
 

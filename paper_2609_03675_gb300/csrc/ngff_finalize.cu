@@ -7,6 +7,12 @@
 //   half up) -- written as sorted indices by a block-wide stream compaction
 //   (ballot + popcount within warps, a scan of the 32 warp totals across them),
 //   one 1024-frame tile at a time.
+// K4 on a stream's retention record (one 1024-thread CTA): the same set for
+//   the prefix a stream has been pushed so far, T read from the stream's
+//   state on the device, the retained frames read from its record (one bit
+//   per frame, written by the selection kernels), one word per thread per
+//   step: popcounts, a block-wide exclusive scan, then each thread writes the
+//   indices of its word's set bits.
 // K5 (2-D grid: frame x slice): copies the m selected frames of a stream back
 //   to back into one buffer (the vision encoder's input), 16 bytes per thread
 //   per step, streaming stores.
@@ -78,6 +84,106 @@ __global__ void __launch_bounds__(kFinThreads) candidates_kernel(const uint8_t* 
   if (tid == 0) *m_out = base;
 }
 
+// Exclusive block-wide prefix sum of one value per thread (kFinThreads
+// threads); *total receives the sum. Uses wsum[kFinWarps] and ends with a
+// barrier, so the caller may reuse both right away.
+__device__ __forceinline__ uint32_t block_exclusive_sum(uint32_t v, uint32_t* wsum, uint32_t* total) {
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  uint32_t x = v;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const uint32_t y = __shfl_up_sync(0xffffffffu, x, d);
+    if (lane >= static_cast<uint32_t>(d)) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t w = wsum[lane];
+    uint32_t z = w;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, z, d);
+      if (lane >= static_cast<uint32_t>(d)) z += y;
+    }
+    wsum[lane] = z - w;
+    if (lane == 31) *total = z;
+  }
+  __syncthreads();
+  const uint32_t r = wsum[warp] + x - v;
+  __syncthreads();
+  return r;
+}
+
+// Bits of record word w of a prefix of T frames that belong to S_c: retained
+// frames before T-1, the last frame T-1, and with `fill` the uniformly spaced
+// frames.
+__device__ __forceinline__ uint32_t candidate_bits(const uint32_t* rec, uint64_t w, uint64_t T, uint32_t m_min,
+                                                   bool fill) {
+  const uint64_t t0 = 32 * w;
+  uint32_t bits = 0;
+  if (t0 < T - 1) {
+    bits = __ldcg(rec + w);
+    if (T - 1 - t0 < 32) bits &= (1u << (T - 1 - t0)) - 1u;
+  }
+  if (T - 1 >= t0 && T - 1 < t0 + 32) bits |= 1u << (T - 1 - t0);
+  if (fill)
+    for (uint32_t i = 0; i < 32 && t0 + i < T; ++i)
+      if (in_uniform(t0 + i, T, m_min)) bits |= 1u << i;
+  return bits;
+}
+
+__global__ void __launch_bounds__(kFinThreads) stream_candidates_kernel(const uint32_t* __restrict__ rec,
+                                                                        uint32_t rec_words,
+                                                                        const StreamState* __restrict__ state,
+                                                                        uint32_t m_min, uint32_t* __restrict__ idx,
+                                                                        uint32_t cap, uint32_t* __restrict__ m_out,
+                                                                        uint32_t* __restrict__ err) {
+  __shared__ uint32_t wsum[kFinWarps];
+  __shared__ uint32_t s_total;
+  const uint32_t tid = threadIdx.x;
+  const uint64_t T = __ldcg(&state->t);
+  if (T > 32ull * rec_words) {  // the stream has run past its record: no candidate set
+    if (tid == 0) {
+      atomicOr(err, kErrRecord);
+      *m_out = 0;
+    }
+    return;
+  }
+  if (T == 0) {
+    if (tid == 0) *m_out = 0;
+    return;
+  }
+  const uint64_t words = (T + 31) / 32;
+  // |S| before the fill: retained frames before T-1, plus T-1
+  uint32_t c = 0;
+  for (uint64_t w = tid; w < words; w += kFinThreads) c += __popc(candidate_bits(rec, w, T, m_min, false));
+  block_exclusive_sum(c, wsum, &s_total);
+  const bool fill = s_total < m_min;
+  uint32_t base = 0;
+  for (uint64_t w0 = 0; w0 < words; w0 += kFinThreads) {
+    const uint64_t w = w0 + tid;
+    uint32_t bits = w < words ? candidate_bits(rec, w, T, m_min, fill) : 0u;
+    const uint32_t off = base + block_exclusive_sum(__popc(bits), wsum, &s_total);
+    for (uint32_t k = 0; bits; ++k, bits &= bits - 1) {
+      const uint32_t pos = off + k;
+      if (pos < cap) idx[pos] = static_cast<uint32_t>(32 * w) + (__ffs(bits) - 1);
+    }
+    base += s_total;
+    __syncthreads();
+  }
+  if (tid == 0) *m_out = base;
+}
+
+// A stream restarts at t = 0: the record bits of the frames it has seen are
+// cleared (bits are set only below t) and its state zeroed.
+__global__ void stream_reset_kernel(StreamState* __restrict__ state, uint32_t* __restrict__ rec, uint32_t rec_words) {
+  const uint64_t t = __ldcg(&state->t);
+  const uint64_t words = min((t + 31) / 32, static_cast<uint64_t>(rec_words));
+  for (uint64_t w = threadIdx.x; w < words; w += blockDim.x) rec[w] = 0;
+  __syncthreads();
+  if (threadIdx.x == 0) *state = StreamState{0ull, 0u, 0u, 0ull};
+}
+
 template <bool kVec>
 __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const uint8_t* __restrict__ frames, uint32_t n_frames,
                                                                 uint64_t frame_bytes, const uint32_t* __restrict__ idx,
@@ -120,6 +226,18 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const uint8_t* _
 cudaError_t launch_candidates(const uint8_t* keep, uint32_t T, uint32_t m_min, uint32_t* idx, uint32_t* m_out,
                               cudaStream_t st) {
   candidates_kernel<<<1, kFinThreads, 0, st>>>(keep, T, m_min, idx, m_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stream_candidates(const uint32_t* rec, uint32_t rec_words, const StreamState* state,
+                                     uint32_t m_min, uint32_t* idx, uint32_t cap, uint32_t* m_out, uint32_t* err,
+                                     cudaStream_t st) {
+  stream_candidates_kernel<<<1, kFinThreads, 0, st>>>(rec, rec_words, state, m_min, idx, cap, m_out, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stream_reset(StreamState* state, uint32_t* rec, uint32_t rec_words, cudaStream_t st) {
+  stream_reset_kernel<<<1, 1024, 0, st>>>(state, rec, rec_words);
   return cudaGetLastError();
 }
 

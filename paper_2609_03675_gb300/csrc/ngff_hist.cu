@@ -345,32 +345,79 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
   }
 }
 
-// Generic kernel: any frame size or alignment. One CTA per (frame, slice of
-// kGenericPixels pixels); byte loads; block-shared counters with atomics.
+// Generic kernel: any frame size or alignment (frames whose pixel count is
+// not a multiple of 16, or that do not start on a 16-byte boundary). Grid
+// (slices, rows): CTA x of row r counts slice x of frame r. A frame's pixels
+// split into a prologue of p_a < 16 pixels, an interior of whole 16-pixel
+// groups that each start on a 16-byte boundary (p_a is the first pixel whose
+// address is 16-byte aligned: frame + 3 p_a = 0 mod 16), and an epilogue of
+// fewer than 16 pixels. Interior groups are loaded with three 128-bit loads
+// and binned as in the fast kernel (two dp2a per pixel, a multiply-high
+// verified on the host); prologue and epilogue pixels with byte loads. Counts
+// go to lane-private shared counters cnt[bin][lane] (bank = lane), folded
+// into the frame's row with one global atomic per bin per CTA.
 constexpr int kGenericThreads = 256;
-constexpr uint32_t kGenericPixels = 16384;
+constexpr uint32_t kGenericGroupsPerCta = 2048;  // 32768 pixels per CTA
+constexpr int kGenericDiv = 3;                   // no verified multiply-high: Y = v / den
 
+template <int kBin>
+__device__ __forceinline__ uint32_t generic_bin(uint32_t v, const LumaConsts& L) {
+  if constexpr (kBin == kGenericDiv) return ((v / L.den) * L.bins) >> 8;
+  else return bin_of<kBin>(v, L);
+}
+
+template <int kBin>
 __global__ void __launch_bounds__(kGenericThreads) hist_generic_kernel(SegTable segs, HistArgs a, LumaConsts L,
                                                                       uint32_t* __restrict__ hist) {
-  __shared__ uint32_t cnt[kMaxBins];
+  extern __shared__ __align__(16) uint32_t gcnt[];  // [B][32]
   pdl_trigger();
-  const uint32_t row = blockIdx.y;
+  const uint32_t row = blockIdx.y, tid = threadIdx.x, lane = tid & 31;
   uint32_t seg = 0;
   while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
   const uint8_t* frame = segs.s[seg].frames + static_cast<uint64_t>(row - segs.s[seg].row0) * a.frame_bytes;
-  for (uint32_t b = threadIdx.x; b < L.bins; b += blockDim.x) cnt[b] = 0;
+  for (uint32_t i = tid; i < L.bins * 32; i += kGenericThreads) gcnt[i] = 0;
   __syncthreads();
-  const uint64_t p0 = static_cast<uint64_t>(blockIdx.x) * kGenericPixels;
-  const uint64_t p1 = min(p0 + kGenericPixels, static_cast<uint64_t>(a.npix));
-  for (uint64_t p = p0 + threadIdx.x; p < p1; p += blockDim.x) {
-    const uint8_t* px = frame + 3 * p;
-    const uint32_t v = L.w[0] * px[0] + L.w[1] * px[1] + L.w[2] * px[2] + L.half;
-    const uint32_t y = v / L.den;
-    if (COFIE_BOUND(((y * L.bins) >> 8) < L.bins)) atomicAdd(&cnt[(y * L.bins) >> 8], 1u);
+  const uint32_t cnt_lane = static_cast<uint32_t>(__cvta_generic_to_shared(gcnt)) + lane * 4;
+  const uint32_t npix = a.npix;
+  // first 16-byte aligned pixel: 3 p = -(frame mod 16) mod 16, and 3 * 11 = 1 mod 16
+  const uint32_t mis = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(frame) & 15u);
+  const uint32_t p_a = min(((16u - mis) * 11u) & 15u, npix);
+  const uint32_t G = (npix - p_a) / 16;
+  const uint32_t g0 = blockIdx.x * kGenericGroupsPerCta, g1 = min(g0 + kGenericGroupsPerCta, G);
+  const uint8_t* base = frame + 3ull * p_a;
+#pragma unroll 2
+  for (uint32_t g = g0 + tid; g < g1; g += kGenericThreads) {
+    const uint4* p = reinterpret_cast<const uint4*>(base + 48ull * g);
+    const uint4 x = __ldcs(p), y = __ldcs(p + 1), z = __ldcs(p + 2);
+    uint32_t v[16];
+    luma4(x.x, x.y, x.z, L, v[0], v[1], v[2], v[3]);
+    luma4(x.w, y.x, y.y, L, v[4], v[5], v[6], v[7]);
+    luma4(y.z, y.w, z.x, L, v[8], v[9], v[10], v[11]);
+    luma4(z.y, z.z, z.w, L, v[12], v[13], v[14], v[15]);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint32_t b = generic_bin<kBin>(v[i], L);
+      if (COFIE_BOUND(b < L.bins)) red_add_shared(cnt_lane + (b << 7));
+    }
   }
+  // the ragged edges: prologue (first CTA of the row) and epilogue (last CTA)
+  const auto scalar = [&](uint32_t q) {
+    const uint8_t* px = frame + 3ull * q;
+    const uint32_t v = L.w[0] * px[0] + L.w[1] * px[1] + L.w[2] * px[2] + L.half;
+    const uint32_t b = generic_bin<kBin>(v, L);
+    if (COFIE_BOUND(b < L.bins)) red_add_shared(cnt_lane + (b << 7));
+  };
+  if (blockIdx.x == 0)
+    for (uint32_t q = tid; q < p_a; q += kGenericThreads) scalar(q);
+  if (blockIdx.x == gridDim.x - 1)
+    for (uint32_t q = p_a + 16 * G + tid; q < npix; q += kGenericThreads) scalar(q);
   __syncthreads();
-  for (uint32_t b = threadIdx.x; b < L.bins; b += blockDim.x)
-    if (cnt[b] && COFIE_BOUND(row < segs.rows)) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, cnt[b]);
+  for (uint32_t b = tid; b < L.bins; b += kGenericThreads) {
+    uint32_t sum = 0;
+#pragma unroll 8
+    for (uint32_t l = 0; l < 32; ++l) sum += gcnt[b * 32 + ((l + b) & 31)];  // rotated: conflict-free
+    if (sum && COFIE_BOUND(row < segs.rows)) atomicAdd(hist + static_cast<uint64_t>(row) * L.bins + b, sum);
+  }
 }
 
 }  // namespace
@@ -437,10 +484,17 @@ cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const Luma
   return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
-cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, uint32_t* hist,
-                                cudaStream_t st) {
-  dim3 grid((a.npix + kGenericPixels - 1) / kGenericPixels, segs.rows);
-  hist_generic_kernel<<<grid, kGenericThreads, 0, st>>>(segs, a, lc, hist);
+cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
+                                uint32_t* hist, cudaStream_t st) {
+  const uint32_t groups = a.npix / 16;  // at least the interior's groups, whatever the alignment
+  dim3 grid(groups ? (groups + kGenericGroupsPerCta - 1) / kGenericGroupsPerCta : 1, segs.rows);
+  const size_t smem = static_cast<size_t>(lc.bins) * 32 * 4;
+  if (bin_path == kBinFast)
+    hist_generic_kernel<kBinFast><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
+  else if (bin_path == kBinTwoStep)
+    hist_generic_kernel<kBinTwoStep><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
+  else
+    hist_generic_kernel<kGenericDiv><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
   return cudaGetLastError();
 }
 

@@ -252,10 +252,18 @@ __global__ void __launch_bounds__(kLazyThreads) lazy_select_kernel(SegTable segs
       }
     }
     __syncthreads();
-    for (uint32_t f = tid; f < m; f += kLazyThreads) {
-      const bool first = t0 + j0 + f == 0;
-      if (sg.scores) sg.scores[j0 + f] = first ? 0.0f : __fdiv_rn(static_cast<float>(sd[f]), a.two_n);
-      if (sg.keep) sg.keep[j0 + f] = scode[f];
+    for (uint32_t base = 0; base < m; base += kLazyThreads) {  // warps stay whole: the record takes a ballot
+      const uint32_t f = base + tid;
+      bool kept = false;
+      if (f < m) {
+        const bool first = t0 + j0 + f == 0;
+        if (sg.scores) sg.scores[j0 + f] = first ? 0.0f : __fdiv_rn(static_cast<float>(sd[f]), a.two_n);
+        if (sg.keep) sg.keep[j0 + f] = scode[f];
+        kept = scode[f] != 0;
+      }
+      const uint32_t bits = __ballot_sync(0xffffffffu, kept);
+      if (lane == 0 && a.record)
+        record_bits(a.record + static_cast<uint64_t>(sg.stream) * a.rec_words, a.rec_words, t0 + j0 + f, bits);
     }
     if (tile + 1 < n_tiles) {
       for (uint32_t b = tid; b < B; b += kLazyThreads) sprev[b] = buf[(m - 1) * B + b];

@@ -26,6 +26,11 @@
 //
 // Small pushes (at most kSmallMax frames per stream) run K2 and K3 as one
 // kernel: the same CTA first computes its stream's distances, then scans.
+// With at most kWalkMaxFrames frames per stream and L_max <= kWalkMaxLmax the
+// push is smaller still and a lighter kernel decides it (select_walk_kernel):
+// one 128-thread CTA per stream keeps the distances and keep bits in shared
+// memory and walks the rule in frame order from the stream's gap, which for
+// so few frames is shorter than composing gap maps.
 #include "ngff_common.cuh"
 
 namespace cofie {
@@ -36,6 +41,9 @@ constexpr int kScanThreads = 1024;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr uint32_t kScanTile = 4096;  // frames per shared-memory tile
 constexpr uint32_t kSmallMax = 64;    // frames per stream segment for the fused small-push kernel
+constexpr int kWalkThreads = 128;
+constexpr uint32_t kWalkMaxFrames = 64;
+constexpr uint32_t kWalkMaxLmax = 64;
 
 __device__ __forceinline__ uint32_t absdiff(uint32_t a, uint32_t b) { return a > b ? a - b : b - a; }
 
@@ -268,19 +276,26 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
       }
     }
     __syncthreads();
-#pragma unroll 4
-    for (uint32_t f = tid; f < m; f += kScanThreads) {
+    for (uint32_t base = 0; base < m; base += kScanThreads) {  // warps stay whole: the record takes a ballot
+      const uint32_t f = base + tid;
       const uint32_t jj = tile0 + f;
-      uint32_t g = sgap[f];
-      if (!COFIE_BOUND(g >= 1 && g <= L)) g = 1;  // checked build: keep the L1 read in its row
-      const uint64_t r = static_cast<uint64_t>(row0 + jj) * L;
-      const uint32_t lm = max(l1[r], l1[r + g - 1]);
-      const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
-      const bool nov = s >= a.tau;
-      const bool scene = a.scd && ((sflag[f >> 5] >> (f & 31)) & 1u);
-      const uint8_t code = nov ? 1 : (scene ? 4 : (g >= L ? 2 : 0));
-      if (sseg.scores) sseg.scores[jj] = s;
-      if (sseg.keep) sseg.keep[jj] = code;
+      bool kept = false;
+      if (f < m) {
+        uint32_t g = sgap[f];
+        if (!COFIE_BOUND(g >= 1 && g <= L)) g = 1;  // checked build: keep the L1 read in its row
+        const uint64_t r = static_cast<uint64_t>(row0 + jj) * L;
+        const uint32_t lm = max(l1[r], l1[r + g - 1]);
+        const float s = __fdiv_rn(static_cast<float>(lm), a.two_n);
+        const bool nov = s >= a.tau;
+        const bool scene = a.scd && ((sflag[f >> 5] >> (f & 31)) & 1u);
+        const uint8_t code = nov ? 1 : (scene ? 4 : (g >= L ? 2 : 0));
+        if (sseg.scores) sseg.scores[jj] = s;
+        if (sseg.keep) sseg.keep[jj] = code;
+        kept = code != 0;
+      }
+      const uint32_t bits = __ballot_sync(0xffffffffu, kept);
+      if (lane == 0 && a.record)
+        record_bits(a.record + static_cast<uint64_t>(stream) * a.rec_words, a.rec_words, t0 + jj, bits);
     }
     g_entry = entry[kScanWarps];
     __syncthreads();
@@ -290,6 +305,7 @@ __device__ __forceinline__ void scan_segment(const Segment& sseg, unsigned long 
     if (t0 == 0) {  // first frame of the stream: always retained, score 0
       if (sseg.scores) sseg.scores[0] = 0.0f;
       if (sseg.keep) sseg.keep[0] = 3;
+      if (a.record) record_bits(a.record + static_cast<uint64_t>(stream) * a.rec_words, a.rec_words, 0ull, 1u);
     }
     state[stream].t = t0 + n;
     state[stream].g = g_entry;
@@ -365,6 +381,161 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
   scan_segment<kOneWord>(sseg, s_t0, s_g, s_acc, a, l1, mask, hist, ring, state, ssm, entry);
 }
 
+// Small pushes, one 128-thread CTA per stream segment (n <= kWalkMaxFrames,
+// L_max <= kWalkMaxLmax), in the order the rule states it:
+//   1. windowed distances, a warp per frame, lane = lag k (the Eq. 2
+//      numerators L1[j][k-1] = sum_b |c_t - c_{t-k}|, from the push's rows or
+//      the stream's ring), and the keep bit of every possible gap g (Eqs. 3-5:
+//      fp32(max(L1[j][0], L1[j][g-1])) / fp32(2N) >= tau_h, or g >= L_max),
+//      into shared memory;
+//   2. one thread walks the frames in order from the stream's gap: frame j is
+//      kept when its bit for the current gap is set (or, with scene changes,
+//      when twin comparison of the adjacent differences finds one, with the
+//      numerator thresholds that equal the fp32 decisions), and the gap
+//      becomes 1 on a keep and g + 1 otherwise;
+//   3. all threads emit scores and keep codes, note retained frames in the
+//      stream's retention record, store the last L_max rows in the ring,
+//      update the stream state and zero the push's rows for the next push.
+template <bool kVec4>
+__global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs, SelectArgs a,
+                                                                   uint32_t* __restrict__ hist,
+                                                                   uint32_t* __restrict__ ring,
+                                                                   StreamState* __restrict__ state) {
+  constexpr uint32_t kWarps = kWalkThreads / 32;
+  extern __shared__ __align__(16) uint32_t wsm[];
+  __shared__ unsigned long long s_t0, s_acc;
+  __shared__ uint32_t s_g;
+  pdl_trigger();  // the next push's first-stage kernel may be scheduled; it waits for this grid before its work
+  pdl_wait();     // every device read follows: the histograms before it, and the state the last push left
+  const Segment sg = segs.s[blockIdx.x];
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t n = sg.n, row0 = sg.row0, stream = sg.stream;
+  const uint32_t B = a.bins, L = a.l_max, W = a.mask_words;
+  if (n == 0) return;
+  uint32_t* sl1 = wsm;               // [n][L]
+  uint32_t* smask = sl1 + n * L;     // [n][W]
+  uint32_t* sgap = smask + n * W;    // [n]: gap, bit 31 a scene change
+  if (tid == 0) {
+    s_t0 = state[stream].t;
+    s_acc = state[stream].acc;
+    s_g = state[stream].g;
+  }
+  __syncthreads();
+  const unsigned long long t0 = s_t0;
+  const uint32_t* ring_s = ring + static_cast<uint64_t>(stream) * L * B;
+
+  // 1. distances and keep bits
+  for (uint32_t j = warp; j < n; j += kWarps) {
+    const unsigned long long t = t0 + j;
+    const uint32_t* ct = hist + static_cast<uint64_t>(row0 + j) * B;
+    uint32_t l_adj = 0;
+    for (uint32_t w = 0; w < W; ++w) {
+      const uint32_t k = 32 * w + lane + 1;
+      const bool valid = k <= L && k <= t;
+      const uint32_t* src = ct;
+      if (valid) src = k <= j ? ct - static_cast<uint64_t>(k) * B : ring_s + ((t - k) % L) * B;
+      uint32_t d = 0;
+      if (kVec4) {
+        const uint4* c4 = reinterpret_cast<const uint4*>(ct);
+        const uint4* s4 = reinterpret_cast<const uint4*>(src);
+#pragma unroll 8
+        for (uint32_t q = 0; q < B / 4; ++q) {
+          const uint4 x = c4[q], y = s4[q];
+          d += absdiff(x.x, y.x) + absdiff(x.y, y.y) + absdiff(x.z, y.z) + absdiff(x.w, y.w);
+        }
+      } else if (a.dist_kind == 1) {  // Hamming distance of bit vectors (dHash)
+        for (uint32_t b = 0; b < B; ++b) d += __popc(ct[b] ^ src[b]);
+      } else {
+#pragma unroll 4
+        for (uint32_t b = 0; b < B; ++b) d += absdiff(ct[b], src[b]);
+      }
+      if (!valid) d = 0;
+      if (w == 0) l_adj = __shfl_sync(0xffffffffu, d, 0);  // lag 1
+      if (k <= L) sl1[j * L + k - 1] = d;
+      bool keep = false;
+      if (k <= L) keep = __fdiv_rn(static_cast<float>(max(l_adj, d)), a.two_n) >= a.tau || k >= L;
+      const uint32_t m = __ballot_sync(0xffffffffu, keep);
+      if (lane == 0) smask[j * W + w] = m;
+    }
+  }
+  __syncthreads();
+
+  // 2. the rule in frame order
+  if (tid == 0) {
+    uint32_t g = s_g;
+    if (g < 1 || g > L) g = L;  // the state only ever holds [1, L]
+    unsigned long long acc = t0 == 0 ? 0ull : s_acc;
+    for (uint32_t j = 0; j < n; ++j) {
+      if (t0 + j == 0) {  // the stream's first frame: kept, the gap restarts
+        sgap[j] = 1;
+        g = 1;
+        continue;
+      }
+      bool scene = false;
+      if (a.scd) {
+        const unsigned long long adj = sl1[j * L];
+        if (adj >= a.x_cut) {  // a cut ends the run
+          scene = true;
+          acc = 0;
+        } else if (adj >= a.x_grad) {  // joins the run: a gradual change where its sum first reaches T_b
+          acc += adj;
+          scene = acc >= a.x_cut && acc - adj < a.x_cut;
+        } else {  // a low difference ends the run
+          acc = 0;
+        }
+      }
+      const bool keep = ((smask[j * W + ((g - 1) >> 5)] >> ((g - 1) & 31)) & 1u) || scene;
+      sgap[j] = g | (scene ? 0x80000000u : 0u);
+      g = keep ? 1u : g + 1u;
+    }
+    s_acc = acc;
+    s_g = g;
+  }
+  __syncthreads();
+
+  // 3. outputs, the retention record, ring, state, and the rows cleared
+  uint32_t* rec = a.record ? a.record + static_cast<uint64_t>(stream) * a.rec_words : nullptr;
+  for (uint32_t base = 0; base < n; base += kWalkThreads) {
+    const uint32_t j = base + tid;
+    bool kept = false;
+    if (j < n) {
+      float s = 0.0f;
+      uint8_t code = 3;
+      if (t0 + j != 0) {
+        uint32_t g = sgap[j] & 0x7fffffffu;
+        if (!COFIE_BOUND(g >= 1 && g <= L)) g = 1;
+        s = __fdiv_rn(static_cast<float>(max(sl1[j * L], sl1[j * L + g - 1])), a.two_n);
+        const bool nov = s >= a.tau, scene = sgap[j] >> 31;
+        code = nov ? 1 : (scene ? 4 : (g >= L ? 2 : 0));
+      }
+      if (sg.scores) sg.scores[j] = s;
+      if (sg.keep) sg.keep[j] = code;
+      kept = code != 0;
+    }
+    const uint32_t bits = __ballot_sync(0xffffffffu, kept);
+    if (lane == 0 && rec) record_bits(rec, a.rec_words, t0 + base + 32 * warp, bits);
+  }
+  const uint32_t keep_n = min(n, L);
+  uint32_t* ring_w = ring + static_cast<uint64_t>(stream) * L * B;
+  for (uint32_t i = tid; i < keep_n * B; i += kWalkThreads) {
+    const uint32_t jj = n - keep_n + i / B, b = i % B;
+    ring_w[((t0 + jj) % L) * B + b] = hist[static_cast<uint64_t>(row0 + jj) * B + b];
+  }
+  if (tid == 0) {
+    state[stream].t = t0 + n;
+    state[stream].g = s_g;
+    state[stream].acc = s_acc;
+  }
+  if (a.zero_hist) {
+    __syncthreads();  // the ring copies above have read the rows
+    for (uint32_t i = tid; i < n * B; i += kWalkThreads) hist[static_cast<uint64_t>(row0) * B + i] = 0;
+  }
+}
+
+size_t walk_smem_bytes(uint32_t n, uint32_t l_max, uint32_t mask_words) {
+  return static_cast<size_t>(n) * (l_max + mask_words + 1) * 4;
+}
+
 // The gap map of one stream segment: map[g-1] = the gap after its last frame
 // when its first frame is entered with gap g (for a stream's first segment,
 // frame 0 is a first frame and every entry gives the same result). One CTA:
@@ -429,6 +600,22 @@ size_t scan_smem_bytes(uint32_t mask_words, uint32_t l_max) {
 }  // namespace
 
 uint32_t select_small_max() { return kSmallMax; }
+uint32_t select_walk_max_frames() { return kWalkMaxFrames; }
+uint32_t select_walk_max_lmax() { return kWalkMaxLmax; }
+
+cudaError_t launch_select_walk(const SegTable& segs, const SelectArgs& a, uint32_t* hist, uint32_t* ring,
+                               StreamState* state, cudaStream_t st, bool pdl) {
+  uint32_t longest = 0;
+  for (uint32_t i = 0; i < segs.count; ++i) longest = max(longest, segs.s[i].n);
+  const size_t smem = walk_smem_bytes(longest, a.l_max, a.mask_words);  // <= 17,152 bytes
+  const cudaError_t e =
+      (a.bins % 4 == 0 && a.dist_kind == 0)
+          ? launch_dependent(pdl, select_walk_kernel<true>, dim3(segs.count), dim3(kWalkThreads), smem, st, segs, a,
+                             hist, ring, state)
+          : launch_dependent(pdl, select_walk_kernel<false>, dim3(segs.count), dim3(kWalkThreads), smem, st, segs, a,
+                             hist, ring, state);
+  return e == cudaSuccess ? cudaGetLastError() : e;
+}
 
 cudaError_t launch_gap_map(const Segment& seg, const SelectArgs& a, unsigned long long t0, const uint32_t* mask,
                            uint16_t* map_out, cudaStream_t st) {

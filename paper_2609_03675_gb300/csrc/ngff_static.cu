@@ -13,9 +13,11 @@
 //
 // It is a variant of the library's scan kernel: one 1024-thread CTA first
 // writes the windowed L1 distances and the per-gap keep bits of every frame
-// into the static array (the work the window kernel does), then runs the same
+// into the static array (the work the window kernel does: a warp per frame,
+// lane = lag, 16-byte loads when the rows allow them), then runs the same
 // gap-map scan over them. Decisions and scores equal those of
-// cofie_ngff_push_ex on a fresh stream.
+// cofie_ngff_push_ex on a fresh stream of the histogram signal without scene
+// changes (other signals are refused).
 //
 // The array holds kStaticScratchWords 32-bit words (4 MiB) on every GPU that
 // loads the library, until the process exits. Every call shares it and it
@@ -45,6 +47,7 @@ __device__ __forceinline__ uint32_t next_gap(const uint32_t* m, uint32_t g) {
   return ((m[(g - 1) >> 5] >> ((g - 1) & 31)) & 1u) ? 1u : g + 1u;
 }
 
+template <bool kVec4>
 __global__ void __launch_bounds__(kThreads) select_static_kernel(const uint32_t* __restrict__ hist, uint32_t n,
                                                                  SelectArgs a, uint32_t* __restrict__ scratch,
                                                                  float* __restrict__ scores,
@@ -55,34 +58,38 @@ __global__ void __launch_bounds__(kThreads) select_static_kernel(const uint32_t*
   const uint32_t B = a.bins, L = a.l_max, W = a.mask_words;
   uint32_t* l1 = scratch;                                   // [n][L]
   uint32_t* mask = scratch + static_cast<uint64_t>(n) * L;  // [n][W]
-  uint32_t* sl1 = sm;                                       // phase 1: [kWarps][L]
 
-  // phase 1: windowed distances and per-gap keep bits of every frame (warp per frame)
+  // phase 1: windowed distances and per-gap keep bits of every frame (warp per
+  // frame, lane = lag k: the lane sums |c_t - c_{t-k}| over all bins, so the
+  // warp's loads are independent and in flight together)
   for (uint32_t t = warp; t < n; t += kWarps) {
     const uint32_t* ct = hist + static_cast<uint64_t>(t) * B;
-    for (uint32_t k = 1; k <= L; ++k) {
-      uint32_t d = 0;
-      if (k <= t) {
-        const uint32_t* cs = ct - static_cast<uint64_t>(k) * B;
-        for (uint32_t b = lane; b < B; b += 32) d += absdiff(ct[b], cs[b]);
-        d = __reduce_add_sync(0xffffffffu, d);
-      }
-      if (lane == 0) sl1[warp * L + k - 1] = d;
-    }
-    __syncwarp();
-    for (uint32_t k = lane; k < L; k += 32) l1[static_cast<uint64_t>(t) * L + k] = sl1[warp * L + k];
-    const uint32_t l_adj = sl1[warp * L];
+    uint32_t l_adj = 0;
     for (uint32_t w = 0; w < W; ++w) {
-      const uint32_t g = 32 * w + lane + 1;
-      bool kp = false;
-      if (g <= L) {
-        const float s = __fdiv_rn(static_cast<float>(max(l_adj, sl1[warp * L + g - 1])), a.two_n);
-        kp = (s >= a.tau) || (g >= L);
+      const uint32_t k = 32 * w + lane + 1;
+      const bool valid = k <= L && k <= t;
+      const uint32_t* cs = valid ? ct - static_cast<uint64_t>(k) * B : ct;
+      uint32_t d = 0;
+      if (kVec4) {
+        const uint4* c4 = reinterpret_cast<const uint4*>(ct);
+        const uint4* s4 = reinterpret_cast<const uint4*>(cs);
+#pragma unroll 8
+        for (uint32_t q = 0; q < B / 4; ++q) {
+          const uint4 x = c4[q], y = s4[q];
+          d += absdiff(x.x, y.x) + absdiff(x.y, y.y) + absdiff(x.z, y.z) + absdiff(x.w, y.w);
+        }
+      } else {
+#pragma unroll 4
+        for (uint32_t b = 0; b < B; ++b) d += absdiff(ct[b], cs[b]);
       }
+      if (!valid) d = 0;
+      if (w == 0) l_adj = __shfl_sync(0xffffffffu, d, 0);  // lag 1
+      if (k <= L) l1[static_cast<uint64_t>(t) * L + k - 1] = d;
+      bool kp = false;
+      if (k <= L) kp = __fdiv_rn(static_cast<float>(max(l_adj, d)), a.two_n) >= a.tau || k >= L;
       const uint32_t m = __ballot_sync(0xffffffffu, kp);
       if (lane == 0) mask[static_cast<uint64_t>(t) * W + w] = m;
     }
-    __syncwarp();
   }
   __syncthreads();
 
@@ -138,9 +145,7 @@ __global__ void __launch_bounds__(kThreads) select_static_kernel(const uint32_t*
 }
 
 size_t static_smem_bytes(uint32_t l_max, uint32_t mask_words) {
-  const size_t phase1 = static_cast<size_t>(kWarps) * l_max * 4;
-  const size_t phase2 = static_cast<size_t>(kTile) * mask_words * 4 + kTile * 2 + static_cast<size_t>(kWarps) * l_max * 2;
-  return phase1 > phase2 ? phase1 : phase2;
+  return static_cast<size_t>(kTile) * mask_words * 4 + kTile * 2 + static_cast<size_t>(kWarps) * l_max * 2;
 }
 
 // Per-device set-up: the device address of the static array, and the kernel's
@@ -154,8 +159,10 @@ cudaError_t setup_device(int dev, uint32_t** out) {
     void* ptr = nullptr;
     cudaError_t e = cudaGetSymbolAddress(&ptr, g_select_scratch);
     if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(select_static_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             static_cast<int>(static_smem_bytes(kMaxLmax, (kMaxLmax + 31) / 32)));
+    const int smem = static_cast<int>(static_smem_bytes(kMaxLmax, (kMaxLmax + 31) / 32));
+    e = cudaFuncSetAttribute(select_static_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(select_static_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     g_scratch_ptr[dev] = static_cast<uint32_t*>(ptr);
   }
@@ -199,6 +206,9 @@ int cofie_ngff_select_static(const cofie_ngff_params* p, const uint32_t* hist, u
   if (p->l_max < 1 || p->l_max > COFIE_NGFF_MAX_LMAX)
     return fail(COFIE_EINVAL, "l_max must be in [1, 256]", err, err_cap);
   if (p->tau != p->tau) return fail(COFIE_EINVAL, "tau is NaN", err, err_cap);
+  if (p->signal != COFIE_SIGNAL_HISTOGRAM)
+    return fail(COFIE_EINVAL, "only the histogram signal (COFIE_SIGNAL_HISTOGRAM, no scene changes) is supported",
+                err, err_cap);
   if (n == 0) return COFIE_OK;
   const uint32_t W = (p->l_max + 31) / 32;
   if (static_cast<uint64_t>(n) * (p->l_max + W) > kStaticScratchWords)
@@ -221,8 +231,12 @@ int cofie_ngff_select_static(const cofie_ngff_params* p, const uint32_t* hist, u
   a.mask_words = W;
   a.tau = p->tau;
   a.two_n = static_cast<float>(2ull * p->width * p->height);
-  select_static_kernel<<<1, kThreads, static_smem_bytes(p->l_max, W), static_cast<cudaStream_t>(cuda_stream)>>>(
-      hist, n, a, scratch, scores_out, keep_out);
+  const size_t smem = static_smem_bytes(p->l_max, W);
+  const cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (p->bins % 4 == 0 && reinterpret_cast<uintptr_t>(hist) % 16 == 0)
+    select_static_kernel<true><<<1, kThreads, smem, st>>>(hist, n, a, scratch, scores_out, keep_out);
+  else
+    select_static_kernel<false><<<1, kThreads, smem, st>>>(hist, n, a, scratch, scores_out, keep_out);
   e = cudaGetLastError();
   if (e != cudaSuccess) return fail(COFIE_ECUDA, cudaGetErrorString(e), err, err_cap);
   return COFIE_OK;

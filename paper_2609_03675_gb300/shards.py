@@ -53,9 +53,21 @@ def sharded_decide(prepare: Callable[[], torch.Tensor], commit: Callable[[int], 
     return commit(entry_gaps([m.tolist() for m in maps])[rank])
 
 
-def sharded_push(f, frames: torch.Tensor, T: int, rank: int, world: int, group=None, stream: int = 0):
-    """Rank's shard of a T-frame stream whose frames (all T, on this rank's
-    device) are given; returns (scores, keep) of frames [a, b)."""
+def shard_frames(T: int, world: int, rank: int, l_max: int) -> tuple[int, int]:
+    """The frames [lo, hi) a rank must hold for its shard of a T-frame stream:
+    its halo of min(a, L_max) frames, then its own frames [a, b)."""
+    a, b, halo = shard_bounds(T, world, rank, l_max)
+    return a - halo, b
+
+
+def sharded_push(f, local_frames: torch.Tensor, T: int, rank: int, world: int, group=None, stream: int = 0):
+    """Decides rank's shard of a T-frame stream. local_frames holds only the
+    frames shard_frames() names (the halo, then the shard: b - a + halo
+    frames on this rank's device), so per-rank memory is the shard plus
+    L_max frames. Returns (scores, keep) of frames [a, b)."""
     a, b, halo = shard_bounds(T, world, rank, f.l_max)
-    return sharded_decide(lambda: f.shard_prepare(frames[a - halo:b], n_halo=halo, t0=a, stream=stream),
+    if local_frames.shape[0] != b - a + halo:
+        raise ValueError(f"rank {rank} needs frames [{a - halo}, {b}) ({b - a + halo} frames), "
+                         f"got {local_frames.shape[0]}")
+    return sharded_decide(lambda: f.shard_prepare(local_frames, n_halo=halo, t0=a, stream=stream),
                           lambda g: f.shard_commit(g, b - a, stream=stream), rank, world, group)

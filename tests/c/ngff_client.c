@@ -1,11 +1,13 @@
 /* A plain C client of libcofie_ngff.so (no CUDA runtime, no Python): reads
  * frames from a file, pushes them from pageable host memory in pieces of the
- * given sizes, and writes every frame's score and keep code (host outputs)
- * to an output file.
+ * given sizes, closing the stream after every piece (its candidate set S_c,
+ * into host memory), and writes every frame's score and keep code (host
+ * outputs) and each piece's candidate set to an output file.
  * Usage: ngff_client IN OUT WIDTH HEIGHT FRAMES TAU L_MAX PIECE...
- * IN holds FRAMES * WIDTH * HEIGHT * 3 bytes; OUT receives FRAMES floats and
- * FRAMES keep bytes. Exit status 0 on success; a failing call prints the
- * library's message. */
+ * IN holds FRAMES * WIDTH * HEIGHT * 3 bytes; OUT receives FRAMES floats,
+ * FRAMES keep bytes, then per piece: the prefix length T (uint32), |S_c|
+ * (uint32) and |S_c| uint32 indices. Exit status 0 on success; a failing
+ * call prints the library's message. */
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
@@ -31,7 +33,8 @@ int main(int argc, char** argv) {
   uint8_t* frames = malloc(frame_bytes * T);
   float* scores = malloc(sizeof(float) * T);
   uint8_t* keep = malloc(T);
-  if (!frames || !scores || !keep) return 3;
+  uint32_t* idx = malloc(sizeof(uint32_t) * (T ? T : 1));
+  if (!frames || !scores || !keep || !idx) return 3;
   FILE* in = fopen(argv[1], "rb");
   if (!in || fread(frames, 1, frame_bytes * T, in) != frame_bytes * T) return 4;
   fclose(in);
@@ -44,6 +47,9 @@ int main(int argc, char** argv) {
   cofie_ngff_t* h = NULL;
   if (check(cofie_ngff_create(&p, &h), NULL, "cofie_ngff_create")) return 1;
 
+  FILE* out = fopen(argv[2], "wb");
+  if (!out) return 5;
+  fseek(out, (long)(T * (sizeof(float) + 1)), SEEK_SET); /* the candidate sets follow scores and keep codes */
   uint32_t off = 0;
   for (int a = 8; a < argc && off < T; ++a) {
     uint32_t n = (uint32_t)strtoul(argv[a], NULL, 10);
@@ -52,6 +58,12 @@ int main(int argc, char** argv) {
               "cofie_ngff_push"))
       return 1;
     off += n;
+    uint32_t m = 0;
+    if (check(cofie_ngff_candidates(h, 0, idx, T, &m, NULL), h, "cofie_ngff_candidates")) return 1;
+    if (m > off) return 6;
+    fwrite(&off, sizeof off, 1, out);
+    fwrite(&m, sizeof m, 1, out);
+    fwrite(idx, sizeof(uint32_t), m, out);
   }
   if (off != T) {
     fprintf(stderr, "pieces cover %u of %u frames\n", off, T);
@@ -60,13 +72,13 @@ int main(int argc, char** argv) {
   if (check(cofie_ngff_status(h, NULL), h, "cofie_ngff_status")) return 1;
   cofie_ngff_destroy(h);
 
-  FILE* out = fopen(argv[2], "wb");
-  if (!out) return 5;
+  fseek(out, 0, SEEK_SET);
   fwrite(scores, sizeof(float), T, out);
   fwrite(keep, 1, T, out);
   fclose(out);
   free(frames);
   free(scores);
   free(keep);
+  free(idx);
   return 0;
 }

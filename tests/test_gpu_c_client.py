@@ -1,7 +1,8 @@
 """The C ABI from plain C: tests/c/ngff_client.c (C99, linked against the
 library only: no CUDA runtime, no Python) pushes seeded frames from pageable
-host memory in uneven pieces; its scores and keep codes must equal the
-oracle's."""
+host memory in uneven pieces and closes the stream after each piece; its
+scores and keep codes must equal the oracle's, and each candidate set the
+oracle's candidate set of that prefix."""
 import os
 import shutil
 import subprocess
@@ -51,7 +52,19 @@ def test_c_client_matches_oracle(client, tau, l_max):
     T = spec.frames
     scores = raw[: 4 * T].view(np.float32).astype(np.float64)
     keep = raw[4 * T: 5 * T]
-    _, so, ko = O.load().run(frames, O.Params(spec.width, spec.height, tau=tau, l_max=l_max))
+    o = O.load()
+    _, so, ko = o.run(frames, O.Params(spec.width, spec.height, tau=tau, l_max=l_max))
     assert np.array_equal(keep, ko), np.flatnonzero(keep != ko)[:10]
     assert np.all(np.abs(scores - so) <= 1e-6 * so)
     assert (ko == O.KEEP_NOVELTY).any()
+    # the candidate set after each piece: S_c of that prefix (Sec. 3.2 closing safeguards)
+    rest = raw[5 * T:].view(np.uint32)
+    pos, prefixes = 0, []
+    while pos < rest.size:
+        t_pre, m = int(rest[pos]), int(rest[pos + 1])
+        got_idx = rest[pos + 2: pos + 2 + m]
+        want_idx = o.candidates(ko[:t_pre], 4)
+        assert np.array_equal(got_idx, want_idx), f"prefix {t_pre}"
+        prefixes.append(t_pre)
+        pos += 2 + m
+    assert prefixes == list(np.cumsum([int(x) for x in pieces]))

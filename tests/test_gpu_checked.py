@@ -131,7 +131,8 @@ n += 1
 # candidates and gather of a closed prefix
 f = NGFF(64, 48, tau=0.05, l_max=12)
 s, k = f.push(dev)
-idx = f.candidates(k)
+idx = f.candidates(0)
+assert torch.equal(f.candidates_from_keep(k), idx)
 out = f.gather(dev, idx)
 torch.cuda.synchronize(); f.status()
 want = O.load().candidates(ko, 4)

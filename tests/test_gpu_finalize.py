@@ -30,7 +30,7 @@ def test_candidates_small_prefixes_exhaustive():
         for m_min, f in handles.items():
             for density in (0.0, 0.1, 0.5):
                 keep = ((g.random(T) < density) * g.integers(1, 4, size=T)).astype(np.uint8)
-                got = f.candidates(torch.from_numpy(keep).cuda()).cpu().numpy().astype(np.uint32)
+                got = f.candidates_from_keep(torch.from_numpy(keep).cuda()).cpu().numpy().astype(np.uint32)
                 want = o.candidates(keep, m_min)
                 assert np.array_equal(got, want), f"T={T} M_min={m_min} keep={keep}"
 
@@ -40,13 +40,15 @@ def test_candidates_small_prefixes_exhaustive():
 def test_candidates_long_prefixes(T, density, m_min):
     g = np.random.default_rng(T + m_min)
     keep = ((g.random(T) < density) * g.integers(1, 4, size=T)).astype(np.uint8)
-    got = _ngff(16, 16, m_min=m_min).candidates(torch.from_numpy(keep).cuda()).cpu().numpy().astype(np.uint32)
+    f = _ngff(16, 16, m_min=m_min)
+    got = f.candidates_from_keep(torch.from_numpy(keep).cuda()).cpu().numpy().astype(np.uint32)
     assert np.array_equal(got, O.load().candidates(keep, m_min))
 
 
 def test_empty_prefix():
     f = _ngff(16, 16)
-    assert f.candidates(torch.zeros(0, dtype=torch.uint8, device="cuda")).numel() == 0
+    assert f.candidates_from_keep(torch.zeros(0, dtype=torch.uint8, device="cuda")).numel() == 0
+    assert f.candidates(0).numel() == 0  # a stream with no frames yet
 
 
 @pytest.mark.parametrize("w,h", [(160, 96), (17, 13)])
@@ -55,8 +57,8 @@ def test_push_candidates_gather_pipeline(w, h):
     fr = synth.generate(spec)
     f = _ngff(w, h, tau=0.05, m_min=4)
     dev = torch.from_numpy(fr).cuda()
-    _, keep = f.push(dev)
-    idx = f.candidates(keep)
+    f.push(dev)
+    idx = f.candidates(0)
     out = f.gather(dev, idx)
     torch.cuda.synchronize()
     f.status()

@@ -47,7 +47,7 @@ def test_hd1080_whole_stream_push():
         band = assert_parity(got, (hist_o, *sel[tau]), tau, f"1080p tau={tau}")
         print(f"1080p tau={tau}: kept {int((got[2] != 0).sum())}/{spec.frames}, band frames {list(band)}")
         # close the prefix and gather the encoder's input
-        idx = f.candidates(torch.from_numpy(got[2]).cuda())
+        idx = f.candidates(0)  # the stream's own retention record
         want_idx = O.load().candidates(sel[tau][1], 4)
         assert np.array_equal(idx.cpu().numpy().astype(np.uint32), want_idx)
         out = f.gather(dev, idx)
@@ -56,6 +56,17 @@ def test_hd1080_whole_stream_push():
         assert torch.equal(out.cpu(), buf[torch.from_numpy(want_idx.astype(np.int64))])
         del out
         f.close()
+    # the same stream pushed in pieces and closed after each (Sec. 3.2 closing
+    # safeguards on the stream's own retention record)
+    f = NGFF(spec.width, spec.height, tau=0.30, max_frames_per_push=1600)
+    off = 0
+    for n in (1, 2, 997, 1000, 1600):
+        f.push(dev[off:off + n])
+        off += n
+        idx = f.candidates(0).cpu().numpy().astype(np.uint32)
+        assert np.array_equal(idx, O.load().candidates(sel[0.30][1][:off], 4)), f"1080p prefix {off}"
+    f.status()
+    f.close()
     del buf
     # every scene cut of the textured stream moves the histogram past tau = 0.30
     cuts = synth.scene_starts(spec)[1:]
@@ -153,6 +164,10 @@ def test_serving_32_streams_batched():
             pos[s] += n
         f.push_batch(items)
         call += 1
+        if call in (1, 2, 57, 201) or min(pos) >= T:  # close every stream at its prefix so far
+            for s in range(S):
+                got = f.candidates(s).cpu().numpy().astype(np.uint32)
+                assert np.array_equal(got, o.candidates(want[s][2][:pos[s]], 4)), f"stream {s} at {pos[s]}"
     torch.cuda.synchronize()
     f.status()
     ks, ss = keep.cpu().numpy(), scores.cpu().numpy()

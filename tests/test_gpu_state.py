@@ -97,7 +97,22 @@ def test_shards_prepared_independently_and_chained(cuts, l_max):
     assert np.array_equal(keep, ko)
     assert np.all(np.abs(score - so) <= 1e-6 * so)
     # the last shard's handle is left exactly as a single pass would leave it
+    # (header, gap and ring); each shard's retention record holds its own
+    # retained frames, and together they are the single pass's record
     single = NGFF(spec.width, spec.height, tau=tau, l_max=l_max)
     single.push(dev)
     torch.cuda.synchronize()
-    assert torch.equal(handles[shards[-1][0]].state_save(), single.state_save())
+    one = single.state_save().numpy()
+    ring_end = 64 + l_max * 32 * 4
+    assert np.array_equal(handles[shards[-1][0]].state_save().numpy()[:ring_end], one[:ring_end])
+    record = (lambda st: np.unpackbits(st[ring_end:], bitorder="little"))
+    union = np.zeros_like(record(one))
+    for a, b in shards:
+        r = record(handles[a].state_save().numpy())
+        assert np.array_equal(np.flatnonzero(r), a + np.flatnonzero(ko[a:b])), f"shard [{a}, {b})"
+        union |= r
+    assert np.array_equal(union, record(one))
+    assert np.array_equal(np.flatnonzero(record(one)), np.flatnonzero(ko))
+    # the sharded stream closed from its shards' keep codes
+    idx = handles[shards[-1][0]].candidates_from_keep(torch.cat([k for _, k in outs]))
+    assert np.array_equal(idx.cpu().numpy().astype(np.uint32), O.load().candidates(ko, 4))

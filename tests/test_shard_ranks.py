@@ -1,9 +1,11 @@
-"""The multi-rank exchange of one sharded stream on CPU (gloo ranks): each
-rank prepares its shard's gap map from its frames and halo, the maps are
-all-gathered, each rank resolves its entry gap and decides its frames. The
-per-shard decisions here come from the oracle's fp32 distances (the GPU
-shard kernels have their own parity tests); the concatenation over ranks must
-equal the oracle's single pass."""
+"""The multi-rank exchange of one sharded stream (gloo ranks): each rank holds
+only its shard and a halo of min(a, L_max) frames before it, prepares its
+shard's gap map, the maps are all-gathered, each rank resolves its entry gap
+and decides its frames. On CPU the per-shard decisions come from the oracle's
+fp32 distances on the rank's own frames (a stand-in for the library); where a
+GPU is present each rank runs the library's own cofie_ngff_shard_prepare and
+_commit through shards.sharded_push, every rank on its own handle. The
+concatenation over ranks must equal the oracle's single pass."""
 import os
 import socket
 
@@ -21,18 +23,22 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def _stream():
+def _spec():
+    import synth
+    return synth.medium(seed=4242).with_(width=W, height=H, frames=T, mean_scene_len=5)
+
+
+def _single_pass():
     import oracle as O
     import synth
-    fr = synth.generate(synth.medium(seed=4242).with_(width=W, height=H, frames=T, mean_scene_len=5))
-    p = O.Params(W, H, tau=TAU, l_max=L)
-    hist, _, keep = O.load().run(fr, p)
-    return hist, keep
+    _, _, keep = O.load().run(synth.generate(_spec()), O.Params(W, H, tau=TAU, l_max=L))
+    return keep
 
 
-def _decide_from(hist, t0, n, g_entry):
+def _decide_from(hist, lo, t0, n, g_entry):
     """Frames [t0, t0 + n) entered with gap g_entry (the last keep before t0
-    was frame t0 - g_entry); returns (keep codes, gap after the last frame)."""
+    was frame t0 - g_entry), from the histograms of frames [lo, t0 + n) only
+    (hist[i] is frame lo + i); returns (keep codes, gap after the last frame)."""
     import oracle as O
     o = O.load()
     r = t0 - g_entry
@@ -41,7 +47,7 @@ def _decide_from(hist, t0, n, g_entry):
         if t == 0:
             code = O.KEEP_FIRST
         else:
-            d = max(o.tv32(hist[t], hist[t - 1], W * H), o.tv32(hist[t], hist[max(r, 0)], W * H))
+            d = max(o.tv32(hist[t - lo], hist[t - 1 - lo], W * H), o.tv32(hist[t - lo], hist[max(r, 0) - lo], W * H))
             code = O.KEEP_NOVELTY if np.float32(d) >= np.float32(TAU) else (O.KEEP_GAP if t - r >= L else O.KEEP_DROP)
         if code:
             r = t
@@ -49,41 +55,78 @@ def _decide_from(hist, t0, n, g_entry):
     return codes, t0 + n - r
 
 
-def _rank(rank, world, port, q):
+def _rank(rank, world, port, q, on_gpu):
     import torch.distributed as dist
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world)
+    import oracle as O
+    import synth
     from paper_2609_03675_gb300 import shards
-    hist, _ = _stream()
     a, b, halo = shards.shard_bounds(T, world, rank, L)
     assert halo == min(a, L)
-    local = hist[: b]  # this rank reads only frames [a - halo, b) below
+    lo, hi = shards.shard_frames(T, world, rank, L)
+    local = synth.generate(_spec(), lo, hi)  # this rank's frames only: the halo, then the shard
+    if on_gpu:
+        from paper_2609_03675_gb300 import NGFF
+        torch.cuda.set_device(0)
+        f = NGFF(W, H, tau=TAU, l_max=L)
+        _, keep = shards.sharded_push(f, torch.from_numpy(local).cuda(), T, rank, world)
+        torch.cuda.synchronize()
+        f.status()
+        codes = keep.cpu().tolist()
+        f.close()
+    else:
+        hist = O.load().run(local, O.Params(W, H, tau=TAU, l_max=L))[0]
 
-    def prepare():
-        return torch.tensor([_decide_from(local, a, b - a, g)[1] for g in range(1, L + 1)], dtype=torch.int32)
+        def prepare():
+            return torch.tensor([_decide_from(hist, lo, a, b - a, g)[1] for g in range(1, L + 1)], dtype=torch.int32)
 
-    codes = shards.sharded_decide(prepare, lambda g: _decide_from(local, a, b - a, g)[0], rank, world)
+        codes = shards.sharded_decide(prepare, lambda g: _decide_from(hist, lo, a, b - a, g)[0], rank, world)
     q.put((rank, codes))
     dist.barrier()
     dist.destroy_process_group()
 
 
-@pytest.mark.parametrize("world", [2, 3])
-def test_sharded_stream_over_gloo_ranks(world):
+def _run_ranks(world, on_gpu):
     ctx = mp.get_context("spawn")
     q = ctx.Queue()
     port = _free_port()
-    procs = [ctx.Process(target=_rank, args=(r, world, port, q)) for r in range(world)]
+    procs = [ctx.Process(target=_rank, args=(r, world, port, q, on_gpu)) for r in range(world)]
     for p in procs:
         p.start()
-    out = dict(q.get(timeout=180) for _ in procs)
+    out = dict(q.get(timeout=300) for _ in procs)
     for p in procs:
         p.join(timeout=120)
         assert p.exitcode == 0
     got = np.concatenate([out[r] for r in range(world)]).astype(np.uint8)
-    _, keep = _stream()
+    keep = _single_pass()
     assert np.array_equal(got, keep)
     assert (keep == 2).any() and (keep == 1).any(), "the stream exercises both rules"
+
+
+@pytest.mark.parametrize("world", [2, 3])
+def test_sharded_stream_over_gloo_ranks(world):
+    _run_ranks(world, on_gpu=False)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("world", [2, 3])
+def test_sharded_stream_over_gloo_ranks_on_the_library(world):
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    _run_ranks(world, on_gpu=True)
+
+
+def test_shard_frames_are_the_halo_and_the_shard():
+    from paper_2609_03675_gb300 import shards
+    for world in (1, 2, 3, 5):
+        covered = []
+        for r in range(world):
+            a, b, halo = shards.shard_bounds(T, world, r, L)
+            lo, hi = shards.shard_frames(T, world, r, L)
+            assert (lo, hi) == (a - halo, b) and hi - lo <= b - a + L
+            covered += list(range(a, b))
+        assert covered == list(range(T))
 
 
 def test_entry_gaps_compose_in_order():
