@@ -47,7 +47,7 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards",
-                                           "signals", "pipeline"],
+                                           "signals", "pipeline", "tiny", "static"],
                     default="hd1080",
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
@@ -1320,6 +1320,49 @@ def bench_signals(args):
     print(json.dumps(out), flush=True)
 
 
+def bench_static(args):
+    """cofie_ngff_select_static (the allocation-free selection, one CTA) at
+    the largest sizes its static array admits and at a typical one: CUDA
+    events around repeated calls on histograms already on the device."""
+    import ctypes
+
+    import numpy as np
+    import torch
+
+    from paper_2609_03675_gb300 import _abi
+    lib = _abi.load()
+    st = torch.cuda.current_stream().cuda_stream
+    out = {"workload": "cofie_ngff_select_static: decisions of a fresh stream from its histograms, one CTA",
+           "cases": []}
+    g = np.random.default_rng(7)
+    for n, bins, l_max in ((3600, 32, 30), (33825, 32, 30), (3970, 256, 256)):
+        hist = torch.from_numpy(g.integers(0, 4096, size=(n, bins), dtype=np.int32)).cuda()
+        s = torch.empty(n, dtype=torch.float32, device="cuda")
+        k = torch.empty(n, dtype=torch.uint8, device="cuda")
+        p = _abi.Params()
+        lib.cofie_ngff_default_params(ctypes.byref(p), 1920, 1080)
+        p.bins, p.l_max, p.tau = bins, l_max, 0.3
+        err = ctypes.create_string_buffer(256)
+
+        def call():
+            rc = lib.cofie_ngff_select_static(ctypes.byref(p), hist.data_ptr(), n, s.data_ptr(), k.data_ptr(), err,
+                                              len(err), st)
+            assert rc == 0, err.value
+
+        for _ in range(3):
+            call()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 10
+        e0.record()
+        for _ in range(reps):
+            call()
+        e1.record()
+        torch.cuda.synchronize()
+        out["cases"].append({"frames": n, "bins": bins, "l_max": l_max, "ms_per_call": e0.elapsed_time(e1) / reps,
+                             "scratch_words": n * (l_max + (l_max + 31) // 32)})
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
@@ -1340,6 +1383,10 @@ def main():
         bench_shards(args)
     elif args.workload == "signals":
         bench_signals(args)
+    elif args.workload == "tiny":
+        print(json.dumps(tiny_figures(args)), flush=True)
+    elif args.workload == "static":
+        bench_static(args)
     else:
         bench_gb300(args)
 
