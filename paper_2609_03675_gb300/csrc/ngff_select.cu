@@ -28,9 +28,10 @@
 // kernel: the same CTA first computes its stream's distances, then scans.
 // With at most kWalkMaxFrames frames per stream and L_max <= kWalkMaxLmax the
 // push is smaller still and a lighter kernel decides it (select_walk_kernel):
-// one 128-thread CTA per stream keeps the distances and keep bits in shared
-// memory and walks the rule in frame order from the stream's gap, which for
-// so few frames is shorter than composing gap maps.
+// one 256-thread CTA per stream stages the stream's ring and the push's rows
+// in shared memory, keeps the distances and keep bits there, and walks the
+// rule in frame order from the stream's gap, which for so few frames is
+// shorter than composing gap maps.
 #include "ngff_common.cuh"
 
 namespace cofie {
@@ -41,9 +42,10 @@ constexpr int kScanThreads = 1024;
 constexpr int kScanWarps = kScanThreads / 32;
 constexpr uint32_t kScanTile = 4096;  // frames per shared-memory tile
 constexpr uint32_t kSmallMax = 64;    // frames per stream segment for the fused small-push kernel
-constexpr int kWalkThreads = 128;
+constexpr int kWalkThreads = 256;
 constexpr uint32_t kWalkMaxFrames = 64;
 constexpr uint32_t kWalkMaxLmax = 64;
+constexpr size_t kWalkStageBudget = 48 * 1024;  // shared memory a walk CTA takes without opting in
 
 __device__ __forceinline__ uint32_t absdiff(uint32_t a, uint32_t b) { return a > b ? a - b : b - a; }
 
@@ -381,13 +383,18 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
   scan_segment<kOneWord>(sseg, s_t0, s_g, s_acc, a, l1, mask, hist, ring, state, ssm, entry);
 }
 
-// Small pushes, one 128-thread CTA per stream segment (n <= kWalkMaxFrames,
+// Small pushes, one 256-thread CTA per stream segment (n <= kWalkMaxFrames,
 // L_max <= kWalkMaxLmax), in the order the rule states it:
+//   0. (kStaged) the stream's ring of the last L_max rows and the push's own
+//      rows are copied into shared memory in one coalesced pass, alongside
+//      the read of the stream's state, so that everything after it reads
+//      shared memory only;
 //   1. windowed distances, a warp per frame, lane = lag k (the Eq. 2
-//      numerators L1[j][k-1] = sum_b |c_t - c_{t-k}|, from the push's rows or
-//      the stream's ring), and the keep bit of every possible gap g (Eqs. 3-5:
-//      fp32(max(L1[j][0], L1[j][g-1])) / fp32(2N) >= tau_h, or g >= L_max),
-//      into shared memory;
+//      numerators L1[j][k-1] = sum_b |c_t - c_{t-k}|), each lane starting at
+//      a column rotated by its lane so a warp's 16-byte reads of different
+//      rows fall in different banks, and the keep bit of every possible gap g
+//      (Eqs. 3-5: fp32(max(L1[j][0], L1[j][g-1])) / fp32(2N) >= tau_h, or
+//      g >= L_max), into shared memory;
 //   2. one thread walks the frames in order from the stream's gap: frame j is
 //      kept when its bit for the current gap is set (or, with scene changes,
 //      when twin comparison of the adjacent differences finds one, with the
@@ -396,7 +403,9 @@ __global__ void __launch_bounds__(kScanThreads) select_small_kernel(SegTable seg
 //   3. all threads emit scores and keep codes, note retained frames in the
 //      stream's retention record, store the last L_max rows in the ring,
 //      update the stream state and zero the push's rows for the next push.
-template <bool kVec4>
+// Without kStaged (rows too wide for the staging budget) the same steps read
+// the rows from global memory.
+template <bool kVec4, bool kStaged>
 __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs, SelectArgs a,
                                                                    uint32_t* __restrict__ hist,
                                                                    uint32_t* __restrict__ ring,
@@ -412,36 +421,55 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
   const uint32_t n = sg.n, row0 = sg.row0, stream = sg.stream;
   const uint32_t B = a.bins, L = a.l_max, W = a.mask_words;
   if (n == 0) return;
-  uint32_t* sl1 = wsm;               // [n][L]
-  uint32_t* smask = sl1 + n * L;     // [n][W]
-  uint32_t* sgap = smask + n * W;    // [n]: gap, bit 31 a scene change
+  uint32_t* srows = wsm;                                   // kStaged: [L + n][B], ring slots then the push
+  uint32_t* sl1 = wsm + (kStaged ? (L + n) * B : 0u);      // [n][L]
+  uint32_t* smask = sl1 + n * L;                           // [n][W]
+  uint32_t* sgap = smask + n * W;                          // [n]: gap, bit 31 a scene change
+  const uint32_t* ring_s = ring + static_cast<uint64_t>(stream) * L * B;
+  const uint32_t* hist_s = hist + static_cast<uint64_t>(row0) * B;
   if (tid == 0) {
     s_t0 = state[stream].t;
     s_acc = state[stream].acc;
     s_g = state[stream].g;
   }
+  if (kStaged) {
+    if (kVec4) {
+      const uint32_t rq = L * B / 4, hq = n * B / 4;
+      for (uint32_t i = tid; i < rq + hq; i += kWalkThreads)
+        reinterpret_cast<uint4*>(srows)[i] =
+            i < rq ? reinterpret_cast<const uint4*>(ring_s)[i] : reinterpret_cast<const uint4*>(hist_s)[i - rq];
+    } else {
+      for (uint32_t i = tid; i < (L + n) * B; i += kWalkThreads)
+        srows[i] = i < L * B ? ring_s[i] : hist_s[i - L * B];
+    }
+  }
   __syncthreads();
   const unsigned long long t0 = s_t0;
-  const uint32_t* ring_s = ring + static_cast<uint64_t>(stream) * L * B;
+  const uint32_t nq = B / 4, rot = kStaged && kVec4 ? lane % max(nq, 1u) : 0u;
 
   // 1. distances and keep bits
   for (uint32_t j = warp; j < n; j += kWarps) {
     const unsigned long long t = t0 + j;
-    const uint32_t* ct = hist + static_cast<uint64_t>(row0 + j) * B;
+    const uint32_t* ct = kStaged ? srows + (L + j) * B : hist_s + static_cast<uint64_t>(j) * B;
     uint32_t l_adj = 0;
     for (uint32_t w = 0; w < W; ++w) {
       const uint32_t k = 32 * w + lane + 1;
       const bool valid = k <= L && k <= t;
       const uint32_t* src = ct;
-      if (valid) src = k <= j ? ct - static_cast<uint64_t>(k) * B : ring_s + ((t - k) % L) * B;
+      if (valid) {
+        if (k <= j) src = ct - static_cast<uint64_t>(k) * B;
+        else src = (kStaged ? srows : ring_s) + ((t - k) % L) * B;  // ring slot of frame t - k
+      }
       uint32_t d = 0;
       if (kVec4) {
         const uint4* c4 = reinterpret_cast<const uint4*>(ct);
         const uint4* s4 = reinterpret_cast<const uint4*>(src);
+        uint32_t q = rot;
 #pragma unroll 8
-        for (uint32_t q = 0; q < B / 4; ++q) {
+        for (uint32_t i = 0; i < nq; ++i) {
           const uint4 x = c4[q], y = s4[q];
           d += absdiff(x.x, y.x) + absdiff(x.y, y.y) + absdiff(x.z, y.z) + absdiff(x.w, y.w);
+          if (++q == nq) q = 0;
         }
       } else if (a.dist_kind == 1) {  // Hamming distance of bit vectors (dHash)
         for (uint32_t b = 0; b < B; ++b) d += __popc(ct[b] ^ src[b]);
@@ -519,7 +547,7 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
   uint32_t* ring_w = ring + static_cast<uint64_t>(stream) * L * B;
   for (uint32_t i = tid; i < keep_n * B; i += kWalkThreads) {
     const uint32_t jj = n - keep_n + i / B, b = i % B;
-    ring_w[((t0 + jj) % L) * B + b] = hist[static_cast<uint64_t>(row0 + jj) * B + b];
+    ring_w[((t0 + jj) % L) * B + b] = kStaged ? srows[(L + jj) * B + b] : hist_s[static_cast<uint64_t>(jj) * B + b];
   }
   if (tid == 0) {
     state[stream].t = t0 + n;
@@ -527,13 +555,13 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
     state[stream].acc = s_acc;
   }
   if (a.zero_hist) {
-    __syncthreads();  // the ring copies above have read the rows
+    if (!kStaged) __syncthreads();  // the ring copies above have read the rows
     for (uint32_t i = tid; i < n * B; i += kWalkThreads) hist[static_cast<uint64_t>(row0) * B + i] = 0;
   }
 }
 
-size_t walk_smem_bytes(uint32_t n, uint32_t l_max, uint32_t mask_words) {
-  return static_cast<size_t>(n) * (l_max + mask_words + 1) * 4;
+size_t walk_smem_bytes(uint32_t n, uint32_t l_max, uint32_t mask_words, uint32_t bins, bool staged) {
+  return (static_cast<size_t>(n) * (l_max + mask_words + 1) + (staged ? static_cast<size_t>(l_max + n) * bins : 0)) * 4;
 }
 
 // The gap map of one stream segment: map[g-1] = the gap after its last frame
@@ -607,13 +635,14 @@ cudaError_t launch_select_walk(const SegTable& segs, const SelectArgs& a, uint32
                                StreamState* state, cudaStream_t st, bool pdl) {
   uint32_t longest = 0;
   for (uint32_t i = 0; i < segs.count; ++i) longest = max(longest, segs.s[i].n);
-  const size_t smem = walk_smem_bytes(longest, a.l_max, a.mask_words);  // <= 17,152 bytes
+  // rows staged in shared memory when they fit the default 48 KiB with the tables
+  const bool staged = walk_smem_bytes(longest, a.l_max, a.mask_words, a.bins, true) <= kWalkStageBudget;
+  const size_t smem = walk_smem_bytes(longest, a.l_max, a.mask_words, a.bins, staged);  // <= 48 KiB
+  const bool vec = a.bins % 4 == 0 && a.dist_kind == 0;
+  const auto kernel = vec ? (staged ? select_walk_kernel<true, true> : select_walk_kernel<true, false>)
+                          : (staged ? select_walk_kernel<false, true> : select_walk_kernel<false, false>);
   const cudaError_t e =
-      (a.bins % 4 == 0 && a.dist_kind == 0)
-          ? launch_dependent(pdl, select_walk_kernel<true>, dim3(segs.count), dim3(kWalkThreads), smem, st, segs, a,
-                             hist, ring, state)
-          : launch_dependent(pdl, select_walk_kernel<false>, dim3(segs.count), dim3(kWalkThreads), smem, st, segs, a,
-                             hist, ring, state);
+      launch_dependent(pdl, kernel, dim3(segs.count), dim3(kWalkThreads), smem, st, segs, a, hist, ring, state);
   return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
