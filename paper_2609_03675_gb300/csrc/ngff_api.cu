@@ -609,7 +609,7 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   h->size_fast = (h->npix % 16) == 0;
   h->seen.assign(p->max_streams, 0);
   const uint32_t rec_frames = p->max_stream_frames ? p->max_stream_frames : kDefaultRecordFrames;
-  h->rec_words = (rec_frames + 31) / 32;
+  h->rec_words = static_cast<uint32_t>((static_cast<uint64_t>(rec_frames) + 31) / 32);
   h->p.max_stream_frames = rec_frames;
 
   LumaConsts& lc = h->lc;

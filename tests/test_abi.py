@@ -36,7 +36,8 @@ def test_exports_every_declared_symbol(lib):
 
 def test_param_struct_layout_matches_header(lib):
     from paper_2609_03675_gb300 import _abi
-    # width..luma_den: 10 x 4 bytes, max_streams, max_frames_per_push, device, pad, u64, signal, reserved
+    # width..luma_den: 10 x 4 bytes, max_streams, max_frames_per_push, device, pad, u64, signal, scd_cut,
+    # scd_gradual, max_stream_frames
     assert ctypes.sizeof(_abi.Params) == 80
     assert ctypes.sizeof(_abi.PushDesc) == 32
 
@@ -50,6 +51,7 @@ def test_defaults_are_the_papers(lib):
     assert (p.bins, p.m_min, p.l_max) == (d["bins"]["value"], d["m_min"]["value"], d["l_max"]["value"])
     assert abs(p.tau - d["tau_h"]["value"]) < 1e-7
     assert list(p.luma_w) == [299, 587, 114] and p.luma_den == 1000
+    assert p.max_stream_frames == 1 << 20  # the retention record's default reach (not from the paper)
 
 
 @pytest.mark.parametrize("field,value,msg", [
@@ -74,6 +76,10 @@ def test_null_handle_calls_are_rejected(lib):
     assert lib.cofie_ngff_push(None, 0, None, 0, None, None, None) == _abi.EINVAL
     assert lib.cofie_ngff_reset(None, 0, None) == _abi.EINVAL
     assert lib.cofie_ngff_status(None, None) == _abi.EINVAL
+    m = ctypes.c_uint32(7)
+    assert lib.cofie_ngff_candidates(None, 0, None, 0, ctypes.addressof(m), None) == _abi.EINVAL
+    assert lib.cofie_ngff_candidates_from_keep(None, None, 0, None, ctypes.addressof(m), None) == _abi.EINVAL
+    assert m.value == 7
     assert lib.cofie_ngff_last_error(None) == b""
     lib.cofie_ngff_destroy(None)
 
