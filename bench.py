@@ -573,7 +573,7 @@ def bench_gb300(args):
                          "select_ms_per_step": prof["select_ms"] / max(prof["select_timed"], 1)},
             "e2e": e2e,
             "cpu_baseline": cpu,
-            "gpu_launches": int(prof["hist_launches"] + prof["select_launches"]),
+            "gpu_launches": int(prof["hist_launches"] + prof["select_launches"] + prof["other_launches"]),
             "clocks": clocks,
             "kept_frames_last_step": kept,
             "parity": parity,
