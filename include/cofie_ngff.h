@@ -132,10 +132,10 @@ typedef struct cofie_ngff cofie_ngff_t;
  *                     the twin-comparison thresholds T_b, T_s of the scene
  *                     change signal (non-NaN); defaults 0.30f and 0.10f.
  *   max_stream_frames frames per stream that the retention record covers
- *                     (cofie_ngff_candidates); 0 picks the default, 1048576
- *                     (9.7 h at 30 frames/s). The record takes
- *                     ceil(max_stream_frames / 32) * 4 bytes of device memory
- *                     per stream (128 KiB at the default).
+ *                     (cofie_ngff_candidates), rounded up to a multiple of 32;
+ *                     0 picks the default, 1048576 (9.7 h at 30 frames/s). The
+ *                     record takes ceil(max_stream_frames / 32) * 4 bytes of
+ *                     device memory per stream (128 KiB at the default).
  */
 typedef struct {
   uint32_t width, height;

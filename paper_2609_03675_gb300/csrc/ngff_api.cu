@@ -610,7 +610,8 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
   h->seen.assign(p->max_streams, 0);
   const uint32_t rec_frames = p->max_stream_frames ? p->max_stream_frames : kDefaultRecordFrames;
   h->rec_words = static_cast<uint32_t>((static_cast<uint64_t>(rec_frames) + 31) / 32);
-  h->p.max_stream_frames = rec_frames;
+  // the record holds whole words: it covers rec_frames rounded up to a multiple of 32
+  h->p.max_stream_frames = static_cast<uint32_t>(std::min<uint64_t>(32ull * h->rec_words, 0xffffffffull));
 
   LumaConsts& lc = h->lc;
   const uint32_t wr = p->luma_w[0], wg = p->luma_w[1], wb = p->luma_w[2], den = p->luma_den;
