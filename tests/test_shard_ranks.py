@@ -102,6 +102,13 @@ def _run_ranks(world, on_gpu):
     keep = _single_pass()
     assert np.array_equal(got, keep)
     assert (keep == 2).any() and (keep == 1).any(), "the stream exercises both rules"
+    if on_gpu:  # the sharded stream closed from its shards' keep codes
+        import oracle as O
+        from paper_2609_03675_gb300 import NGFF
+        f = NGFF(W, H, tau=TAU, l_max=L)
+        idx = f.candidates_from_keep(torch.from_numpy(got).cuda()).cpu().numpy().astype(np.uint32)
+        assert np.array_equal(idx, O.load().candidates(keep, 4))
+        f.close()
 
 
 @pytest.mark.parametrize("world", [2, 3])
