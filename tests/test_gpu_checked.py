@@ -1,7 +1,8 @@
 """The checked build (kernels compiled with -DCOFIE_DEBUG_CHECKS=1, which
 check every computed index against their launch arguments and report a
 failed check through cofie_ngff_status) run over representative workloads:
-the fast and generic histogram kernels, one- and two-word gap masks, the
+the fast and generic histogram kernels (odd sizes, an odd byte offset), the
+small-push walk kernel on staged and unstaged rows, one- and two-word gap masks, the
 spatial signals on both of their kernels, scene changes across scan tiles,
 the frame-order walk (L_max = 0), batches, shards, candidates and gather,
 and QER on both scoring kernels.
@@ -69,6 +70,19 @@ for (w, h) in ((64, 48), (37, 23)):
             sg, kg = run(f, fr, chunks)
             same(sg, kg, so, ko, f"hist {w}x{h} B{bins} L{l_max} {chunks[:2]}")
             n += 1
+# frames at an odd byte offset (the generic kernel on a pixel count the fast kernel takes), and the
+# walk kernel reading 256-bin rows from global memory (too wide to stage) for pushes of 20 frames
+fr = frames(64, 48, 120, seed=690)
+raw = torch.empty(fr.nbytes + 64, dtype=torch.uint8, device="cuda")
+raw[3:3 + fr.nbytes].copy_(torch.from_numpy(fr.reshape(-1)))
+_, so, ko = O.load().run(fr, O.Params(64, 48, tau=0.05, l_max=30))
+f = NGFF(64, 48, tau=0.05, l_max=30)
+s1, k1 = f.push(raw[3:3 + fr.nbytes].view(fr.shape))
+torch.cuda.synchronize(); f.status()
+same(s1.cpu().numpy().astype(np.float64), k1.cpu().numpy(), so, ko, "generic kernel, offset 3"); n += 1
+_, so, ko = O.load().run(fr, O.Params(64, 48, bins=256, tau=0.05, l_max=64))
+f = NGFF(64, 48, bins=256, tau=0.05, l_max=64)
+same(*run(f, fr, [20] * 6), so, ko, "walk on unstaged 256-bin rows"); n += 1
 # spatial signals: streaming cell kernel (64x48) and per-frame kernel (72x40)
 for (w, h) in ((64, 48), (72, 40)):
     fr = frames(w, h, 200, seed=640 + w)
@@ -177,4 +191,4 @@ def test_checked_build_runs_clean_and_matches_the_oracle():
                   build_dir=os.path.join(d, "obj"))
     r = subprocess.run([sys.executable, "-c", CHILD, lib, REPO], capture_output=True, text=True, timeout=900)
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-4000:]
-    assert "checked workloads 25" in r.stdout, r.stdout[-2000:]
+    assert "checked workloads 27" in r.stdout, r.stdout[-2000:]
