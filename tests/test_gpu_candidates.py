@@ -244,3 +244,31 @@ def test_stream_past_its_record():
     assert np.array_equal(f.candidates(0).cpu().numpy().astype(np.uint32), O.load().candidates(ko[:10], 4))
     f.status()
     f.close()
+
+
+@pytest.mark.parametrize("m_min", [4, 5000])
+def test_long_stream_crosses_record_tiles(m_min):
+    """40,000 frames (the record is compacted 32,768 frames per pass of the
+    closing kernel) closed at prefixes on both sides of a pass boundary, with
+    a small M_min and with one larger than the retained set (the uniform fill
+    over many record words)."""
+    from paper_2609_03675_gb300 import NGFF
+    T = 40_000
+    spec = synth.medium(seed=81).with_(width=16, height=16, frames=T, mean_scene_len=30)
+    fr = synth.generate(spec)
+    o = O.load()
+    _, _, ko = o.run(fr, O.Params(16, 16, tau=0.35, l_max=45))
+    f = NGFF(16, 16, tau=0.35, l_max=45, m_min=m_min, max_frames_per_push=4096)
+    dev = torch.from_numpy(fr).cuda()
+    pos = 0
+    for close in (32_767, 32_768, 32_769, 40_000):
+        while pos < close:
+            n = min(4096, close - pos)
+            f.push(dev[pos:pos + n])
+            pos += n
+        got = f.candidates(0).cpu().numpy().astype(np.uint32)
+        want = o.candidates(ko[:close], m_min)
+        assert np.array_equal(got, want), f"T={close} M_min={m_min}"
+    f.status()
+    assert (ko != 0).sum() < 5000, "the fill case must exercise the uniform frames"
+    f.close()
