@@ -829,6 +829,33 @@ def medium_figures(args):
         glat.append((time.perf_counter() - c0) * 1e3)
     f.status()
     prof = f.profile_read()
+    # end to end: the same pushes from pinned host frames, scores and keep
+    # codes to pinned host memory, one synchronise at the end (and per push
+    # for the latency), through the same C entry point
+    host = torch.from_numpy(frames_np).pin_memory()
+    hs = torch.empty(spec.frames, dtype=torch.float32, pin_memory=True)
+    hk = torch.empty(spec.frames, dtype=torch.uint8, pin_memory=True)
+    hptrs = [(host.data_ptr() + i * fb, hs.data_ptr() + 4 * i, hk.data_ptr() + i) for i in range(0, spec.frames, 8)]
+
+    def run_host(sync_each):
+        f.reset()
+        lat = []
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for fp, sp, kp in hptrs:
+            c0 = time.perf_counter()
+            f.push_raw(0, fp, 8, sp, kp, None, st)
+            if sync_each:
+                torch.cuda.synchronize()
+                lat.append((time.perf_counter() - c0) * 1e3)
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0, lat
+
+    run_host(False)
+    el_host, _ = run_host(False)
+    _, hlat = run_host(True)
+    f.status()
+    assert torch.equal(hk, keep.cpu()), "end-to-end keep codes differ from the device-resident run"
     f.close()
     return {"workload": "medium: 600 uint8 RGB frames of 448x448 pushed in chunks of 8, B=32, L_max=30, tau_h=0.30",
             "pushes": len(lat), "pipelined_frames_per_s": spec.frames / el_pipe,
@@ -837,6 +864,9 @@ def medium_figures(args):
             "graph_latency_ms_p50": _pct(glat, 50), "graph_latency_ms_p99": _pct(glat, 99),
             "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99),
             "latency": "host wall time of one push plus a device synchronise",
+            "e2e": {"frames_per_s": spec.frames / el_host, "latency_ms_p50": _pct(hlat, 50),
+                    "latency_ms_p99": _pct(hlat, 99), "h2d_bytes_per_push": 8 * fb, "d2h_bytes_per_push": 8 * 5,
+                    "how": "pinned host frames in, pinned host scores and keep codes out, through the same call"},
             "kernels_per_push": (prof["hist_launches"] + prof["select_launches"]) / max(1, prof["hist_launches"]),
             "kept": int((keep != 0).sum().item()), "parity": par}
 
@@ -862,6 +892,22 @@ def rare_event_figures(args):
     dev = host.cuda()
     o = O.load()
     hist_o = o.histograms_parallel(host.data_ptr(), spec.frames, O.Params(spec.width, spec.height))
+    # end to end at tau_h = 0.30: the whole stream from pinned host memory, outputs to pinned host memory
+    fe = NGFF(spec.width, spec.height)
+    hs = torch.empty(spec.frames, dtype=torch.float32, pin_memory=True)
+    hk = torch.empty(spec.frames, dtype=torch.uint8, pin_memory=True)
+    e2e_s = []
+    for i in range(4):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        fe.reset()
+        fe.push(host, scores=hs, keep=hk)
+        torch.cuda.synchronize()
+        if i:
+            e2e_s.append(time.perf_counter() - t0)
+    fe.status()
+    fe.close()
+    hk_e2e = hk.clone()
     del host
     events = torch.from_numpy(synth.event_mask(spec).astype(bool)).cuda()
     starts = synth.event_mask(spec)
@@ -892,6 +938,8 @@ def rare_event_figures(args):
         caught = sum(1 for a, b in runs if kc[a:b].any())
         so, ko = o.select(hist_o, O.Params(spec.width, spec.height, tau=tau))
         par = parity_block(tau, scores.cpu().numpy(), keep.cpu().numpy(), so, ko)
+        if tau == 0.30:
+            keep30 = keep.cpu().numpy()
         out["taus"][str(tau)] = {"frames_per_s": 20 * spec.frames / (e0.elapsed_time(e1) / 1e3),
                                  "keep_ratio": float(kept.float().mean().item()),
                                  "event_frame_recall": float(kept[events].float().mean().item()),
@@ -901,6 +949,11 @@ def rare_event_figures(args):
                                             "band_frames": par["band_frames"]}}
         f.close()
     t30 = out["taus"]["0.3"]
+    el = statistics.median(e2e_s)
+    out["e2e"] = {"frames_per_s": spec.frames / el, "ms_per_push": el * 1e3,
+                  "h2d_bytes_per_push": spec.frames * spec.frame_bytes, "d2h_bytes_per_push": spec.frames * 5,
+                  "statistic": "median of 3 whole-stream pushes at tau_h 0.30",
+                  "keep_equal_device_run": bool(np.array_equal(hk_e2e.numpy(), keep30))}
     out["frames_per_s"] = t30["frames_per_s"]
     out["pixel_gbs"] = t30["frames_per_s"] * spec.frame_bytes / 1e9
     out["events"] = len(_event_runs(starts.astype(bool)))
