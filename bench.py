@@ -1374,7 +1374,7 @@ def bench_signals(args):
 
 
 def bench_static(args):
-    """cofie_ngff_select_static (the allocation-free selection, one CTA) at
+    """cofie_ngff_select_static (the allocation-free selection) at
     the largest sizes its static array admits and at a typical one: CUDA
     events around repeated calls on histograms already on the device."""
     import ctypes
@@ -1385,7 +1385,8 @@ def bench_static(args):
     from paper_2609_03675_gb300 import _abi
     lib = _abi.load()
     st = torch.cuda.current_stream().cuda_stream
-    out = {"workload": "cofie_ngff_select_static: decisions of a fresh stream from its histograms, one CTA",
+    out = {"workload": "cofie_ngff_select_static: decisions of a fresh stream from its histograms (a grid of "
+                       "distance warps, then one scan CTA)",
            "cases": []}
     g = np.random.default_rng(7)
     for n, bins, l_max in ((3600, 32, 30), (33825, 32, 30), (3970, 256, 256)):

@@ -439,8 +439,9 @@ int cofie_ngff_profile_read(cofie_ngff_t* h, cofie_ngff_profile* out);
  * stream of the histogram signal (no scene changes). Needs no handle and
  * allocates nothing: its working tables live in a static device array of
  * 1048576 32-bit words (4 MiB) that every GPU loading the library holds until
- * the process exits. One CTA does the work: at the largest n it takes
- * milliseconds, not microseconds.
+ * the process exits. Two launches on cuda_stream: a grid computes every
+ * frame's windowed distances, then one CTA scans them (0.22 ms at the
+ * largest n for L_max = 30 on GB300).
  *   p           width, height, bins, l_max and tau are used; signal must be
  *               COFIE_SIGNAL_HISTOGRAM (else COFIE_EINVAL); the rest is ignored.
  *   hist        n * bins uint32 counts, row-major, device memory on the

@@ -11,13 +11,13 @@
 // live in a file-scope static device array of a fixed size, so the call
 // allocates nothing.
 //
-// It is a variant of the library's scan kernel: one 1024-thread CTA first
-// writes the windowed L1 distances and the per-gap keep bits of every frame
-// into the static array (the work the window kernel does: a warp per frame,
-// lane = lag, 16-byte loads when the rows allow them), then runs the same
-// gap-map scan over them. Decisions and scores equal those of
-// cofie_ngff_push_ex on a fresh stream of the histogram signal without scene
-// changes (other signals are refused).
+// It is a variant of the library's window and scan kernels: a grid of warps
+// (one per frame, lane = lag, 16-byte loads when the rows allow them) writes
+// the windowed L1 distances and the per-gap keep bits of every frame into the
+// static array, then one 1024-thread CTA runs the same gap-map scan over
+// them. Decisions and scores equal those of cofie_ngff_push_ex on a fresh
+// stream of the histogram signal without scene changes (other signals are
+// refused).
 //
 // The array holds kStaticScratchWords 32-bit words (4 MiB) on every GPU that
 // loads the library, until the process exits. Every call shares it and it
@@ -47,22 +47,20 @@ __device__ __forceinline__ uint32_t next_gap(const uint32_t* m, uint32_t g) {
   return ((m[(g - 1) >> 5] >> ((g - 1) & 31)) & 1u) ? 1u : g + 1u;
 }
 
+constexpr int kWinThreads = 256;  // the distance kernel: 8 frames per CTA
+
+// Phase 1: windowed distances and per-gap keep bits of every frame (warp per
+// frame, lane = lag k: the lane sums |c_t - c_{t-k}| over all bins, so the
+// warp's loads are independent and in flight together).
 template <bool kVec4>
-__global__ void __launch_bounds__(kThreads) select_static_kernel(const uint32_t* __restrict__ hist, uint32_t n,
-                                                                 SelectArgs a, uint32_t* __restrict__ scratch,
-                                                                 float* __restrict__ scores,
-                                                                 uint8_t* __restrict__ keep) {
-  extern __shared__ __align__(16) uint32_t sm[];
-  __shared__ uint32_t entry[kWarps + 1];
-  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+__global__ void __launch_bounds__(kWinThreads) static_window_kernel(const uint32_t* __restrict__ hist, uint32_t n,
+                                                                    SelectArgs a, uint32_t* __restrict__ scratch) {
+  const uint32_t lane = threadIdx.x & 31;
   const uint32_t B = a.bins, L = a.l_max, W = a.mask_words;
   uint32_t* l1 = scratch;                                   // [n][L]
   uint32_t* mask = scratch + static_cast<uint64_t>(n) * L;  // [n][W]
-
-  // phase 1: windowed distances and per-gap keep bits of every frame (warp per
-  // frame, lane = lag k: the lane sums |c_t - c_{t-k}| over all bins, so the
-  // warp's loads are independent and in flight together)
-  for (uint32_t t = warp; t < n; t += kWarps) {
+  const uint32_t warps = gridDim.x * (kWinThreads / 32);
+  for (uint32_t t = blockIdx.x * (kWinThreads / 32) + (threadIdx.x >> 5); t < n; t += warps) {
     const uint32_t* ct = hist + static_cast<uint64_t>(t) * B;
     uint32_t l_adj = 0;
     for (uint32_t w = 0; w < W; ++w) {
@@ -91,9 +89,20 @@ __global__ void __launch_bounds__(kThreads) select_static_kernel(const uint32_t*
       if (lane == 0) mask[static_cast<uint64_t>(t) * W + w] = m;
     }
   }
-  __syncthreads();
+}
 
-  // phase 2: gap-map scan from a fresh stream (frame 0 is the first frame)
+// Phase 2: gap-map scan from a fresh stream (frame 0 is the first frame), one
+// CTA, over the distances and keep bits the kernel before it wrote.
+__global__ void __launch_bounds__(kThreads) select_static_kernel(uint32_t n, SelectArgs a,
+                                                                 const uint32_t* __restrict__ scratch,
+                                                                 float* __restrict__ scores,
+                                                                 uint8_t* __restrict__ keep) {
+  extern __shared__ __align__(16) uint32_t sm[];
+  __shared__ uint32_t entry[kWarps + 1];
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t L = a.l_max, W = a.mask_words;
+  const uint32_t* l1 = scratch;                                   // [n][L]
+  const uint32_t* mask = scratch + static_cast<uint64_t>(n) * L;  // [n][W]
   uint32_t* smask = sm;                                              // [kTile][W]
   uint16_t* sgap = reinterpret_cast<uint16_t*>(smask + kTile * W);   // [kTile]
   uint16_t* sexit = sgap + kTile;                                    // [kWarps][L]
@@ -160,9 +169,7 @@ cudaError_t setup_device(int dev, uint32_t** out) {
     cudaError_t e = cudaGetSymbolAddress(&ptr, g_select_scratch);
     if (e != cudaSuccess) return e;
     const int smem = static_cast<int>(static_smem_bytes(kMaxLmax, (kMaxLmax + 31) / 32));
-    e = cudaFuncSetAttribute(select_static_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(select_static_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(select_static_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     g_scratch_ptr[dev] = static_cast<uint32_t*>(ptr);
   }
@@ -233,10 +240,14 @@ int cofie_ngff_select_static(const cofie_ngff_params* p, const uint32_t* hist, u
   a.two_n = static_cast<float>(2ull * p->width * p->height);
   const size_t smem = static_smem_bytes(p->l_max, W);
   const cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const uint32_t win_grid = (n + kWinThreads / 32 - 1) / (kWinThreads / 32);
   if (p->bins % 4 == 0 && reinterpret_cast<uintptr_t>(hist) % 16 == 0)
-    select_static_kernel<true><<<1, kThreads, smem, st>>>(hist, n, a, scratch, scores_out, keep_out);
+    static_window_kernel<true><<<win_grid, kWinThreads, 0, st>>>(hist, n, a, scratch);
   else
-    select_static_kernel<false><<<1, kThreads, smem, st>>>(hist, n, a, scratch, scores_out, keep_out);
+    static_window_kernel<false><<<win_grid, kWinThreads, 0, st>>>(hist, n, a, scratch);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(COFIE_ECUDA, cudaGetErrorString(e), err, err_cap);
+  select_static_kernel<<<1, kThreads, smem, st>>>(n, a, scratch, scores_out, keep_out);
   e = cudaGetLastError();
   if (e != cudaSuccess) return fail(COFIE_ECUDA, cudaGetErrorString(e), err, err_cap);
   return COFIE_OK;
