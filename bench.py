@@ -380,6 +380,40 @@ def hd1080_parity(f, dev, host, spec, signal, l_max):
     return out
 
 
+def _compact(x, digits=5):
+    """x with floats rounded to `digits` significant digits (a short line)."""
+    if isinstance(x, float):
+        return float(f"{x:.{digits}g}")
+    if isinstance(x, dict):
+        return {k: _compact(v, digits) for k, v in x.items()}
+    if isinstance(x, list):
+        return [_compact(v, digits) for v in x]
+    return x
+
+
+def _config_summary(name, d):
+    """The figures of one config kept in the headline line (the full figures
+    are printed by bench.py --workload NAME)."""
+    keep = {"tiny": ("workload", "frames_per_s", "ms_per_step", "pixel_gbs", "latency_ms_p50", "latency_ms_p99", "e2e",
+                     "kept", "parity"),
+            "medium": ("workload", "pipelined_frames_per_s", "graph_frames_per_s", "graph_ms_per_push",
+                       "latency_ms_p50", "latency_ms_p99", "e2e", "kernels_per_push", "kept", "parity"),
+            "serving": ("workload", "calls", "pipelined_frames_per_s", "graph_frames_per_s", "graph_ms_per_call",
+                        "latency_ms_p50", "latency_ms_p99", "keep_ratio", "parity"),
+            "rare_event": ("workload", "frames_per_s", "pixel_gbs", "events", "e2e", "taus")}[name]
+    out = {k: d[k] for k in keep if k in d}
+    for e in ("e2e",):
+        if isinstance(out.get(e), dict):
+            out[e] = {k: v for k, v in out[e].items() if k not in ("how", "statistic")}
+    par = out.get("parity")
+    if isinstance(par, dict):
+        out["parity"] = {k: v for k, v in par.items() if k in ("frames", "hist_equal", "keep_equal", "max_rel_score_err",
+                                                                 "band_frames", "candidates_equal")}
+    if "seconds" in d:
+        out["seconds"] = d["seconds"]
+    return _compact(out)
+
+
 def other_configs(args):
     """Figures of the benchmark's other streams, each at its full size, in one
     run after the headline: tiny (64 x 224x224), medium (600 x 448x448 in
@@ -396,10 +430,11 @@ def other_configs(args):
             out[name] = {"skipped": f"the {args.configs_budget:.0f} s budget was spent ({el:.0f} s)"}
             continue
         t0 = time.perf_counter()
-        out[name] = fn(args)
-        out[name]["seconds"] = time.perf_counter() - t0
+        d = fn(args)
+        d["seconds"] = time.perf_counter() - t0
+        out[name] = _config_summary(name, d)
         torch.cuda.empty_cache()
-    out["seconds"] = time.perf_counter() - t_start
+    out["seconds"] = round(time.perf_counter() - t_start, 1)
     return out
 
 
@@ -579,6 +614,8 @@ def bench_gb300(args):
             "parity": parity,
             "configs": configs,
         }
+        for k in ("pixel_gbs", "frac_of_nominal_8tbs", "roofline", "e2e", "cpu_baseline", "parity"):
+            line[k] = _compact(line[k], 6)
         print(json.dumps(line), flush=True)
     f.close()
     if world > 1:
