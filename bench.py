@@ -402,13 +402,20 @@ def _config_summary(name, d):
                         "latency_ms_p50", "latency_ms_p99", "keep_ratio", "parity"),
             "rare_event": ("workload", "frames_per_s", "pixel_gbs", "events", "e2e", "taus")}[name]
     out = {k: d[k] for k in keep if k in d}
+    if name == "rare_event":  # per tau: keep ratio, event-frame recall, per-event recall; one parity summary
+        taus = out.pop("taus")
+        out["recall_by_tau"] = {t: [v["keep_ratio"], v["event_frame_recall"], v["event_recall"]] for t, v in taus.items()}
+        out["recall_fields"] = ["keep_ratio", "event_frame_recall", "event_recall"]
+        out["parity"] = {"keep_equal_every_tau": all(v["parity"]["keep_equal"] for v in taus.values()),
+                         "max_rel_score_err": max(v["parity"]["max_rel_score_err"] for v in taus.values()),
+                         "band_frames": sorted({f for v in taus.values() for f in v["parity"]["band_frames"]})}
     for e in ("e2e",):
         if isinstance(out.get(e), dict):
             out[e] = {k: v for k, v in out[e].items() if k not in ("how", "statistic")}
     par = out.get("parity")
     if isinstance(par, dict):
-        out["parity"] = {k: v for k, v in par.items() if k in ("frames", "hist_equal", "keep_equal", "max_rel_score_err",
-                                                                 "band_frames", "candidates_equal")}
+        out["parity"] = {k: v for k, v in par.items() if k in ("frames", "hist_equal", "keep_equal", "keep_equal_every_tau",
+                                                                 "max_rel_score_err", "band_frames", "candidates_equal")}
     if "seconds" in d:
         out["seconds"] = d["seconds"]
     return _compact(out)
