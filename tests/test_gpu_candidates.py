@@ -272,3 +272,45 @@ def test_long_stream_crosses_record_tiles(m_min):
     f.status()
     assert (ko != 0).sum() < 5000, "the fill case must exercise the uniform frames"
     f.close()
+
+
+def test_full_batch_of_64_streams():
+    """The most streams one batched call takes (64), each pushing 0-9 frames
+    per call in a shuffled descriptor order, with the scene-change signal so
+    that every rule of the walk runs; every stream's keep codes, scores and
+    candidate set against the oracle's."""
+    from oracle import scd_oracle as SC
+    from paper_2609_03675_gb300 import NGFF, _abi
+    g = np.random.default_rng(64)
+    S, T, w, h = _abi.MAX_BATCH, 60, 32, 16
+    o = O.load()
+    frs = [synth.generate(synth.medium(seed=900 + s).with_(width=w, height=h, frames=T, mean_scene_len=4))
+           for s in range(S)]
+    want = []
+    for fr in frs:
+        hist = o.run(fr, O.Params(w, h))[0]
+        want.append(SC.select(hist, O.Params(w, h, tau=0.2, l_max=9), 0.15, 0.05))
+    f = NGFF(w, h, tau=0.2, l_max=9, signal=_abi.SIGNAL_SCD, scd_cut=0.15, scd_gradual=0.05, max_streams=S)
+    devs = [torch.from_numpy(x).cuda() for x in frs]
+    sc = torch.zeros((S, T), dtype=torch.float32, device="cuda")
+    kp = torch.full((S, T), 255, dtype=torch.uint8, device="cuda")
+    pos = [0] * S
+    while min(pos) < T:
+        items = []
+        for s in g.permutation(S):
+            s = int(s)
+            n = int(min(g.integers(0, 10), T - pos[s]))
+            items.append((s, devs[s][pos[s]:pos[s] + n], sc[s, pos[s]:pos[s] + n], kp[s, pos[s]:pos[s] + n]))
+            pos[s] += n
+        f.push_batch(items)
+    torch.cuda.synchronize()
+    f.status()
+    ks, ss = kp.cpu().numpy(), sc.cpu().numpy().astype(np.float64)
+    for s in range(S):
+        so, ko = want[s]
+        assert np.array_equal(ks[s], ko), f"stream {s}"
+        assert (np.abs(ss[s] - so) <= 1e-6 * so).all(), f"stream {s}"
+        got = f.candidates(s).cpu().numpy().astype(np.uint32)
+        assert np.array_equal(got, o.candidates(ko, 4)), f"stream {s}"
+    assert any((w_[1] == SC.KEEP_SCENE).any() for w_ in want), "scene changes occur"
+    f.close()
