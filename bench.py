@@ -1124,8 +1124,18 @@ def bench_pipeline(args):
                     f"({qs.n_text} text tokens, {qs.tokens_per_frame} synthetic keys per frame)",
         "steps": steps, "ms_per_step": float(ms.sum()), "frames_per_s": spec.frames / (ms.sum() / 1e3),
         "candidates": m, "qer_selected": int(k_dev.item()),
+        "drop_ratios": drop_ratios(spec.frames, m, int(k_dev.item())),
         "phase_ms": {"ngff_push": ms[0], "candidates": ms[1], "gather": ms[2], "qer": ms[3]},
         "timing": "CUDA events between phases on one stream, device synchronised after each step"}), flush=True)
+
+
+def drop_ratios(frames: int, candidates: int, selected: int) -> dict:
+    """Drop ratios of the coarse-to-fine path (Eq. 9): NGFF keeps `candidates`
+    of `frames`, QER keeps `selected` of the candidates, and the total drop is
+    D_total = 1 - (1 - D_NGFF)(1 - D_QER)."""
+    d_ngff = 1.0 - candidates / frames if frames else 0.0
+    d_qer = 1.0 - selected / candidates if candidates else 0.0
+    return {"ngff": d_ngff, "qer": d_qer, "total": 1.0 - (1.0 - d_ngff) * (1.0 - d_qer)}
 
 
 def peaks_bf16():
