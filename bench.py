@@ -47,7 +47,7 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="target CPU work of the oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--workload", choices=["hd1080", "serving", "medium", "rare_event", "gather", "qer", "shards",
-                                           "signals", "pipeline", "tiny", "static"],
+                                           "signals", "pipeline", "tiny", "static", "sensitivity"],
                     default="hd1080",
                     help="hd1080 is the benchmark line; the others print their own JSON lines (latency, recall, "
                          "finalize + gather bandwidth)")
@@ -1427,6 +1427,75 @@ def bench_signals(args):
     print(json.dumps(out), flush=True)
 
 
+SENSITIVITY_ROWS = (  # (M_min, L_max, tau_h): the rows of the paper's NGFF sensitivity table (App. B.2)
+    (2, 30, 0.30), (4, 30, 0.30), (8, 30, 0.30),
+    (4, 15, 0.30), (4, 45, 0.30),
+    (4, 30, 0.15), (4, 30, 0.45), (4, 30, 0.60), (4, 30, 0.75))
+
+
+def bench_sensitivity(args):
+    """The synthetic counterpart of the paper's NGFF sensitivity table: for
+    each (M_min, L_max, tau_h) row, the stream is pushed whole and closed, and
+    the line reports the drop ratio 1 - |S_c| / T (the last frame and the
+    M_min fill included), the device-resident frames/s of push + close, and
+    the keep codes and candidate set against the oracle. Streams: the 1080p
+    stream (3600 frames; its scene cuts change the histogram by far more than
+    any tau of the table and little else moves it), the medium stream (600
+    frames with brightness drift, pushed whole) and the tiny stream (64
+    frames, where M_min can matter)."""
+    import numpy as np
+    import torch
+
+    import oracle as O
+    import synth
+    from paper_2609_03675_gb300 import NGFF
+    out = {"workload": "sensitivity: the rows of the NGFF sensitivity table on the 1080p, medium and tiny streams",
+           "fields": ["m_min", "l_max", "tau", "drop_pct", "frames_per_s", "keep_equal", "candidates_equal"],
+           "streams": {}}
+    o = O.load()
+    for name, spec in (("1080p", synth.hd1080()), ("medium", synth.medium()), ("tiny", synth.tiny())):
+        T = spec.frames
+        host = torch.empty((T, spec.height, spec.width, 3), dtype=torch.uint8, pin_memory=True)
+        synth.generate(spec, out=host.data_ptr())
+        dev = host.cuda()
+        hist_o = o.histograms_parallel(host.data_ptr(), T, O.Params(spec.width, spec.height))
+        del host
+        keep = torch.empty(T, dtype=torch.uint8, device="cuda")
+        idx = torch.empty(T, dtype=torch.int32, device="cuda")
+        m_dev = torch.zeros(1, dtype=torch.int32, device="cuda")
+        rows = []
+        for m_min, l_max, tau in SENSITIVITY_ROWS:
+            f = NGFF(spec.width, spec.height, m_min=m_min, l_max=l_max, tau=tau, max_frames_per_push=T)
+
+            def step():
+                f.reset()
+                f.push(dev, keep=keep)
+                f.candidates_raw(0, idx.data_ptr(), T, m_dev.data_ptr())
+
+            for _ in range(3):
+                step()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = 10
+            e0.record()
+            for _ in range(reps):
+                step()
+            e1.record()
+            torch.cuda.synchronize()
+            f.status()
+            m = int(m_dev.item())
+            _, ko = o.select(hist_o, O.Params(spec.width, spec.height, m_min=m_min, l_max=l_max, tau=tau))
+            want = o.candidates(ko, m_min)
+            rows.append([m_min, l_max, tau, round(100.0 * (1.0 - m / T), 2),
+                         round(reps * T / (e0.elapsed_time(e1) / 1e3)),
+                         bool(np.array_equal(keep.cpu().numpy(), ko)),
+                         bool(np.array_equal(idx[:m].cpu().numpy().astype(np.uint32), want))])
+            f.close()
+        out["streams"][name] = {"frames": T, "size": f"{spec.width}x{spec.height}", "rows": rows}
+        del dev
+        torch.cuda.empty_cache()
+    print(json.dumps(out), flush=True)
+
+
 def bench_static(args):
     """cofie_ngff_select_static (the allocation-free selection) at
     the largest sizes its static array admits and at a typical one: CUDA
@@ -1495,6 +1564,8 @@ def main():
         print(json.dumps(tiny_figures(args)), flush=True)
     elif args.workload == "static":
         bench_static(args)
+    elif args.workload == "sensitivity":
+        bench_sensitivity(args)
     else:
         bench_gb300(args)
 
