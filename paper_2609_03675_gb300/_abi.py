@@ -1,8 +1,8 @@
 """ctypes view of the C ABI in include/cofie_ngff.h (argument marshalling only).
 
 Loads ``libcofie_ngff.so`` from this package directory. There is no fallback:
-if the library has not been built, importing fails with an error that says
-how to build it.
+if the library has not been built, loading it (the first NGFF or QER handle
+created) fails with an error that says how to build it.
 """
 from __future__ import annotations
 

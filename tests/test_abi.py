@@ -143,3 +143,15 @@ def test_header_is_c99_and_a_c_client_links(tmp_path):
                         os.path.join(REPO, "tests", "c", "ngff_client.c"), "-o", str(exe), "-L", lib_dir,
                         "-lcofie_ngff", f"-Wl,-rpath,{lib_dir}"], capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """No fallback: with the library absent, creating a handle raises an error
+    that says how to build it (nothing runs on the CPU instead)."""
+    from paper_2609_03675_gb300 import NGFF, QER, _abi
+    monkeypatch.setattr(_abi, "LIB_PATH", str(tmp_path / "libcofie_ngff.so"))
+    monkeypatch.setattr(_abi, "_lib", None)
+    with pytest.raises(RuntimeError, match="has not been built"):
+        NGFF(64, 48)
+    with pytest.raises(RuntimeError, match="has not been built"):
+        QER(8, 32, 8, 128, 4, 16, 0.3)

@@ -20,7 +20,7 @@ pytestmark = pytest.mark.gpu
 def _cuda():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
-    from paper_2609_03675_gb300 import NGFF  # noqa: F401  (fails loudly if the library is missing)
+    from paper_2609_03675_gb300 import NGFF  # noqa: F401  (creating a handle fails loudly if the library is missing)
 
 
 def _ngff(w, h, **kw):
