@@ -415,7 +415,8 @@ def _config_summary(name, d):
     par = out.get("parity")
     if isinstance(par, dict):
         out["parity"] = {k: v for k, v in par.items() if k in ("frames", "hist_equal", "keep_equal", "keep_equal_every_tau",
-                                                                 "max_rel_score_err", "band_frames", "candidates_equal")}
+                                                                 "keep_mismatch_outside_band", "max_rel_score_err",
+                                                                 "band_frames", "candidates_equal")}
     if "seconds" in d:
         out["seconds"] = d["seconds"]
     return _compact(out)
