@@ -236,6 +236,7 @@ def oracle_parallel_sample(frames_u8_ptr, spec, target_s: float, l_max: int = 30
 
 
 SCORE_RTOL = 1e-6  # the fp32 score against the oracle's double-precision distance
+SERVING_E2E_FRAMES = 300  # frames per stream of the serving workload's end-to-end leg (6.6 GB of pinned frames)
 
 
 def parity_block(tau, scores, keep, want_scores, want_keep, hist=None, want_hist=None, idx=None, want_idx=None):
@@ -399,7 +400,7 @@ def _config_summary(name, d):
             "medium": ("workload", "pipelined_frames_per_s", "graph_frames_per_s", "graph_ms_per_push",
                        "latency_ms_p50", "latency_ms_p99", "e2e", "kernels_per_push", "kept", "parity"),
             "serving": ("workload", "calls", "pipelined_frames_per_s", "graph_frames_per_s", "graph_ms_per_call",
-                        "latency_ms_p50", "latency_ms_p99", "keep_ratio", "parity"),
+                        "latency_ms_p50", "latency_ms_p99", "keep_ratio", "e2e", "parity"),
             "rare_event": ("workload", "frames_per_s", "pixel_gbs", "events", "e2e", "taus")}[name]
     out = {k: d[k] for k in keep if k in d}
     if name == "rare_event":  # per tau: keep ratio, event-frame recall, per-event recall; one parity summary
@@ -791,6 +792,55 @@ def serving_figures(args, parity: bool = True):
 
     el_graph = _graph_seconds(lambda: [f.push_batch_raw(arr, nd) for arr, nd in plan], reset_all)
     f.status()
+
+    # end to end: the same calls over the first E frames of every stream with
+    # the frames in pinned host memory and the scores and keep codes written
+    # to pinned host memory, through the same batched entry point
+    E = min(T, SERVING_E2E_FRAMES)
+    host_fr = torch.empty((S, E, H, W, 3), dtype=torch.uint8, pin_memory=True)
+    for s in range(S):
+        host_fr[s].copy_(dev[s][:E])
+    hs = torch.empty((S, E), dtype=torch.float32, pin_memory=True)
+    hk = torch.empty((S, E), dtype=torch.uint8, pin_memory=True)
+    hplan, pos, call = [], [0] * S, 0
+    while min(pos) < E:
+        items = []
+        for s in range(S):
+            if pos[s] >= E:
+                continue
+            n = int(min(sizes[s][call], E - pos[s]))
+            items.append((s, host_fr[s, pos[s]:pos[s] + n], hs[s, pos[s]:pos[s] + n], hk[s, pos[s]:pos[s] + n]))
+            pos[s] += n
+        hplan.append(f.make_batch(items))
+        call += 1
+    torch.cuda.synchronize()
+
+    def run_host(sync_each):
+        reset_all()
+        hlat = []
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for arr, nd in hplan:
+            c0 = time.perf_counter()
+            f.push_batch_raw(arr, nd, st)
+            if sync_each:
+                torch.cuda.synchronize()
+                hlat.append((time.perf_counter() - c0) * 1e3)
+        torch.cuda.synchronize()
+        return time.perf_counter() - t0, hlat
+
+    run_host(False)
+    el_host, _ = run_host(False)
+    _, hlat = run_host(True)
+    f.status()
+    assert torch.equal(hk, keep[:, :E].cpu()), "end-to-end keep codes differ from the device-resident run"
+    bytes_h2d = S * E * W * H * 3
+    e2e = {"frames_per_s": S * E / el_host, "latency_ms_p50": _pct(hlat, 50), "latency_ms_p99": _pct(hlat, 99),
+           "calls": len(hplan), "h2d_bytes_per_call": bytes_h2d / len(hplan),
+           "d2h_bytes_per_call": S * E * 5 / len(hplan), "h2d_gbs": bytes_h2d / el_host / 1e9,
+           "how": f"the first {E} frames of every stream: pinned host frames in, pinned host scores and keep codes "
+                  "out, through the same batched call"}
+    del host_fr
     line = {"workload": "serving: 32 streams x 1800 uint8 RGB frames of 640x360, U{1..8} frames per stream per "
                         "batched call, B=32, L_max=30, tau_h=0.30",
             "calls": len(plan), "frames": frames_total,
@@ -799,7 +849,7 @@ def serving_figures(args, parity: bool = True):
             "sync_frames_per_s": frames_total / el_sync,
             "latency_ms_p50": _pct(lat, 50), "latency_ms_p99": _pct(lat, 99), "latency_ms_max": max(lat),
             "latency": "host wall time of one push_batch call plus a device synchronise",
-            "keep_ratio": float((keep != 0).float().mean().item()), "parity": par}
+            "keep_ratio": float((keep != 0).float().mean().item()), "e2e": e2e, "parity": par}
     f.close()
     return line
 

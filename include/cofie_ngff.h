@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define COFIE_NGFF_ABI_VERSION 4
+#define COFIE_NGFF_ABI_VERSION 5
 
 /* Return codes. */
 #define COFIE_OK 0
@@ -159,9 +159,9 @@ typedef struct {
 typedef struct {
   uint32_t stream;        /* stream index, < max_streams; distinct within one batch */
   uint32_t n;             /* number of frames, may be 0 */
-  const uint8_t* frames;  /* n frames, device memory, 16-byte aligned */
-  float* scores_out;      /* n floats, device memory, or NULL */
-  uint8_t* keep_out;      /* n keep codes, device memory, or NULL */
+  const uint8_t* frames;  /* n frames: device memory (16-byte aligned) or host memory */
+  float* scores_out;      /* n floats, device or host memory, or NULL */
+  uint8_t* keep_out;      /* n keep codes, device or host memory, or NULL */
 } cofie_ngff_push_desc;
 
 /* uint32 words per frame of the handle's signal features (bins for the histogram). */
@@ -218,10 +218,17 @@ int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, 
 /*
  * Pushes frames of several streams in one set of launches (serving many
  * concurrent streams). desc[i] is as in cofie_ngff_push for stream
- * desc[i].stream; device memory only; streams distinct within the call;
- * nd <= COFIE_NGFF_MAX_BATCH and the total frame count <= max_frames_per_push.
- * Equivalent to one cofie_ngff_push per descriptor, and capturable into a
- * CUDA graph as cofie_ngff_push is. Errors: COFIE_EINVAL, COFIE_ECUDA.
+ * desc[i].stream; streams distinct within the call; nd <=
+ * COFIE_NGFF_MAX_BATCH and the total frame count <= max_frames_per_push.
+ * Frames and outputs may be device or host memory, descriptor by descriptor:
+ * the host frames of one call are copied (one copy per descriptor, on the
+ * handle's copy stream) into one of the two staging buffers, so together
+ * they must fit host_stage_bytes (COFIE_EINVAL otherwise); host outputs are
+ * copied back on cuda_stream after the selection. Equivalent to one
+ * cofie_ngff_push per descriptor. With device frames and outputs only, the
+ * call is capturable into a CUDA graph as cofie_ngff_push is (host memory
+ * while capturing is COFIE_EINVAL). Errors: COFIE_EINVAL, COFIE_ENOMEM (the
+ * staging buffers, allocated on first use), COFIE_ECUDA.
  */
 int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream);
 

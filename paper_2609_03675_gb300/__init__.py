@@ -127,7 +127,8 @@ class NGFF:
 
     def make_batch(self, items):
         """Descriptor array for push_batch_raw from a list of
-        (stream, frames[cuda uint8], scores[cuda f32] | None, keep[cuda u8] | None)."""
+        (stream, frames[uint8], scores[f32] | None, keep[u8] | None), each
+        tensor on the handle's device or in (preferably pinned) host memory."""
         arr = (_abi.PushDesc * max(1, len(items)))()
         for i, (stream, frames, scores, keep) in enumerate(items):
             n = self._frames(frames)
@@ -136,7 +137,9 @@ class NGFF:
         return arr, len(items)
 
     def push_batch(self, items, cuda_stream=None):
-        """items: list of (stream, frames[cuda uint8], scores[cuda f32] | None, keep[cuda u8] | None)."""
+        """items: list of (stream, frames[uint8], scores[f32] | None, keep[u8] | None),
+        device or host tensors; host frames of one call must fit one staging
+        buffer (host_stage_bytes)."""
         arr, nd = self.make_batch(items)
         self.push_batch_raw(arr, nd, cuda_stream)
 

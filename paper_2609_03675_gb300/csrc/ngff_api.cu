@@ -735,37 +735,90 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
   if (!guard.ok) return h->fail(COFIE_ECUDA, "cannot select the handle's device");
   SegTable segs;
   memset(&segs, 0, sizeof segs);
-  uint64_t rows = 0;
+  uint64_t rows = 0, staged_bytes = 0;
+  bool host_frames = false, host_out = false;
+  MemKind kf[COFIE_NGFF_MAX_BATCH], ks[COFIE_NGFF_MAX_BATCH], kk[COFIE_NGFF_MAX_BATCH];
+  uint64_t stage_off[COFIE_NGFF_MAX_BATCH];
   std::vector<uint8_t> used(h->p.max_streams, 0);
   for (uint32_t i = 0; i < nd; ++i) {
     const cofie_ngff_push_desc& d = desc[i];
     if (d.stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
     if (used[d.stream]) return h->fail(COFIE_EINVAL, "a stream appears twice in one batch");
     used[d.stream] = 1;
+    kf[i] = ks[i] = kk[i] = kNull;
+    stage_off[i] = 0;
     if (d.n > 0) {
       int fdev = -1;
-      if (!d.frames || classify(d.frames, &fdev) != kDevice || fdev != h->device)
-        return h->fail(COFIE_EINVAL, "batched frames must be device memory on the handle's device");
-      if ((d.scores_out && classify(d.scores_out) != kDevice) || (d.keep_out && classify(d.keep_out) != kDevice))
-        return h->fail(COFIE_EINVAL, "batched outputs must be device memory");
+      kf[i] = d.frames ? classify(d.frames, &fdev) : kNull;
+      if (kf[i] == kNull || (kf[i] == kDevice && fdev != h->device))
+        return h->fail(COFIE_EINVAL, "batched frames must be device memory on the handle's device, or host memory");
+      int sdev = -1, kdev = -1;
+      ks[i] = classify(d.scores_out, &sdev);
+      kk[i] = classify(d.keep_out, &kdev);
+      if ((ks[i] == kDevice && sdev != h->device) || (kk[i] == kDevice && kdev != h->device))
+        return h->fail(COFIE_EINVAL, "batched outputs live on another device");
+      if (kf[i] != kDevice) {  // staged back to back, each descriptor's frames from a 16-byte boundary
+        host_frames = true;
+        stage_off[i] = staged_bytes;
+        staged_bytes += (static_cast<uint64_t>(d.n) * h->frame_bytes + 15) & ~uint64_t(15);
+      }
+      host_out = host_out || (ks[i] != kDevice && ks[i] != kNull) || (kk[i] != kDevice && kk[i] != kNull);
     }
-    Segment& s = segs.s[segs.count++];
-    s.frames = d.frames;
-    s.n = d.n;
-    s.row0 = static_cast<uint32_t>(rows);
-    s.stream = d.stream;
-    s.scores = d.scores_out;
-    s.keep = d.keep_out;
     rows += d.n;
   }
   if (rows > h->p.max_frames_per_push) return h->fail(COFIE_EINVAL, "batch exceeds max_frames_per_push frames");
-  segs.rows = static_cast<uint32_t>(rows);
   const cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   const int cap = capture_state(st);
   if (cap < 0) return h->fail(COFIE_ECUDA, "cannot read the CUDA stream's capture state");
+  if (cap && (host_frames || host_out))
+    return h->fail(COFIE_EINVAL, "a batch captured into a CUDA graph takes device frames and outputs only");
+  uint32_t slot = 0;
+  if (host_frames) {
+    int rc = ensure_staging(h);
+    if (rc != COFIE_OK) return rc;
+    if (staged_bytes > h->stage_bytes)
+      return h->fail(COFIE_EINVAL, "the batch's host frames exceed one staging buffer (host_stage_bytes)");
+    // one copy per host descriptor on the copy stream, into the staging slot
+    // the kernels of the call before the last have finished reading
+    slot = h->stage_next;
+    h->stage_next ^= 1u;
+    cudaError_t e = cudaStreamWaitEvent(h->copy_stream, h->ev_free[slot], 0);
+    for (uint32_t i = 0; i < nd && e == cudaSuccess; ++i)
+      if (desc[i].n > 0 && kf[i] != kDevice)
+        e = cudaMemcpyAsync(h->d_stage[slot] + stage_off[i], desc[i].frames,
+                            static_cast<uint64_t>(desc[i].n) * h->frame_bytes, cudaMemcpyHostToDevice, h->copy_stream);
+    if (e == cudaSuccess) e = cudaEventRecord(h->ev_copied[slot], h->copy_stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_copied[slot], 0);
+    if (e != cudaSuccess) return h->cuda_fail(e, "host frame staging");
+  }
+  rows = 0;
+  for (uint32_t i = 0; i < nd; ++i) {
+    const cofie_ngff_push_desc& d = desc[i];
+    Segment& s = segs.s[segs.count++];
+    s.frames = (d.n > 0 && kf[i] != kDevice) ? h->d_stage[slot] + stage_off[i] : d.frames;
+    s.n = d.n;
+    s.row0 = static_cast<uint32_t>(rows);
+    s.stream = d.stream;
+    // host outputs are written to the row's place in the device scratch and copied back below
+    s.scores = ks[i] == kDevice ? d.scores_out : (ks[i] == kNull ? nullptr : h->d_scores + rows);
+    s.keep = kk[i] == kDevice ? d.keep_out : (kk[i] == kNull ? nullptr : h->d_keep + rows);
+    rows += d.n;
+  }
+  segs.rows = static_cast<uint32_t>(rows);
   h->shard.ready = false;
   int rc = run_segments(h, segs, st, false, cap == 1);
   if (rc != COFIE_OK) return rc;
+  cudaError_t e = cudaSuccess;
+  for (uint32_t i = 0; i < nd && e == cudaSuccess; ++i) {
+    const Segment& s = segs.s[i];
+    if (desc[i].n == 0) continue;
+    if (ks[i] == kHostPinned || ks[i] == kHostPageable)
+      e = cudaMemcpyAsync(desc[i].scores_out, s.scores, desc[i].n * sizeof(float), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess && (kk[i] == kHostPinned || kk[i] == kHostPageable))
+      e = cudaMemcpyAsync(desc[i].keep_out, s.keep, desc[i].n, cudaMemcpyDeviceToHost, st);
+  }
+  if (e == cudaSuccess && host_frames) e = cudaEventRecord(h->ev_free[slot], st);
+  if (e != cudaSuccess) return h->cuda_fail(e, "batched output copy");
   if (!cap)
     for (uint32_t i = 0; i < nd; ++i) h->seen[desc[i].stream] += desc[i].n;
   h->err.clear();

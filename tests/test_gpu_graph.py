@@ -182,8 +182,13 @@ def test_capture_refuses_host_memory():
             f.push(host, scores=sc, keep=kp)
         with pytest.raises(NGFFError) as e2:
             f.push(buf, scores=sc_host, keep=kp)
+        with pytest.raises(NGFFError) as e3:  # the batched call: host frames
+            f.push_batch([(0, host, sc, kp)])
+        with pytest.raises(NGFFError) as e4:  # and host outputs
+            f.push_batch([(0, buf, sc_host, kp)])
         f.push(buf, scores=sc, keep=kp)
-    assert e1.value.code == _abi.EINVAL and e2.value.code == _abi.EINVAL
+    assert all(e.value.code == _abi.EINVAL for e in (e1, e2, e3, e4))
+    assert "device frames and outputs only" in str(e3.value) and "device frames and outputs only" in str(e4.value)
     s_all, k_all = [], []
     for i in range(0, 24, 8):
         buf.copy_(dev[i:i + 8])

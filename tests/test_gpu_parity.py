@@ -136,6 +136,69 @@ def test_multistream_batch_equals_single():
         assert (np.abs(got_s - so) <= 1e-6 * so).all()
 
 
+def test_batch_with_host_frames_and_outputs():
+    """push_batch with each descriptor's frames and outputs in device, pinned
+    host or pageable host memory (the mix changes from call to call), staged
+    through buffers that several calls reuse in turn, against the oracle."""
+    from paper_2609_03675_gb300 import _abi
+    g = np.random.default_rng(11)
+    S, T, w, h = 5, 90, 48, 32
+    specs = [synth.medium(seed=200 + s).with_(width=w, height=h, frames=T) for s in range(S)]
+    frames_np = [synth.generate(sp) for sp in specs]
+    frames_dev = [torch.from_numpy(x).cuda() for x in frames_np]
+    frames_pin = [torch.from_numpy(x).pin_memory() for x in frames_np]
+    p = O.Params(w, h, tau=0.05)
+    want = [oracle_run(x, p) for x in frames_np]
+    fb = specs[0].frame_bytes
+    # staging of 40 frames: a call of up to 5 x 8 host frames fits one buffer
+    f = _ngff(w, h, tau=0.05, max_streams=S, host_stage_bytes=40 * fb)
+    out_dev = [(torch.zeros(T, dtype=torch.float32, device="cuda"), torch.zeros(T, dtype=torch.uint8, device="cuda"))
+               for _ in range(S)]
+    out_pin = [(torch.zeros(T, dtype=torch.float32).pin_memory(), torch.zeros(T, dtype=torch.uint8).pin_memory())
+               for _ in range(S)]
+    out_np = [(np.zeros(T, np.float32), np.zeros(T, np.uint8)) for _ in range(S)]
+    # where each frame's outputs went: 0 device, 1 pinned, 2 pageable
+    where = np.full((S, T), -1)
+    pos = [0] * S
+    while min(pos) < T:
+        arr = (_abi.PushDesc * S)()
+        nd = 0
+        for s in g.permutation(S):
+            if pos[s] >= T:
+                continue
+            n = int(min(g.integers(0, 9), T - pos[s]))
+            a, fk, ok = pos[s], int(g.integers(0, 3)), int(g.integers(0, 3))
+            d = arr[nd]
+            d.stream, d.n = int(s), n
+            d.frames = (frames_dev[s].data_ptr(), frames_pin[s].data_ptr(), frames_np[s].ctypes.data)[fk] + a * fb
+            if ok == 0:
+                d.scores_out, d.keep_out = out_dev[s][0].data_ptr() + 4 * a, out_dev[s][1].data_ptr() + a
+            elif ok == 1:
+                d.scores_out, d.keep_out = out_pin[s][0].data_ptr() + 4 * a, out_pin[s][1].data_ptr() + a
+            else:
+                d.scores_out, d.keep_out = out_np[s][0].ctypes.data + 4 * a, out_np[s][1].ctypes.data + a
+            where[s, a:a + n] = ok
+            pos[s] += n
+            nd += 1
+        f.push_batch_raw(arr, nd)
+    torch.cuda.synchronize()
+    f.status()
+    for s in range(S):
+        sc = np.select([where[s] == 0, where[s] == 1], [out_dev[s][0].cpu().numpy(), out_pin[s][0].numpy()],
+                       out_np[s][0])
+        kc = np.select([where[s] == 0, where[s] == 1], [out_dev[s][1].cpu().numpy(), out_pin[s][1].numpy()],
+                       out_np[s][1])
+        _, so, ko = want[s]
+        assert np.array_equal(kc, ko), f"stream {s}: keep codes differ at {np.flatnonzero(kc != ko)[:10]}"
+        assert (np.abs(sc.astype(np.float64) - so) <= 1e-6 * so).all(), f"stream {s}"
+    # host frames beyond one staging buffer are refused before anything is enqueued
+    big = (_abi.PushDesc * 1)()
+    big[0].stream, big[0].n, big[0].frames = 0, 41, frames_pin[0].data_ptr()
+    assert f._lib.cofie_ngff_push_batch(f._h, big, 1, None) == _abi.EINVAL
+    assert b"staging" in f._lib.cofie_ngff_last_error(f._h)
+    f.close()
+
+
 def test_host_frames_and_host_outputs():
     spec = synth.medium().with_(width=128, height=96, frames=70)
     fr = synth.generate(spec)
