@@ -485,8 +485,9 @@ int push_impl(cofie_ngff* h, uint32_t stream, const uint8_t* frames, uint32_t n,
       if (e != cudaSuccess) return h->cuda_fail(e, "host frame staging");
       rc = run_piece(h, stream, h->d_stage[slot], m, scores ? scores + off : nullptr, ks, keep ? keep + off : nullptr,
                      kk, hist_out ? hist_out + static_cast<size_t>(off) * B : nullptr, kh, st, false);
-      if (rc != COFIE_OK) return rc;
+      // the slot is free again only behind whatever of this piece was enqueued, failed or not
       e = cudaEventRecord(h->ev_free[slot], st);
+      if (rc != COFIE_OK) return rc;
       if (e != cudaSuccess) return h->cuda_fail(e, "staging event");
     }
   }
@@ -807,7 +808,10 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
   segs.rows = static_cast<uint32_t>(rows);
   h->shard.ready = false;
   int rc = run_segments(h, segs, st, false, cap == 1);
-  if (rc != COFIE_OK) return rc;
+  if (rc != COFIE_OK) {
+    if (host_frames) cudaEventRecord(h->ev_free[slot], st);  // behind whatever of the call was enqueued
+    return rc;
+  }
   cudaError_t e = cudaSuccess;
   for (uint32_t i = 0; i < nd && e == cudaSuccess; ++i) {
     const Segment& s = segs.s[i];
