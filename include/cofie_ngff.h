@@ -285,7 +285,9 @@ int cofie_ngff_candidates_from_keep(cofie_ngff_t* h, const uint8_t* keep, uint32
  * Copies the m frames idx[0..m) of `frames` back to back into `out`: the
  * frames S_c that go on to the vision encoder (Sec. 3.2, "only these m frames
  * are sent to the encoder").
- *   frames   n_frames frames of 3 W H bytes, device memory.
+ *   frames   n_frames frames of 3 W H bytes: device memory, or pinned host
+ *            memory (read by the kernel over the host link through the
+ *            device's mapping of it; pageable host memory is COFIE_EINVAL).
  *   idx      m frame indices, device memory (for example the idx_out of cofie_ngff_candidates).
  *   out      m * 3 W H bytes, device memory, not overlapping frames.
  * An index >= n_frames is skipped and reported as COFIE_EDEVICE by

@@ -177,7 +177,8 @@ class NGFF:
         return idx[: m.value]
 
     def gather(self, frames: torch.Tensor, idx: torch.Tensor, out: torch.Tensor | None = None, cuda_stream=None):
-        """frames[idx] back to back (cuda uint8 [m, H, W, 3]): the encoder's input."""
+        """frames[idx] back to back (cuda uint8 [m, H, W, 3]): the encoder's input.
+        frames may be on the device or in pinned host memory; idx is on the device."""
         n = self._frames(frames)
         m = idx.numel()
         if out is None:

@@ -1198,12 +1198,25 @@ int cofie_ngff_gather(cofie_ngff_t* h, const uint8_t* frames, uint32_t n_frames,
   NvtxRange nvtx("ngff.gather");
   if (!h) return COFIE_EINVAL;
   if (m == 0) return COFIE_OK;
-  int d0 = -1, d1 = -1, d2 = -1;
-  if (!frames || !idx || !out || classify(frames, &d0) != kDevice || classify(idx, &d1) != kDevice ||
-      classify(out, &d2) != kDevice || d0 != h->device || d1 != h->device || d2 != h->device)
-    return h->fail(COFIE_EINVAL, "frames, idx and out must be device memory on the handle's device");
   DeviceGuard guard(h->device);
-  cudaError_t e = launch_gather(frames, n_frames, h->frame_bytes, idx, m, out, h->d_err,
+  if (!guard.ok) return h->fail(COFIE_ECUDA, "cannot select the handle's device");
+  int d0 = -1, d1 = -1, d2 = -1;
+  const MemKind kf = frames ? classify(frames, &d0) : kNull;
+  if (!idx || !out || classify(idx, &d1) != kDevice || classify(out, &d2) != kDevice || d1 != h->device ||
+      d2 != h->device)
+    return h->fail(COFIE_EINVAL, "idx and out must be device memory on the handle's device");
+  // frames: device memory, or pinned host memory that the kernel reads through the device's mapping of it
+  const uint8_t* src = nullptr;
+  if (kf == kDevice && d0 == h->device) {
+    src = frames;
+  } else if (kf == kHostPinned) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, frames) == cudaSuccess) src = static_cast<const uint8_t*>(a.devicePointer);
+    cudaGetLastError();
+  }
+  if (!src)
+    return h->fail(COFIE_EINVAL, "frames must be device memory on the handle's device, or pinned host memory");
+  cudaError_t e = launch_gather(src, n_frames, h->frame_bytes, idx, m, out, h->d_err, kf == kHostPinned,
                                 static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return h->cuda_fail(e, "gather kernel launch");
   h->n_other += 1;

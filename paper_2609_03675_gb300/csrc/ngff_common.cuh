@@ -262,6 +262,6 @@ cudaError_t launch_stream_candidates(const uint32_t* rec, uint32_t rec_words, co
                                      cudaStream_t st);
 cudaError_t launch_stream_reset(StreamState* state, uint32_t* rec, uint32_t rec_words, cudaStream_t st);
 cudaError_t launch_gather(const uint8_t* frames, uint32_t n_frames, uint64_t frame_bytes, const uint32_t* idx, uint32_t m,
-                          uint8_t* out, uint32_t* err, cudaStream_t st);
+                          uint8_t* out, uint32_t* err, bool host_src, cudaStream_t st);
 
 }  // namespace cofie

@@ -184,7 +184,9 @@ __global__ void stream_reset_kernel(StreamState* __restrict__ state, uint32_t* _
   if (threadIdx.x == 0) *state = StreamState{0ull, 0u, 0u, 0ull};
 }
 
-template <bool kVec>
+// kHostSrc: the frames are pinned host memory read through the device's
+// mapping of it (plain loads; the read-only path is kept for device frames).
+template <bool kVec, bool kHostSrc>
 __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const uint8_t* __restrict__ frames, uint32_t n_frames,
                                                                 uint64_t frame_bytes, const uint32_t* __restrict__ idx,
                                                                 uint32_t m, uint8_t* __restrict__ out,
@@ -206,7 +208,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const uint8_t* _
 #pragma unroll
       for (uint32_t u = 0; u < kGatherVecPerThread; ++u) {
         const uint64_t i = i0 + u * kGatherThreads;
-        if (i < n16) v[u] = __ldg(s4 + i);
+        if (i < n16) v[u] = kHostSrc ? s4[i] : __ldg(s4 + i);
       }
 #pragma unroll
       for (uint32_t u = 0; u < kGatherVecPerThread; ++u) {
@@ -242,18 +244,21 @@ cudaError_t launch_stream_reset(StreamState* state, uint32_t* rec, uint32_t rec_
 }
 
 cudaError_t launch_gather(const uint8_t* frames, uint32_t n_frames, uint64_t frame_bytes, const uint32_t* idx, uint32_t m,
-                          uint8_t* out, uint32_t* err, cudaStream_t st) {
+                          uint8_t* out, uint32_t* err, bool host_src, cudaStream_t st) {
   const bool vec = frame_bytes % 16 == 0 && reinterpret_cast<uintptr_t>(frames) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(out) % 16 == 0;
   const uint32_t gy = m < 65535u ? m : 65535u;
   if (vec) {
     const uint64_t per_block = static_cast<uint64_t>(kGatherThreads) * kGatherVecPerThread;
     dim3 grid(static_cast<uint32_t>((frame_bytes / 16 + per_block - 1) / per_block), gy);
-    gather_kernel<true><<<grid, kGatherThreads, 0, st>>>(frames, n_frames, frame_bytes, idx, m, out, err);
+    if (host_src)
+      gather_kernel<true, true><<<grid, kGatherThreads, 0, st>>>(frames, n_frames, frame_bytes, idx, m, out, err);
+    else
+      gather_kernel<true, false><<<grid, kGatherThreads, 0, st>>>(frames, n_frames, frame_bytes, idx, m, out, err);
   } else {
     const uint64_t want = (frame_bytes + kGatherThreads - 1) / kGatherThreads;
     dim3 grid(static_cast<uint32_t>(want < 1024 ? want : 1024), gy);
-    gather_kernel<false><<<grid, kGatherThreads, 0, st>>>(frames, n_frames, frame_bytes, idx, m, out, err);
+    gather_kernel<false, false><<<grid, kGatherThreads, 0, st>>>(frames, n_frames, frame_bytes, idx, m, out, err);
   }
   return cudaGetLastError();
 }

@@ -81,3 +81,32 @@ def test_gather_rejects_bad_index_without_reading_it():
     assert e.value.code == _abi.EDEVICE
     assert torch.equal(out[[0, 1, 3]], dev[[0, 3, 9]]) and int(out[2].sum()) == 0
     f.status()  # the error word was cleared; the handle keeps working
+
+
+@pytest.mark.parametrize("w,h", [(160, 96), (17, 13)])
+def test_gather_from_pinned_host_frames(w, h):
+    """Frames pushed from pinned host memory and gathered from it (the kernel
+    reads the host frames through the device's mapping): the same bytes as
+    indexing the frames on the host; pageable host frames are refused."""
+    from paper_2609_03675_gb300 import NGFFError, _abi
+    spec = synth.medium(seed=33).with_(width=w, height=h, frames=150, mean_scene_len=10)
+    fr = synth.generate(spec)
+    pinned = torch.from_numpy(fr).pin_memory()
+    f = _ngff(w, h, tau=0.05, m_min=4)
+    f.push(pinned)
+    idx = f.candidates(0)
+    out = f.gather(pinned, idx)
+    torch.cuda.synchronize()
+    f.status()
+    _, _, ko = O.load().run(fr, O.Params(w, h, tau=0.05))
+    want_idx = O.load().candidates(ko, 4)
+    assert np.array_equal(idx.cpu().numpy().astype(np.uint32), want_idx)
+    assert np.array_equal(out.cpu().numpy(), fr[want_idx])
+    # a frame-offset view of the pinned buffer (16-byte aligned only when the frame size is)
+    out2 = f.gather(pinned[1:], idx[idx < 149])
+    torch.cuda.synchronize()
+    f.status()
+    assert np.array_equal(out2.cpu().numpy(), fr[1:][want_idx[want_idx < 149]])
+    with pytest.raises(NGFFError) as e:
+        f.gather(torch.from_numpy(fr), idx)  # pageable host memory
+    assert e.value.code == _abi.EINVAL and "pinned host memory" in str(e.value)
