@@ -740,12 +740,11 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
   bool host_frames = false, host_out = false;
   MemKind kf[COFIE_NGFF_MAX_BATCH], ks[COFIE_NGFF_MAX_BATCH], kk[COFIE_NGFF_MAX_BATCH];
   uint64_t stage_off[COFIE_NGFF_MAX_BATCH];
-  std::vector<uint8_t> used(h->p.max_streams, 0);
   for (uint32_t i = 0; i < nd; ++i) {
     const cofie_ngff_push_desc& d = desc[i];
     if (d.stream >= h->p.max_streams) return h->fail(COFIE_EINVAL, "stream index out of range");
-    if (used[d.stream]) return h->fail(COFIE_EINVAL, "a stream appears twice in one batch");
-    used[d.stream] = 1;
+    for (uint32_t j = 0; j < i; ++j)  // at most 64 descriptors: no table the size of max_streams
+      if (desc[j].stream == d.stream) return h->fail(COFIE_EINVAL, "a stream appears twice in one batch");
     kf[i] = ks[i] = kk[i] = kNull;
     stage_off[i] = 0;
     if (d.n > 0) {

@@ -196,6 +196,11 @@ def test_batch_with_host_frames_and_outputs():
     big[0].stream, big[0].n, big[0].frames = 0, 41, frames_pin[0].data_ptr()
     assert f._lib.cofie_ngff_push_batch(f._h, big, 1, None) == _abi.EINVAL
     assert b"staging" in f._lib.cofie_ngff_last_error(f._h)
+    twice = (_abi.PushDesc * 3)()
+    for i, st in enumerate((1, 3, 1)):
+        twice[i].stream, twice[i].n, twice[i].frames = st, 1, frames_dev[st].data_ptr()
+    assert f._lib.cofie_ngff_push_batch(f._h, twice, 3, None) == _abi.EINVAL
+    assert b"appears twice" in f._lib.cofie_ngff_last_error(f._h)
     f.close()
 
 
