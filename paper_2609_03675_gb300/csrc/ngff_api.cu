@@ -65,6 +65,7 @@ struct cofie_ngff {
   int bin_path = -1;  // kBinFast, kBinTwoStep, or -1 (generic kernel only)
   bool size_fast = false;
   int hist_grid = 0;
+  uint64_t generic_wave = 0;  // CTAs of the generic kernel resident at once (0: never chosen over K1)
   int cells_grid = 0;    // the TMA kernel's grid for the spatial signals (0: not usable)
   unsigned long long x_tau = 0, x_cut = 0, x_grad = 0;  // integer forms of the fp32 decisions
   uint32_t m_gpr = 0, m_h = 0, m_gw = 0;  // its multiply-high divisors (16-pixel groups per row, height, grid columns)
@@ -262,6 +263,18 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
     cudaError_t e = launch_cells_fast(segs, ha, h->lc, dhash ? h->d_cells : h->d_hist, h->d_err, grid, st, pdl);
     if (e == cudaSuccess && dhash) e = launch_dhash_finish(h->d_cells, segs.rows, h->fa, h->d_hist, st, true);
     return e;
+  }
+  // A launch whose generic grid fills the GPU in one wave of resident CTAs
+  // (at least two per SM) runs the generic kernel: its CTAs start as SMs free
+  // and need no ring to fill, which K1's persistent CTAs, each with a fixed
+  // share of the chunks, pay on launches of that size (a batched call of 32
+  // streams of 640x360: 23.2 against 21.0 us). Smaller launches keep K1, whose
+  // CTAs are scheduled while the kernel before it runs; larger ones too, where
+  // the generic grid would end in a partial wave.
+  if (fast) {
+    const uint64_t gen_ctas = static_cast<uint64_t>(hist_generic_slices(h->npix)) * segs.rows;
+    if (gen_ctas >= 2ull * h->num_sms && gen_ctas <= h->generic_wave)
+      return launch_hist_generic(segs, ha, h->lc, h->bin_path, h->d_hist, st);
   }
   if (fast) {
     const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;
@@ -684,6 +697,9 @@ int cofie_ngff_create(const cofie_ngff_params* p, cofie_ngff_t** out) {
     const int per_sm = hist_blocks_per_sm(h->bin_path, p->bins);
     if (per_sm <= 0) e = cudaGetLastError() != cudaSuccess ? cudaErrorInvalidConfiguration : cudaErrorInvalidValue;
     h->hist_grid = h->num_sms * (per_sm > 0 ? per_sm : 1);
+    const int gen_per_sm = hist_generic_blocks_per_sm(h->bin_path, p->bins);
+    if (gen_per_sm < 0) cudaGetLastError();
+    h->generic_wave = gen_per_sm > 0 ? static_cast<uint64_t>(h->num_sms) * gen_per_sm : 0;
   }
   if (p->signal == COFIE_SIGNAL_LOWRES || p->signal == COFIE_SIGNAL_DHASH) {
     const uint32_t gpr = p->width / 16, gw = h->fa.grid_w, gh = h->fa.grid_h;

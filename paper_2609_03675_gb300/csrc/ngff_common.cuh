@@ -226,6 +226,9 @@ cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const Luma
                              uint32_t* hist, uint32_t* err, int grid, cudaStream_t st, bool pdl = false);
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
                                 uint32_t* hist, cudaStream_t st);
+// the generic kernel's CTAs per frame, and its resident CTAs per SM (-1 on error)
+uint32_t hist_generic_slices(uint32_t npix);
+int hist_generic_blocks_per_sm(int bin_path, uint32_t bins);
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
                           const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl = false);
 cudaError_t launch_scan(const SegTable& segs, const SelectArgs& a, const uint32_t* l1, const uint32_t* mask,

@@ -484,10 +484,26 @@ cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const Luma
   return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
+uint32_t hist_generic_slices(uint32_t npix) {
+  const uint32_t groups = npix / 16;  // at least the interior's groups, whatever the alignment
+  return groups ? (groups + kGenericGroupsPerCta - 1) / kGenericGroupsPerCta : 1;
+}
+
+int hist_generic_blocks_per_sm(int bin_path, uint32_t bins) {
+  int n = 0;
+  const size_t smem = static_cast<size_t>(bins) * 32 * 4;
+  const cudaError_t e =
+      bin_path == kBinFast
+          ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, hist_generic_kernel<kBinFast>, kGenericThreads, smem)
+      : bin_path == kBinTwoStep
+          ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, hist_generic_kernel<kBinTwoStep>, kGenericThreads, smem)
+          : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, hist_generic_kernel<kGenericDiv>, kGenericThreads, smem);
+  return e == cudaSuccess ? n : -1;
+}
+
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
                                 uint32_t* hist, cudaStream_t st) {
-  const uint32_t groups = a.npix / 16;  // at least the interior's groups, whatever the alignment
-  dim3 grid(groups ? (groups + kGenericGroupsPerCta - 1) / kGenericGroupsPerCta : 1, segs.rows);
+  dim3 grid(hist_generic_slices(a.npix), segs.rows);
   const size_t smem = static_cast<size_t>(lc.bins) * 32 * 4;
   if (bin_path == kBinFast)
     hist_generic_kernel<kBinFast><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
