@@ -265,15 +265,16 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
     return e;
   }
   // A launch whose generic grid fills the GPU in one wave of resident CTAs
-  // (at least two per SM) runs the generic kernel: its CTAs start as SMs free
-  // and need no ring to fill, which K1's persistent CTAs, each with a fixed
-  // share of the chunks, pay on launches of that size (a batched call of 32
-  // streams of 640x360: 23.2 against 21.0 us). Smaller launches keep K1, whose
-  // CTAs are scheduled while the kernel before it runs; larger ones too, where
-  // the generic grid would end in a partial wave.
+  // (at least two per SM, and at most an eighth of a second wave) runs the
+  // generic kernel: its CTAs start as SMs free and need no ring to fill,
+  // which K1's persistent CTAs, each with a fixed share of the chunks, pay on
+  // launches of that size (a batched call of 32 streams of 640x360: 23.2
+  // against 20.8 us). Smaller launches keep K1, whose CTAs are scheduled
+  // while the kernel before it runs; larger ones too, where the generic grid
+  // would end in a larger partial wave (a quarter of a wave already loses 6 %).
   if (fast) {
     const uint64_t gen_ctas = static_cast<uint64_t>(hist_generic_slices(h->npix)) * segs.rows;
-    if (gen_ctas >= 2ull * h->num_sms && gen_ctas <= h->generic_wave)
+    if (gen_ctas >= 2ull * h->num_sms && gen_ctas <= h->generic_wave + h->generic_wave / 8)
       return launch_hist_generic(segs, ha, h->lc, h->bin_path, h->d_hist, st);
   }
   if (fast) {
