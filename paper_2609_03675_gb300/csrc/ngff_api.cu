@@ -8,6 +8,9 @@
 // overlapping the copy of piece i+1 with the kernels of piece i. Outputs in
 // host memory are written to device scratch and copied back on the caller's
 // stream.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <algorithm>
 #include <cstddef>
 #include <cstdio>
@@ -136,6 +139,64 @@ MemKind classify(const void* ptr, int* dev_out = nullptr) {
     default:
       return kHostPageable;
   }
+}
+
+// The allocation a pointer was last found in, with its kind: a batched call
+// names three pointers per stream but usually few allocations (one frames
+// tensor per stream, one scores and one keep tensor for all of them), so
+// each descriptor field keeps the range of the last pointer it classified
+// and a pointer inside it needs no query.
+struct KindRange {
+  uintptr_t lo = 0, hi = 0;
+  MemKind kind = kNull;
+  int dev = -1;
+};
+
+PFN_cuPointerGetAttributes_v7000 pointer_attributes_fn() {
+  static PFN_cuPointerGetAttributes_v7000 fn = [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    return cudaGetDriverEntryPointByVersion("cuPointerGetAttributes", &p, 7000, cudaEnableDefault, &q) ==
+                       cudaSuccess &&
+                   q == cudaDriverEntryPointSuccess
+               ? reinterpret_cast<PFN_cuPointerGetAttributes_v7000>(p)
+               : nullptr;
+  }();
+  return fn;
+}
+
+// classify() with the range cache: one driver query gives the kind, the
+// device and the allocation's address range (a pointer the driver does not
+// know, such as pageable host memory, gets null attributes and is not cached).
+MemKind classify_in(const void* ptr, int* dev_out, KindRange* last) {
+  if (!ptr) return kNull;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(ptr);
+  if (a >= last->lo && a < last->hi) {
+    if (dev_out) *dev_out = last->dev;
+    return last->kind;
+  }
+  const PFN_cuPointerGetAttributes_v7000 fn = pointer_attributes_fn();
+  if (!fn) return classify(ptr, dev_out);
+  unsigned int type = 0, managed = 0;
+  int ordinal = -1;
+  CUdeviceptr start = 0;
+  size_t size = 0;
+  CUpointer_attribute attrs[5] = {CU_POINTER_ATTRIBUTE_MEMORY_TYPE, CU_POINTER_ATTRIBUTE_IS_MANAGED,
+                                  CU_POINTER_ATTRIBUTE_DEVICE_ORDINAL, CU_POINTER_ATTRIBUTE_RANGE_START_ADDR,
+                                  CU_POINTER_ATTRIBUTE_RANGE_SIZE};
+  void* data[5] = {&type, &managed, &ordinal, &start, &size};
+  if (fn(5, attrs, data, static_cast<CUdeviceptr>(a)) != CUDA_SUCCESS) return classify(ptr, dev_out);
+  const MemKind k = (managed || type == CU_MEMORYTYPE_DEVICE) ? kDevice
+                    : type == CU_MEMORYTYPE_HOST              ? kHostPinned
+                                                              : kHostPageable;
+  if (dev_out) *dev_out = ordinal;
+  if (k != kHostPageable && size > 0 && a >= start && a - start < size) {
+    last->lo = static_cast<uintptr_t>(start);
+    last->hi = static_cast<uintptr_t>(start) + size;
+    last->kind = k;
+    last->dev = ordinal;
+  }
+  return k;
 }
 
 // m = ceil(2^32 / d) with e = m d - 2^32 gives umulhi(n, m) = floor(n / d)
@@ -756,6 +817,7 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
   uint64_t rows = 0, staged_bytes = 0;
   bool host_frames = false, host_out = false;
   MemKind kf[COFIE_NGFF_MAX_BATCH], ks[COFIE_NGFF_MAX_BATCH], kk[COFIE_NGFF_MAX_BATCH];
+  KindRange rf, rs, rk;  // the allocations the last frames, scores and keep pointers were found in
   uint64_t stage_off[COFIE_NGFF_MAX_BATCH];
   for (uint32_t i = 0; i < nd; ++i) {
     const cofie_ngff_push_desc& d = desc[i];
@@ -766,12 +828,12 @@ int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uin
     stage_off[i] = 0;
     if (d.n > 0) {
       int fdev = -1;
-      kf[i] = d.frames ? classify(d.frames, &fdev) : kNull;
+      kf[i] = d.frames ? classify_in(d.frames, &fdev, &rf) : kNull;
       if (kf[i] == kNull || (kf[i] == kDevice && fdev != h->device))
         return h->fail(COFIE_EINVAL, "batched frames must be device memory on the handle's device, or host memory");
       int sdev = -1, kdev = -1;
-      ks[i] = classify(d.scores_out, &sdev);
-      kk[i] = classify(d.keep_out, &kdev);
+      ks[i] = classify_in(d.scores_out, &sdev, &rs);
+      kk[i] = classify_in(d.keep_out, &kdev, &rk);
       if ((ks[i] == kDevice && sdev != h->device) || (kk[i] == kDevice && kdev != h->device))
         return h->fail(COFIE_EINVAL, "batched outputs live on another device");
       if (kf[i] != kDevice) {  // staged back to back, each descriptor's frames from a 16-byte boundary
