@@ -233,8 +233,8 @@ int cofie_ngff_push_ex(cofie_ngff_t* h, uint32_t stream, const uint8_t* frames, 
 int cofie_ngff_push_batch(cofie_ngff_t* h, const cofie_ngff_push_desc* desc, uint32_t nd, void* cuda_stream);
 
 /*
- * Closes stream `stream` at the frames pushed so far (Sec. 3.2, "Gap-aware
- * frame retention": the safeguards that need the end of the prefix) and
+ * Closes stream `stream` at the frames pushed so far (Sec. 3.2, the
+ * retention safeguards that need the end of the prefix) and
  * writes its candidate set S_c as ascending frame indices. With T the number
  * of frames the stream has been pushed when the call runs on cuda_stream
  * (read on the device, so the call may be captured into a CUDA graph after
@@ -283,8 +283,8 @@ int cofie_ngff_candidates_from_keep(cofie_ngff_t* h, const uint8_t* keep, uint32
 
 /*
  * Copies the m frames idx[0..m) of `frames` back to back into `out`: the
- * frames S_c that go on to the vision encoder (Sec. 3.2, "only these m frames
- * are sent to the encoder").
+ * frames S_c that go on to the vision encoder (Sec. 3.2: the encoder
+ * sees the candidate frames and no others).
  *   frames   n_frames frames of 3 W H bytes: device memory, or pinned host
  *            memory (read by the kernel over the host link through the
  *            device's mapping of it; pageable host memory is COFIE_EINVAL).

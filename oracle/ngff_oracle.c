@@ -7,7 +7,7 @@
  * the library never calls it and shares no code, header or table with it.
  *
  * What it computes, step by step in the paper's order:
- *   1. Grayscale (Sec. 3.2, "Lightweight histogram-based novelty"): the paper
+ *   1. Grayscale (Sec. 3.2, the histogram novelty paragraph): the paper
  *      does not give the conversion. Reading used here: ITU-R BT.601 luma
  *      with integer weights and round-half-up,
  *          Y = floor((wR*R + wG*G + wB*B + floor(den/2)) / den),

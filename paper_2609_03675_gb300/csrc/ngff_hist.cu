@@ -1,5 +1,5 @@
-// K1: per-frame grayscale histograms (CoFiE Sec. 3.2 "Lightweight
-// histogram-based novelty"; B = 32 bins per App. A).
+// K1: per-frame grayscale histograms (CoFiE Sec. 3.2, the histogram
+// novelty paragraph; B = 32 bins per App. A).
 //
 // Per pixel: Y = floor((wR R + wG G + wB B + floor(den/2)) / den) (BT.601
 // reading), bin = floor(Y B / 256), count[bin] += 1. Integer arithmetic only,

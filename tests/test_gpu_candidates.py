@@ -1,6 +1,6 @@
 """Closing a stream through its retention record: cofie_ngff_candidates(h,
 stream, idx_out, cap, &m) after pushes, against the oracle's candidate set
-(last frame, M_min uniform fill; Sec. 3.2 "Gap-aware frame retention") of the
+(last frame, M_min uniform fill; the retention safeguards of Sec. 3.2) of the
 oracle's keep codes for the same prefix.
 
 The keep codes of a prefix are those of the whole stream cut at the prefix
