@@ -6,8 +6,11 @@
  * Usage: ngff_client IN OUT WIDTH HEIGHT FRAMES TAU L_MAX PIECE...
  * IN holds FRAMES * WIDTH * HEIGHT * 3 bytes; OUT receives FRAMES floats,
  * FRAMES keep bytes, then per piece: the prefix length T (uint32), |S_c|
- * (uint32) and |S_c| uint32 indices. Exit status 0 on success; a failing
- * call prints the library's message. */
+ * (uint32) and |S_c| uint32 indices. It then pushes the same frames as two
+ * streams of one handle through cofie_ngff_push_batch in the same pieces
+ * and checks that both equal the single-stream results (exit status 7 if
+ * not). Exit status 0 on success; a failing call prints the library's
+ * message. */
 #include <stdint.h>
 #include <stdio.h>
 #include <stdlib.h>
@@ -71,6 +74,42 @@ int main(int argc, char** argv) {
   }
   if (check(cofie_ngff_status(h, NULL), h, "cofie_ngff_status")) return 1;
   cofie_ngff_destroy(h);
+
+  /* The same frames as two streams of one handle through the batched call,
+   * in the same pieces, from pageable host memory into host outputs: each
+   * stream's scores and keep codes must equal the single-stream run's. */
+  p.max_streams = 2;
+  p.max_frames_per_push = 2 * (T ? T : 1);
+  cofie_ngff_t* hb = NULL;
+  if (check(cofie_ngff_create(&p, &hb), NULL, "cofie_ngff_create (batch)")) return 1;
+  float* bs = malloc(sizeof(float) * 2 * (T ? T : 1));
+  uint8_t* bk = malloc(2 * (T ? T : 1));
+  if (!bs || !bk) return 3;
+  off = 0;
+  for (int a = 8; a < argc && off < T; ++a) {
+    uint32_t n = (uint32_t)strtoul(argv[a], NULL, 10);
+    if (n > T - off) n = T - off;
+    cofie_ngff_push_desc d[2];
+    for (uint32_t s = 0; s < 2; ++s) {
+      d[s].stream = s;
+      d[s].n = n;
+      d[s].frames = frames + (size_t)off * frame_bytes;
+      d[s].scores_out = bs + (size_t)s * T + off;
+      d[s].keep_out = bk + (size_t)s * T + off;
+    }
+    if (check(cofie_ngff_push_batch(hb, d, 2, NULL), hb, "cofie_ngff_push_batch")) return 1;
+    off += n;
+  }
+  if (check(cofie_ngff_status(hb, NULL), hb, "cofie_ngff_status (batch)")) return 1;
+  cofie_ngff_destroy(hb);
+  for (uint32_t s = 0; s < 2; ++s)
+    for (uint32_t t = 0; t < T; ++t)
+      if (bk[(size_t)s * T + t] != keep[t] || bs[(size_t)s * T + t] != scores[t]) {
+        fprintf(stderr, "batched stream %u differs from the single-stream run at frame %u\n", s, t);
+        return 7;
+      }
+  free(bs);
+  free(bk);
 
   fseek(out, 0, SEEK_SET);
   fwrite(scores, sizeof(float), T, out);

@@ -2,7 +2,9 @@
 library only: no CUDA runtime, no Python) pushes seeded frames from pageable
 host memory in uneven pieces and closes the stream after each piece; its
 scores and keep codes must equal the oracle's, and each candidate set the
-oracle's candidate set of that prefix."""
+oracle's candidate set of that prefix. The client then pushes the same
+frames as two streams through the batched call (pageable host frames and
+outputs) and checks both against its single-stream results itself."""
 import os
 import shutil
 import subprocess
