@@ -66,6 +66,8 @@ def parse():
                     help="seconds the other streams' figures may take after the headline (a config that would start "
                          "past the budget is skipped and says so)")
     ap.add_argument("--no-parity", action="store_true", help="hd1080 line without the oracle parity block")
+    ap.add_argument("--serving-frames", type=int, default=0,
+                    help="frames per stream of the serving workload (0: all 1800; fewer for profiling captures)")
     ap.add_argument("--size", default="1920x1080",
                     help="frame size WxH of the hd1080 workload's stream (same recipe); a pixel count that is not a "
                          "multiple of 16 runs the generic histogram kernel")
@@ -721,6 +723,8 @@ def serving_figures(args, parity: bool = True):
     from paper_2609_03675_gb300 import NGFF
     S = synth.SERVING_STREAMS
     specs = [synth.serving_stream(s) for s in range(S)]
+    if getattr(args, "serving_frames", 0):
+        specs = [sp.with_(frames=min(sp.frames, args.serving_frames)) for sp in specs]
     T, W, H = specs[0].frames, specs[0].width, specs[0].height
     host = torch.empty((T, H, W, 3), dtype=torch.uint8, pin_memory=True)
     dev, want = [], []
@@ -841,7 +845,7 @@ def serving_figures(args, parity: bool = True):
            "how": f"the first {E} frames of every stream: pinned host frames in, pinned host scores and keep codes "
                   "out, through the same batched call"}
     del host_fr
-    line = {"workload": "serving: 32 streams x 1800 uint8 RGB frames of 640x360, U{1..8} frames per stream per "
+    line = {"workload": f"serving: 32 streams x {T} uint8 RGB frames of 640x360, U{{1..8}} frames per stream per "
                         "batched call, B=32, L_max=30, tau_h=0.30",
             "calls": len(plan), "frames": frames_total,
             "pipelined_frames_per_s": frames_total / el_pipe, "pipelined_ms_per_call": el_pipe / len(plan) * 1e3,
