@@ -36,6 +36,7 @@ thread_local std::string g_global_error;
 enum MemKind { kNull = 0, kDevice = 1, kHostPinned = 2, kHostPageable = 3 };
 
 constexpr uint64_t kDefaultStageBytes = 256ull << 20;
+constexpr uint32_t kSmallSliceGroups = 256;  // the generic kernel's slice for small launches (12 KiB of frame)
 constexpr uint32_t kDefaultRecordFrames = 1u << 20;  // frames per stream the retention record covers
 constexpr uint64_t kTimeoutNs = 2000000000ull;  // bounded device waits: 2 s
 constexpr size_t kMaxTimedEvents = 1u << 16;
@@ -330,13 +331,22 @@ cudaError_t launch_first_stage(cofie_ngff* h, const SegTable& segs, cudaStream_t
   // generic kernel: its CTAs start as SMs free and need no ring to fill,
   // which K1's persistent CTAs, each with a fixed share of the chunks, pay on
   // launches of that size (a batched call of 32 streams of 640x360: 23.2
-  // against 20.8 us). Smaller launches keep K1, whose CTAs are scheduled
-  // while the kernel before it runs; larger ones too, where the generic grid
-  // would end in a larger partial wave (a quarter of a wave already loses 6 %).
+  // against 20.8 us). Launches too small for that window with the default
+  // slices take slices of kSmallSliceGroups groups if those land in it, as a
+  // programmatic dependent of the kernel before them (8-frame 448x448 pushes:
+  // 7.27 against 6.56 us per push); a grid near one wave stays an ordinary
+  // launch, because CTAs made resident ahead of time keep SMs the previous
+  // kernel still holds (the serving call went from 21 to 27 us). Smaller
+  // launches keep K1, whose CTAs are scheduled while the kernel before it
+  // runs; larger ones too, where the generic grid would end in a larger
+  // partial wave (a quarter of a wave already loses 6 %).
   if (fast) {
+    const uint64_t lo = 2ull * h->num_sms, hi = h->generic_wave + h->generic_wave / 8;
     const uint64_t gen_ctas = static_cast<uint64_t>(hist_generic_slices(h->npix)) * segs.rows;
-    if (gen_ctas >= 2ull * h->num_sms && gen_ctas <= h->generic_wave + h->generic_wave / 8)
-      return launch_hist_generic(segs, ha, h->lc, h->bin_path, h->d_hist, st);
+    if (gen_ctas >= lo && gen_ctas <= hi) return launch_hist_generic(segs, ha, h->lc, h->bin_path, h->d_hist, st);
+    const uint64_t small_ctas = static_cast<uint64_t>(hist_generic_slices(h->npix, kSmallSliceGroups)) * segs.rows;
+    if (gen_ctas < lo && small_ctas >= lo && small_ctas <= hi)
+      return launch_hist_generic(segs, ha, h->lc, h->bin_path, h->d_hist, st, kSmallSliceGroups, pdl);
   }
   if (fast) {
     const uint64_t chunks = static_cast<uint64_t>(segs.rows) * ha.chunks_per_frame;

@@ -155,6 +155,7 @@ struct HistArgs {
   uint32_t gpr, m_gpr, m_h;
   uint32_t wide;  // every cell column is at least 16 pixels wide
   uint32_t m_gw;  // multiply-high constant for / grid_w (wide path)
+  uint32_t slice_groups;  // generic kernel only: 16-pixel groups per CTA
 };
 
 struct SelectArgs {
@@ -224,10 +225,13 @@ uint32_t hist_chunk_groups();
 size_t hist_smem_bytes(uint32_t bins);
 cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
                              uint32_t* hist, uint32_t* err, int grid, cudaStream_t st, bool pdl = false);
+// The generic kernel over CTAs of slice_groups 16-pixel groups (0: the
+// default 2048); with pdl a programmatic dependent of the kernel before it.
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
-                                uint32_t* hist, cudaStream_t st);
-// the generic kernel's CTAs per frame, and its resident CTAs per SM (-1 on error)
-uint32_t hist_generic_slices(uint32_t npix);
+                                uint32_t* hist, cudaStream_t st, uint32_t slice_groups = 0, bool pdl = false);
+// the generic kernel's CTAs per frame (slices of slice_groups groups, 0: the
+// default), and its resident CTAs per SM (-1 on error)
+uint32_t hist_generic_slices(uint32_t npix, uint32_t slice_groups = 0);
 int hist_generic_blocks_per_sm(int bin_path, uint32_t bins);
 cudaError_t launch_window(const SegTable& segs, const SelectArgs& a, const uint32_t* hist, const uint32_t* ring,
                           const StreamState* state, uint32_t* l1, uint32_t* mask, cudaStream_t st, bool pdl = false);

@@ -357,7 +357,7 @@ __global__ void __launch_bounds__(Shape<kBin>::threads) hist_fast_kernel(SegTabl
 // go to lane-private shared counters cnt[bin][lane] (bank = lane), folded
 // into the frame's row with one global atomic per bin per CTA.
 constexpr int kGenericThreads = 256;
-constexpr uint32_t kGenericGroupsPerCta = 2048;  // 32768 pixels per CTA
+constexpr uint32_t kGenericGroupsPerCta = 2048;  // 32768 pixels per CTA, unless the launch asks for fewer
 constexpr int kGenericDiv = 3;                   // no verified multiply-high: Y = v / den
 
 template <int kBin>
@@ -376,6 +376,11 @@ __global__ void __launch_bounds__(kGenericThreads) hist_generic_kernel(SegTable 
   while (seg + 1 < segs.count && row >= segs.s[seg + 1].row0) ++seg;
   const uint8_t* frame = segs.s[seg].frames + static_cast<uint64_t>(row - segs.s[seg].row0) * a.frame_bytes;
   for (uint32_t i = tid; i < L.bins * 32; i += kGenericThreads) gcnt[i] = 0;
+  // Launched as a programmatic dependent of the kernel before it (small
+  // launches), this CTA has set up while that kernel ran; no frame is read
+  // and no row written until that kernel has completed and its memory is
+  // visible. A no-op for an ordinary launch.
+  pdl_wait();
   __syncthreads();
   const uint32_t cnt_lane = static_cast<uint32_t>(__cvta_generic_to_shared(gcnt)) + lane * 4;
   const uint32_t npix = a.npix;
@@ -383,7 +388,8 @@ __global__ void __launch_bounds__(kGenericThreads) hist_generic_kernel(SegTable 
   const uint32_t mis = static_cast<uint32_t>(reinterpret_cast<uintptr_t>(frame) & 15u);
   const uint32_t p_a = min(((16u - mis) * 11u) & 15u, npix);
   const uint32_t G = (npix - p_a) / 16;
-  const uint32_t g0 = blockIdx.x * kGenericGroupsPerCta, g1 = min(g0 + kGenericGroupsPerCta, G);
+  const uint32_t spc = a.slice_groups;
+  const uint32_t g0 = blockIdx.x * spc, g1 = min(g0 + spc, G);
   const uint8_t* base = frame + 3ull * p_a;
 #pragma unroll 2
   for (uint32_t g = g0 + tid; g < g1; g += kGenericThreads) {
@@ -484,9 +490,10 @@ cudaError_t launch_hist_fast(const SegTable& segs, const HistArgs& a, const Luma
   return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
-uint32_t hist_generic_slices(uint32_t npix) {
+uint32_t hist_generic_slices(uint32_t npix, uint32_t slice_groups) {
+  const uint32_t spc = slice_groups ? slice_groups : kGenericGroupsPerCta;
   const uint32_t groups = npix / 16;  // at least the interior's groups, whatever the alignment
-  return groups ? (groups + kGenericGroupsPerCta - 1) / kGenericGroupsPerCta : 1;
+  return groups ? (groups + spc - 1) / spc : 1;
 }
 
 int hist_generic_blocks_per_sm(int bin_path, uint32_t bins) {
@@ -502,16 +509,16 @@ int hist_generic_blocks_per_sm(int bin_path, uint32_t bins) {
 }
 
 cudaError_t launch_hist_generic(const SegTable& segs, const HistArgs& a, const LumaConsts& lc, int bin_path,
-                                uint32_t* hist, cudaStream_t st) {
-  dim3 grid(hist_generic_slices(a.npix), segs.rows);
+                                uint32_t* hist, cudaStream_t st, uint32_t slice_groups, bool pdl) {
+  HistArgs b = a;
+  b.slice_groups = slice_groups ? slice_groups : kGenericGroupsPerCta;
+  const dim3 grid(hist_generic_slices(a.npix, b.slice_groups), segs.rows);
   const size_t smem = static_cast<size_t>(lc.bins) * 32 * 4;
-  if (bin_path == kBinFast)
-    hist_generic_kernel<kBinFast><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
-  else if (bin_path == kBinTwoStep)
-    hist_generic_kernel<kBinTwoStep><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
-  else
-    hist_generic_kernel<kGenericDiv><<<grid, kGenericThreads, smem, st>>>(segs, a, lc, hist);
-  return cudaGetLastError();
+  const auto kernel = bin_path == kBinFast      ? hist_generic_kernel<kBinFast>
+                      : bin_path == kBinTwoStep ? hist_generic_kernel<kBinTwoStep>
+                                                : hist_generic_kernel<kGenericDiv>;
+  const cudaError_t e = launch_dependent(pdl, kernel, grid, dim3(kGenericThreads), smem, st, segs, b, lc, hist);
+  return e == cudaSuccess ? cudaGetLastError() : e;
 }
 
 uint32_t take_bounds_errors_hist() { return take_local_bounds_errors(); }
