@@ -413,7 +413,7 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
   constexpr uint32_t kWarps = kWalkThreads / 32;
   extern __shared__ __align__(16) uint32_t wsm[];
   __shared__ unsigned long long s_t0, s_acc;
-  __shared__ uint32_t s_g;
+  __shared__ uint32_t s_g, s_slot0;
   pdl_trigger();  // the next push's first-stage kernel may be scheduled; it waits for this grid before its work
   pdl_wait();     // every device read follows: the histograms before it, and the state the last push left
   const Segment sg = segs.s[blockIdx.x];
@@ -431,6 +431,7 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
     s_t0 = state[stream].t;
     s_acc = state[stream].acc;
     s_g = state[stream].g;
+    s_slot0 = static_cast<uint32_t>(s_t0 % L);  // the ring slot of the push's first frame (one 64-bit division)
   }
   if (kStaged) {
     if (kVec4) {
@@ -445,6 +446,7 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
   }
   __syncthreads();
   const unsigned long long t0 = s_t0;
+  const int slot0 = static_cast<int>(s_slot0), Li = static_cast<int>(L);
   const uint32_t nq = B / 4, rot = kStaged && kVec4 ? lane % max(nq, 1u) : 0u;
 
   // 1. distances and keep bits
@@ -458,7 +460,11 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
       const uint32_t* src = ct;
       if (valid) {
         if (k <= j) src = ct - static_cast<uint64_t>(k) * B;
-        else src = (kStaged ? srows : ring_s) + ((t - k) % L) * B;  // ring slot of frame t - k
+        else {  // ring slot of frame t - k: (slot0 + j - k) mod L, with |j - k| < 2^7
+          int slot = (slot0 + static_cast<int>(j) - static_cast<int>(k)) % Li;
+          if (slot < 0) slot += Li;
+          src = (kStaged ? srows : ring_s) + static_cast<uint32_t>(slot) * B;
+        }
       }
       uint32_t d = 0;
       if (kVec4) {
@@ -547,7 +553,7 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
   uint32_t* ring_w = ring + static_cast<uint64_t>(stream) * L * B;
   for (uint32_t i = tid; i < keep_n * B; i += kWalkThreads) {
     const uint32_t jj = n - keep_n + i / B, b = i % B;
-    ring_w[((t0 + jj) % L) * B + b] = kStaged ? srows[(L + jj) * B + b] : hist_s[static_cast<uint64_t>(jj) * B + b];
+    ring_w[((s_slot0 + jj) % L) * B + b] = kStaged ? srows[(L + jj) * B + b] : hist_s[static_cast<uint64_t>(jj) * B + b];
   }
   if (tid == 0) {
     state[stream].t = t0 + n;
