@@ -487,7 +487,8 @@ __global__ void __launch_bounds__(kWalkThreads) select_walk_kernel(SegTable segs
       if (w == 0) l_adj = __shfl_sync(0xffffffffu, d, 0);  // lag 1
       if (k <= L) sl1[j * L + k - 1] = d;
       bool keep = false;
-      if (k <= L) keep = __fdiv_rn(static_cast<float>(max(l_adj, d)), a.two_n) >= a.tau || k >= L;
+      // fp32(max) / 2N >= tau exactly when max >= x_tau (the smallest such numerator)
+      if (k <= L) keep = max(l_adj, d) >= a.x_tau || k >= L;
       const uint32_t m = __ballot_sync(0xffffffffu, keep);
       if (lane == 0) smask[j * W + w] = m;
     }
